@@ -1,0 +1,452 @@
+"""Benchmark of the CCI-sparse forward layer (arXiv 1910.11971) on GB300.
+
+Default workload: the ResNet 1x1 bottleneck as a CCI product, fp32:
+N = 32*56*56 = 100352 columns, 256 -> 1024 channels, G = 8, K = 2 (75% sparse),
+W ~ N(0, 2/256), X = ReLU(N(0, 1)), seeded synthetic data.
+
+One step = the whole hot path on one batch: cci_pack of the dense weights
+(per-group top-K) + cci_linear (scatter-accumulate), inputs resident in HBM.
+The metric is nonzero TFLOP/s (2*N*R*Cout*K/G per step); the roofline is the
+CUDA-core FMA peak (the path is bound by fp32 FMA, not HBM).  L2 (129 MB) is
+flushed between timed steps by writing a 256 MB buffer outside the timed events.
+
+``--impl reference`` times the fp64 CPU oracle on a bounded sample of the same
+workload instead (the reported CPU baseline).
+
+Prints one JSON line (rank 0).  Multi-GPU (torchrun): every rank runs its own
+batch (weak scaling, no collective on the data path); the step time is the max
+over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_1910_11971_gb300 import workloads as wl  # noqa: E402
+
+METRIC = "CCI layer nonzero TFLOP/s & fraction of roofline vs K/G; speedup over dense"
+UNIT = "TFLOP/s"
+MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
+# CUDA-core fp32 FMA peak from unit counts and clock: 152 SMs x 128 FP32 lanes
+# x 2 flop x 2.070 GHz (maximum SM clock); the FFMA path is ALU-bound.
+N_SM, FMA_LANES, SM_MAX_GHZ = 152, 128, 2.070
+ALU_PEAK_TFLOPS = N_SM * FMA_LANES * 2 * SM_MAX_GHZ / 1e3
+L2_FLUSH_BYTES = 256 << 20
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--extras", type=int, default=1, help="also measure the sweep / conv workloads")
+    ap.add_argument("--cpu-sample-seconds", type=float, default=12.0)
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# distributed plumbing (weak scaling: no collective on the data path)
+# ---------------------------------------------------------------------------
+def dist_init(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# the reported CPU baseline: the fp64 oracle on a bounded sample
+# ---------------------------------------------------------------------------
+def oracle_rate(case: wl.LinearCase, seconds: float):
+    """Nonzero TFLOP/s of the oracle on the first `rows` columns of the workload,
+    with `rows` grown until one call takes about `seconds`."""
+    import numpy as np
+
+    import oracle
+    X, W = wl.linear_inputs(case, N=min(case.N, 65536))
+    Xf = X.to(torch.float64).numpy()
+    v, i = oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
+    Wd, mask = oracle.decompress(v, i, case.Cout, case.G)
+    rows = 64
+    while True:
+        t0 = time.perf_counter()
+        oracle.linear(Xf[:rows], Wd, mask)
+        dt = time.perf_counter() - t0
+        if dt >= seconds or rows >= Xf.shape[0]:
+            break
+        rows = min(Xf.shape[0], int(rows * max(2.0, 1.2 * seconds / max(dt, 1e-3))))
+    flops = 2.0 * rows * case.R * case.Cout * case.K / case.G
+    return flops / dt / 1e12, rows, dt, oracle.threads()
+
+
+def run_reference(args, rank, world):
+    case = wl.BOTTLENECK_1X1
+    if rank != 0:
+        return 0
+    import numpy as np  # noqa: F401
+
+    import oracle
+    X, W = wl.linear_inputs(case, N=4096)
+    Xf = X.to(torch.float64).numpy()
+    # size one step's sample so that warmup + steps stay within a few minutes
+    v, i = oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
+    Wd, mask = oracle.decompress(v, i, case.Cout, case.G)
+    rows = 256
+    t0 = time.perf_counter()
+    oracle.linear(Xf[:rows], Wd, mask)
+    dt = time.perf_counter() - t0
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    rows = max(16, min(Xf.shape[0], int(rows * budget / max(dt, 1e-4))))
+    for _ in range(args.warmup):
+        oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
+        oracle.linear(Xf[:rows], Wd, mask)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        vv, ii = oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
+        Wd, mask = oracle.decompress(vv, ii, case.Cout, case.G)
+        oracle.linear(Xf[:rows], Wd, mask)
+    dt = (time.perf_counter() - t0) / args.steps
+    flops = 2.0 * rows * case.R * case.Cout * case.K / case.G
+    value = flops / dt / 1e12
+    sample = (f"{rows} of {case.N} columns per step (pack + decompress + dense-mask product in "
+              f"fp64), {case.Cin}->{case.Cout}, G={case.G}, K={case.K}")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": config_of(case, extra={"sample_columns": rows}),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_of(case, extra=None):
+    c = {"workload": case.name, "N": case.N, "Cin": case.Cin, "Cout": case.Cout, "G": case.G,
+         "K": case.K, "sparsity": 1 - case.K / case.G, "dtype_in": case.dtype,
+         "l2": "flushed between timed steps (256 MB write outside the timed events)",
+         "parallelism": "one independent batch per GPU"}
+    if extra:
+        c.update(extra)
+    return c
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_1910_11971_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on
+    the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    r = rec.get(kernel)
+    if not r or r.get("source_hash") != kernel_source_hash():
+        return None
+    return r.get("dram_bytes_per_launch")
+
+
+def time_device(fn, reps, flush, stream):
+    """Per-rep CUDA-event durations (ms) on `stream`, L2 flushed before each rep."""
+    out = []
+    for _ in range(reps):
+        flush()
+        s = torch.cuda.Event(enable_timing=True)
+        e = torch.cuda.Event(enable_timing=True)
+        s.record(stream)
+        fn()
+        e.record(stream)
+        e.synchronize()
+        out.append(s.elapsed_time(e))
+    return out
+
+
+def run_ours(args, rank, world, local):
+    import paper_1910_11971_gb300 as cci
+    from paper_1910_11971_gb300 import build as cci_build
+
+    cci_build.build()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+    torch.backends.cuda.matmul.allow_tf32 = False
+    torch.backends.cudnn.allow_tf32 = False
+    case = wl.BOTTLENECK_1X1
+    X, W = wl.linear_inputs(case, device="cpu")
+    X_host = X.pin_memory()
+    W_host = W.pin_memory()
+    Xd, Wd = X.to(dev), W.to(dev)
+    values = torch.empty((case.Cout // case.G, case.R, case.K), dtype=Xd.dtype, device=dev)
+    idx = torch.empty((case.Cout // case.G, case.R, case.K), dtype=torch.uint8, device=dev)
+    Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
+    status = cci.new_status(dev)
+    flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def flush():
+        flush_buf.fill_(1.0)
+
+    def step():
+        cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
+        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    assert cci.read_status(status) == 0
+
+    # ---- timed region: K steps, per-step events (pack | linear), L2 flushed between ----
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clk:
+        t_wall0 = time.perf_counter()
+        for k in range(args.steps):
+            flush()
+            a, b, c = ev[k]
+            a.record(stream)
+            cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
+            b.record(stream)
+            cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status)
+            c.record(stream)
+        torch.cuda.synchronize(dev)
+        t_wall = time.perf_counter() - t_wall0
+    barrier(world)
+    step_ms = [a.elapsed_time(c) for a, b, c in ev]
+    lin_ms = [b.elapsed_time(c) for a, b, c in ev]
+    pack_ms = [a.elapsed_time(b) for a, b, c in ev]
+    assert cci.read_status(status) == 0
+    ms_step = max_over_ranks(sum(step_ms) / len(step_ms), world, dev)
+    nzf = case.nz_flops()
+    value = world * nzf / (ms_step * 1e-3) / 1e12
+    lin_avg = statistics.mean(lin_ms)
+    kname = cci.kernel_name(torch.float32, case.Cin, case.R, case.Cout, case.G, case.K)
+    achieved = nzf / (lin_avg * 1e-3) / 1e12
+    roofline = {"bound": "alu", "achieved": achieved, "peak": ALU_PEAK_TFLOPS, "unit": "TFLOP/s",
+                "frac": achieved / ALU_PEAK_TFLOPS, "traffic": measured_traffic(kname),
+                "kernel": kname,
+                "peak_source": "derived: 152 SMs x 128 FP32 FMA lanes x 2 flop x 2.070 GHz max clock",
+                "algorithmic_flops_per_launch": nzf,
+                "hbm_bytes_per_launch": case.N * case.Cin * 4 + case.N * case.Cout * 4
+                + (case.Cout // case.G) * case.R * case.K * 5}
+
+    # ---- end to end through the public API: host X,W -> device, step, Y -> host ----
+    Y_host = torch.empty((case.N, case.Cout), dtype=torch.float32).pin_memory()
+
+    def e2e_step():
+        Xd.copy_(X_host, non_blocking=True)
+        Wd.copy_(W_host, non_blocking=True)
+        cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
+        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status)
+        Y_host.copy_(Y, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize(dev)
+    e2e_ms = statistics.mean(time_device(e2e_step, max(3, args.steps // 4), flush, stream))
+    e2e_ms = max_over_ranks(e2e_ms, world, dev)
+    e2e = {"value": world * nzf / (e2e_ms * 1e-3) / 1e12, "unit": UNIT,
+           "h2d_bytes_per_step": X_host.numel() * 4 + W_host.numel() * 4,
+           "d2h_bytes_per_step": Y_host.numel() * 4, "ms_per_step": e2e_ms}
+
+    # ---- dense reference line: cuBLAS fp32 (TF32 off) on the masked dense weights ----
+    Wm = torch.zeros_like(Wd)
+    Wm.view(case.Cout // case.G, case.G, case.R).scatter_(
+        1, idx.permute(0, 2, 1).long(), values.permute(0, 2, 1))
+    dense_ms = statistics.median(time_device(lambda: torch.matmul(Xd, Wm.t()), 10, flush, stream))
+    dense = {"kernel": "torch.matmul fp32 (cuBLAS, TF32 off)", "ms": dense_ms,
+             "dense_tflops": case.dense_flops() / (dense_ms * 1e-3) / 1e12,
+             "speedup_cci_over_dense": dense_ms / lin_avg}
+
+    extras = {}
+    if args.extras and rank == 0:
+        extras = run_extras(cci, dev, stream, flush)
+
+    cpu = None
+    if rank == 0 and world == 1:
+        rate, rows, dt, cores = oracle_rate(case, args.cpu_sample_seconds)
+        cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"first {rows} of {case.N} columns, one fp64 dense-mask product "
+                         f"({dt:.1f} s), nonzero flops counted"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": config_of(case), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": 2 * args.steps, "clocks": clk.summary(),
+            "breakdown_ms": {"pack": statistics.mean(pack_ms), "linear": lin_avg,
+                             "wall_per_step_incl_flush": t_wall * 1e3 / args.steps},
+            "dense_reference": dense, **extras,
+        }
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_extras(cci, dev, stream, flush):
+    """K/G sweep (4096 -> 4096, N = 8192, bf16) and the 3x3 conv workload, each
+    against its dense cuBLAS / cuDNN line on the masked dense weights."""
+    out = {"sweep_4096": [], "conv3x3_28": None}
+    for G, K in wl.SWEEP_POINTS:
+        case = wl.sweep_case(G, K)
+        X, W = wl.linear_inputs(case, device=str(dev))
+        v, i = cci.pack(W, G, K)
+        Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
+        fn = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y)  # noqa: E731
+        fn()
+        ms = statistics.median(time_device(fn, 10, flush, stream))
+        Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
+        Wm.view(case.Cout // G, G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
+        dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), 10, flush, stream))
+        tf = case.nz_flops() / (ms * 1e-3) / 1e12
+        out["sweep_4096"].append({"G": G, "K": K, "K_over_G": K / G, "ms": ms, "nz_tflops": tf,
+                                  "dense_equiv_tflops": case.dense_flops() / (ms * 1e-3) / 1e12,
+                                  "roofline_frac": tf / ALU_PEAK_TFLOPS,
+                                  "dense_bf16_ms": dms, "speedup_over_dense": dms / ms,
+                                  "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R,
+                                                            case.Cout, G, K)})
+        del X, W, v, i, Y, Wm
+    case = wl.CONV3X3_28
+    X, W = wl.conv_inputs(case, device=str(dev))
+    v, i = cci.pack(W, case.G, case.K)
+    fn = lambda: cci.conv2d(X, v, i, case.Cout, case.G, case.K, 3, 3, (1, 1), (1, 1))  # noqa: E731
+    fn()
+    ms = statistics.median(time_device(fn, 10, flush, stream))
+    Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
+    Wm.view(case.Cout // case.G, case.G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
+    w4 = Wm.view(case.Cout, 3, 3, case.Cin).permute(0, 3, 1, 2).contiguous(memory_format=torch.channels_last)
+    x4 = X.permute(0, 3, 1, 2)  # NHWC memory, NCHW view = channels_last
+    dms = statistics.median(time_device(
+        lambda: torch.nn.functional.conv2d(x4, w4, padding=1), 10, flush, stream))
+    tf = case.nz_flops() / (ms * 1e-3) / 1e12
+    out["conv3x3_28"] = {"ms": ms, "nz_tflops": tf, "roofline_frac": tf / ALU_PEAK_TFLOPS,
+                         "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
+                         "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R, case.Cout,
+                                                   case.G, case.K)}
+    return out
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        # the CPU oracle needs no process group: rank 0 runs it, other ranks exit
+        return run_reference(args, int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")))
+    rank, world, local = dist_init(args)
+    rc = run_ours(args, rank, world, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return rc
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,192 @@
+/*
+ * cci.h -- C ABI of libcci.so: forward products of layers with cross-channel
+ * intragroup (CCI) sparsity on NVIDIA GB300 (sm_103a).
+ *
+ * Method: Yu et al., "Cross-Channel Intragroup Sparsity Neural Network"
+ * (arXiv 1910.11971).  For every input feature r of a layer (for a convolution,
+ * every tap (kh, kw, ci)), the weights of G neighbouring output channels form a
+ * group, and exactly K of the G are kept (Sec. 3.1, Fig. 1).  Every G rows of the
+ * weight matrix therefore compress into K rows of (value, index) pairs, each with
+ * as many columns as the original matrix; the index is the plain row index
+ * inside the group (log2 G bits, Sec. 3.1).  The product H = W x X is then Alg. 2
+ * of Sec. 3.2: H(G*i + Idx, j) += Val * X(k, j).
+ *
+ * Layouts (all row-major, dense, contiguous; element = dtype unless stated):
+ *   W       [Cout][R]              dense weights (pack input); R = Cin*KH*KW,
+ *                                  r = (kh*KW + kw)*Cin + ci for convolutions
+ *                                  (OHWI order)
+ *   values  [Cout/G][R][K]         kept weights, per (group, r) in increasing index
+ *   idx     [Cout/G][R][K] uint8   index j in [0, G) of each kept weight
+ *   X       [N][Cin]               product input: N columns of Cin features
+ *                                  (the paper's column-major X)
+ *   X       [B][H][W][Cin]         convolution input (NHWC)
+ *   Y       [N][Cout] float32      product output (the paper's H, transposed)
+ *   Y       [B][P][Q][Cout] float32  convolution output (NHWC),
+ *                                  P = (H + 2*pad_h - KH)/stride_h + 1, Q likewise
+ *
+ * Ownership and execution: the caller allocates every buffer; all data pointers
+ * are DEVICE pointers; the library allocates nothing and keeps no state between
+ * calls.  Every call is asynchronous on `stream` (NULL = the legacy default
+ * stream) and returns once its kernels are enqueued.  Calls on different
+ * streams may run concurrently when their outputs do not overlap.
+ *
+ * Errors:
+ *   - Argument errors are detected on the host, before anything is enqueued, and
+ *     returned directly (nothing is written).
+ *   - A failed launch returns CCI_ERR_CUDA.
+ *   - Errors found by the kernels while they run (NaN in a pack input, a packed
+ *     index >= G, an expired bounded wait) are OR-ed as bits (1u << code) into
+ *     the caller's device word `*dev_status`, if it is not NULL; read it after
+ *     synchronising the stream and decode it with cci_decode_device_status().
+ *     The library never clears that word.  When a kernel reports an error its
+ *     outputs are unspecified.
+ */
+#ifndef CCI_H_
+#define CCI_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st; /* the same type as cudaStream_t */
+typedef struct CUstream_st *cci_stream_t;
+
+typedef enum cci_status {
+    CCI_OK = 0,
+    CCI_ERR_NULL = 1,         /* a required pointer is NULL */
+    CCI_ERR_SHAPE = 2,        /* a size is negative/zero where not allowed, too large,
+                                 or the convolution geometry has no output */
+    CCI_ERR_GROUP = 3,        /* G not in [1, 256], K not in [1, G], or Cout % G != 0 */
+    CCI_ERR_DTYPE = 4,        /* dtype is not a cci_dtype */
+    CCI_ERR_ALIGN = 5,        /* a pointer is not aligned to its element size */
+    CCI_ERR_VALUE = 6,        /* device: NaN among the weights given to cci_pack */
+    CCI_ERR_CUDA = 7,         /* a CUDA launch or runtime call failed */
+    CCI_ERR_TIMEOUT = 8,      /* device: a bounded wait inside a kernel expired */
+    CCI_ERR_UNSUPPORTED = 9,  /* valid request this build does not implement */
+    CCI_ERR_INDEX = 10        /* device: a packed index >= G given to a product */
+} cci_status;
+
+typedef enum cci_dtype {
+    CCI_F32 = 0,   /* IEEE binary32 */
+    CCI_BF16 = 1   /* bfloat16; products accumulate in fp32 on the exact values */
+} cci_dtype;
+
+/* Kernel family for cci_linear_ex / cci_conv2d_ex. */
+typedef enum cci_algo {
+    CCI_ALGO_AUTO = 0,      /* register-tiled scatter kernel when (G, K, dtype, shape)
+                               has one, else the generic kernel */
+    CCI_ALGO_GENERIC = 1,   /* generic kernel: any G <= 256, any K, any alignment */
+    CCI_ALGO_REGTILE = 2,   /* register-tiled scatter kernel only; CCI_ERR_UNSUPPORTED
+                               when (G, K, dtype, shape) has none */
+    CCI_ALGO_DENSE_TC = 3   /* comparison only: decompress to bf16 tiles in shared
+                               memory and multiply densely on the tensor cores
+                               (tcgen05); bf16 only */
+} cci_algo;
+
+/*
+ * cci_pack -- choose and compress the kept weights (Sec. 3.1 format, Sec. 5.1
+ * selection: the weights of largest |w| survive).
+ *
+ * For every group gi in [0, Cout/G) and r in [0, R), the G weights
+ * W[gi*G + j][r], j = 0..G-1, are ranked by decreasing |w| (compared in the
+ * storage dtype; -0 and +0 are equal, +-inf is largest); equal magnitudes rank by
+ * increasing j.  The first K survive and are written in increasing j:
+ * values[gi][r][s] = W[gi*G + j_s][r] (bit-exact copy), idx[gi][r][s] = j_s.
+ *
+ *   W          device, [Cout][R] of dtype, aligned to the element size
+ *   values     device, [Cout/G][R][K] of dtype (written)
+ *   idx        device, [Cout/G][R][K] uint8 (written)
+ *   dev_status device uint32 or NULL; NaN in W sets bit (1u << CCI_ERR_VALUE)
+ *              (with NULL, NaN goes unreported and ranks above +inf)
+ * Errors: CCI_ERR_NULL, CCI_ERR_SHAPE (Cout or R < 1), CCI_ERR_GROUP,
+ *         CCI_ERR_DTYPE, CCI_ERR_ALIGN, CCI_ERR_CUDA.
+ */
+cci_status cci_pack(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K,
+                    void *values, uint8_t *idx, uint32_t *dev_status, cci_stream_t stream);
+
+/*
+ * cci_linear -- Y = X W-hat^T for a CCI-sparse fully connected layer (Alg. 2 of
+ * Sec. 3.2 over all N columns, with the slot loop for K > 1):
+ *   Y[n][gi*G + idx[gi][r][s]] += values[gi][r][s] * X[n][r]
+ * summed over r and s in fp32, starting from zero.  A repeated index inside one
+ * (group, r) adds both values, as Alg. 2 does.
+ *
+ *   X          device, [N][Cin] of dtype (R = Cin)
+ *   values,idx device, as written by cci_pack for (Cout, R = Cin, G, K)
+ *   Y          device, [N][Cout] float32 (written, every element)
+ *   dev_status device uint32 or NULL; an index >= G sets bit (1u << CCI_ERR_INDEX)
+ * N = 0 is valid and enqueues nothing.
+ * Errors: CCI_ERR_NULL, CCI_ERR_SHAPE, CCI_ERR_GROUP, CCI_ERR_DTYPE, CCI_ERR_ALIGN,
+ *         CCI_ERR_CUDA.
+ */
+cci_status cci_linear(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
+                      const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
+                      float *Y, uint32_t *dev_status, cci_stream_t stream);
+
+/*
+ * cci_conv2d -- CCI-sparse 2-D convolution (Sec. 3.1: the structure applies to
+ * convolutional layers with one group per tap (kh, kw, ci)), computed as an
+ * implicit product: column n = (b, p, q), reduction index
+ * r = (kh*KW + kw)*Cin + ci, and
+ *   x[n][r] = X[b][p*stride_h - pad_h + kh][q*stride_w - pad_w + kw][ci]
+ * or 0 outside the image (cross-correlation, zero padding, floor output size, no
+ * dilation, conv groups or bias).
+ *
+ *   X          device NHWC [B][H][W][Cin] of dtype
+ *   values,idx device, cci_pack output for W[Cout][KH*KW*Cin] (OHWI)
+ *   Y          device NHWC [B][P][Q][Cout] float32 (written, every element)
+ * B = 0 is valid and enqueues nothing.
+ * Errors: as cci_linear; CCI_ERR_SHAPE also when P or Q < 1.
+ */
+cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W,
+                      int64_t Cin, const void *values, const uint8_t *idx, int64_t Cout,
+                      int KH, int KW, int stride_h, int stride_w, int pad_h, int pad_w, int G,
+                      int K, float *Y, uint32_t *dev_status, cci_stream_t stream);
+
+/* As cci_linear / cci_conv2d, with the kernel family chosen by `algo`. */
+cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
+                         const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
+                         float *Y, uint32_t *dev_status, cci_algo algo, cci_stream_t stream);
+cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W,
+                         int64_t Cin, const void *values, const uint8_t *idx, int64_t Cout,
+                         int KH, int KW, int stride_h, int stride_w, int pad_h, int pad_w,
+                         int G, int K, float *Y, uint32_t *dev_status, cci_algo algo,
+                         cci_stream_t stream);
+
+/*
+ * cci_kernel_name -- the name of the kernel that cci_linear_ex / cci_conv2d_ex
+ * would launch for a layer with these sizes (R = Cin for a product, Cin*KH*KW
+ * for a convolution) when every pointer is 16-byte aligned: a static string, ""
+ * when the call would be rejected.  No device work; used to label results.
+ */
+const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K,
+                            cci_algo algo);
+
+/* Human-readable text of a status code (static string). */
+const char *cci_status_string(cci_status status);
+
+/* The lowest-numbered error among the bits set in a device status word, or
+ * CCI_OK when none is set. */
+cci_status cci_decode_device_status(uint32_t word);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int cci_version(void);
+
+/*
+ * cci_fma_probe -- measurement helper, not part of the method: enqueue one
+ * kernel of `blocks` x `threads` threads, each running `iters` iterations of 16
+ * independent packed fp32 FMAs (fma.rn.f32x2, 2 FMAs each), and write one float
+ * per thread to `out` (device, blocks*threads floats) so the work is kept.
+ * Flops performed = blocks * threads * iters * 64.  Time it with CUDA events to
+ * measure the CUDA-core FMA throughput.
+ * Errors: CCI_ERR_NULL, CCI_ERR_SHAPE, CCI_ERR_CUDA.
+ */
+cci_status cci_fma_probe(float *out, int blocks, int threads, int iters, cci_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CCI_H_ */

@@ -1,0 +1,194 @@
+"""Python binding of libcci.so: CCI-sparse layers (arXiv 1910.11971) on GB300.
+
+Argument marshalling only.  Every step of the computation runs in the CUDA
+kernels of ``libcci.so`` (built from ``csrc/`` by ``build.py``); PyTorch is used
+for device memory and the current stream.  There is no CPU path: if the
+library is missing or a call fails, an exception is raised.
+
+    values, idx = pack(W, G, K)                         # Sec. 3.1 / 5.1
+    Y = linear(X, values, idx, Cout, G, K)              # Alg. 2, Y[N][Cout] fp32
+    Y = conv2d(X, values, idx, Cout, G, K, KH, KW, stride, pad)  # NHWC
+
+Layouts are those of ``include/cci.h``: W [Cout][R], values/idx [Cout/G][R][K],
+X [N][Cin] (product) or NHWC [B][H][W][Cin] (convolution), Y fp32.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional, Sequence, Tuple
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libcci.so")
+
+F32, BF16 = 0, 1
+ALGO_AUTO, ALGO_GENERIC, ALGO_REGTILE, ALGO_DENSE_TC = 0, 1, 2, 3
+
+STATUS_NAMES = {
+    0: "CCI_OK", 1: "CCI_ERR_NULL", 2: "CCI_ERR_SHAPE", 3: "CCI_ERR_GROUP", 4: "CCI_ERR_DTYPE",
+    5: "CCI_ERR_ALIGN", 6: "CCI_ERR_VALUE", 7: "CCI_ERR_CUDA", 8: "CCI_ERR_TIMEOUT",
+    9: "CCI_ERR_UNSUPPORTED", 10: "CCI_ERR_INDEX",
+}
+
+# exported symbols with their ctypes signatures (the declarations of cci.h)
+_P, _I64, _I32, _U32P = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p
+SIGNATURES = {
+    "cci_pack": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, _P, _P, _U32P, _P]),
+    "cci_linear": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P, _P]),
+    "cci_linear_ex": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P, _I32, _P]),
+    "cci_conv2d": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32, _I32,
+                          _I32, _I32, _I32, _I32, _P, _U32P, _P]),
+    "cci_conv2d_ex": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32, _I32,
+                             _I32, _I32, _I32, _I32, _P, _U32P, _I32, _P]),
+    "cci_kernel_name": (ctypes.c_char_p, [_I32, _I64, _I64, _I64, _I32, _I32, _I32]),
+    "cci_status_string": (ctypes.c_char_p, [_I32]),
+    "cci_decode_device_status": (_I32, [ctypes.c_uint32]),
+    "cci_version": (_I32, []),
+    "cci_fma_probe": (_I32, [_P, _I32, _I32, _I32, _P]),
+}
+
+_lib = None
+
+
+class CCIError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = int(status)
+        text = lib().cci_status_string(self.status).decode() if _lib is not None else ""
+        super().__init__(f"{where}: {STATUS_NAMES.get(self.status, self.status)} ({text})")
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libcci.so.  Raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"libcci.so is not built ({LIB_PATH}); run "
+                               "`python -m paper_1910_11971_gb300.build` (needs nvcc)")
+        h = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(h, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = h
+    return _lib
+
+
+def status_string(code: int) -> str:
+    return lib().cci_status_string(int(code)).decode()
+
+
+def decode_status(word: int) -> int:
+    return int(lib().cci_decode_device_status(ctypes.c_uint32(int(word) & 0xffffffff)))
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return F32
+    if t.dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"unsupported dtype {t.dtype}: float32 or bfloat16")
+
+
+def _stream(device: torch.device) -> int:
+    return torch.cuda.current_stream(device).cuda_stream
+
+
+def _cuda_contig(t: torch.Tensor, name: str) -> None:
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def _check(code: int, where: str) -> None:
+    if code != 0:
+        raise CCIError(code, where)
+
+
+def new_status(device) -> torch.Tensor:
+    """A zeroed device status word for the ``status=`` argument of the calls."""
+    return torch.zeros(1, dtype=torch.int32, device=device)
+
+
+def read_status(status: torch.Tensor) -> int:
+    """Synchronise and return the first error recorded in a status word (0 = none)."""
+    return decode_status(int(status.item()))
+
+
+def pack(W: torch.Tensor, G: int, K: int, *, status: Optional[torch.Tensor] = None,
+         check: bool = True, out: Optional[Tuple[torch.Tensor, torch.Tensor]] = None):
+    """Per-group top-K by |w| (ties to the lower index) -> (values, idx).
+
+    W: CUDA [Cout][R] float32 or bfloat16.  With ``check`` (the default) the call
+    synchronises and raises on NaN weights; with ``check=False`` it stays
+    asynchronous and records errors only in ``status`` (if given)."""
+    _cuda_contig(W, "W")
+    Cout, R = W.shape
+    if G < 1 or Cout % G:
+        raise CCIError(3, "pack")
+    if out is None:
+        values = torch.empty((Cout // G, R, K), dtype=W.dtype, device=W.device)
+        idx = torch.empty((Cout // G, R, K), dtype=torch.uint8, device=W.device)
+    else:
+        values, idx = out
+    own_status = status is None and check
+    if own_status:
+        status = new_status(W.device)
+    code = lib().cci_pack(W.data_ptr(), _dtype_code(W), Cout, R, G, K, values.data_ptr(),
+                          idx.data_ptr(), status.data_ptr() if status is not None else None,
+                          _stream(W.device))
+    _check(code, "cci_pack")
+    if check:
+        dev = read_status(status)
+        if dev:
+            raise CCIError(dev, "cci_pack (device)")
+    return values, idx
+
+
+def linear(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int, *,
+           out: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
+           algo: int = ALGO_AUTO) -> torch.Tensor:
+    """Y[N][Cout] (fp32) = the CCI-sparse product of X[N][Cin] (Alg. 2)."""
+    _cuda_contig(X, "X")
+    N, Cin = X.shape
+    Y = out if out is not None else torch.empty((N, Cout), dtype=torch.float32, device=X.device)
+    code = lib().cci_linear_ex(X.data_ptr(), _dtype_code(X), N, Cin, values.data_ptr(),
+                               idx.data_ptr(), Cout, G, K, Y.data_ptr(),
+                               status.data_ptr() if status is not None else None, algo,
+                               _stream(X.device))
+    _check(code, "cci_linear")
+    return Y
+
+
+def conv_out_hw(H: int, W: int, KH: int, KW: int, stride: Sequence[int], pad: Sequence[int]):
+    return (H + 2 * pad[0] - KH) // stride[0] + 1, (W + 2 * pad[1] - KW) // stride[1] + 1
+
+
+def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int,
+           KH: int, KW: int, stride=(1, 1), pad=(0, 0), *, out: Optional[torch.Tensor] = None,
+           status: Optional[torch.Tensor] = None, algo: int = ALGO_AUTO) -> torch.Tensor:
+    """Y NHWC [B][P][Q][Cout] (fp32) = CCI-sparse convolution of X NHWC [B][H][W][Cin]."""
+    _cuda_contig(X, "X")
+    B, H, W, Cin = X.shape
+    P, Q = conv_out_hw(H, W, KH, KW, stride, pad)
+    Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=torch.float32,
+                                                device=X.device)
+    code = lib().cci_conv2d_ex(X.data_ptr(), _dtype_code(X), B, H, W, Cin, values.data_ptr(),
+                               idx.data_ptr(), Cout, KH, KW, stride[0], stride[1], pad[0], pad[1],
+                               G, K, Y.data_ptr(), status.data_ptr() if status is not None else None,
+                               algo, _stream(X.device))
+    _check(code, "cci_conv2d")
+    return Y
+
+
+def kernel_name(dtype: torch.dtype, Cin: int, R: int, Cout: int, G: int, K: int,
+                algo: int = ALGO_AUTO) -> str:
+    code = F32 if dtype == torch.float32 else BF16
+    return lib().cci_kernel_name(code, Cin, R, Cout, G, K, algo).decode()
+
+
+def fma_probe(out: torch.Tensor, blocks: int, threads: int, iters: int) -> None:
+    _check(lib().cci_fma_probe(out.data_ptr(), blocks, threads, iters, _stream(out.device)),
+           "cci_fma_probe")

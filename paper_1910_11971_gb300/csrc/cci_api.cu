@@ -1,0 +1,253 @@
+// cci_api.cu -- the extern "C" entry points of libcci.so (declared in cci.h).
+//
+// Host side only: argument checks (all before anything is enqueued), choice of
+// kernel, launch on the caller's stream.  The library allocates nothing.
+#include <cstdint>
+#include <cstring>
+
+#include "cci_kernels.h"
+
+namespace cci {
+
+extern const RegtileEntry kRegtile_f32_a[];
+extern const RegtileEntry kRegtile_f32_b[];
+extern const RegtileEntry kRegtile_bf16_a[];
+extern const RegtileEntry kRegtile_bf16_b[];
+
+namespace {
+
+constexpr int64_t kMaxElems = int64_t(1) << 62;
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+size_t elem_size(int dtype) { return dtype == CCI_F32 ? 4 : 2; }
+
+bool valid_dtype(int dtype) { return dtype == CCI_F32 || dtype == CCI_BF16; }
+
+// a*b without overflow past kMaxElems (all inputs >= 0)
+bool mul_ok(int64_t a, int64_t b)
+{
+    if (a == 0 || b == 0) return true;
+    return a <= kMaxElems / b;
+}
+
+cci_status check_group(int64_t Cout, int G, int K)
+{
+    if (G < 1 || G > 256 || K < 1 || K > G) return CCI_ERR_GROUP;
+    if (Cout % G != 0) return CCI_ERR_GROUP;
+    return CCI_OK;
+}
+
+const RegtileEntry *find_regtile(int dtype, int G, int K)
+{
+    const RegtileEntry *tables[] = {kRegtile_f32_a, kRegtile_f32_b, kRegtile_bf16_a, kRegtile_bf16_b};
+    for (const RegtileEntry *t : tables)
+        for (; t->launch; ++t)
+            if (t->dtype == dtype && t->G == G && t->K == K) return t;
+    return nullptr;
+}
+
+// shape conditions of the register-tiled kernel (16-byte vector copies)
+bool regtile_shape_ok(int dtype, int64_t Cin, int64_t R, int K)
+{
+    const int64_t vec = 16 / static_cast<int64_t>(elem_size(dtype));
+    return (Cin % vec == 0) && ((R * K) % 16 == 0) && (R < (int64_t(1) << 31));
+}
+
+bool regtile_ptr_ok(const FwdParams &p)
+{
+    return aligned(p.X, 16) && aligned(p.values, 16) && aligned(p.idx, 16) && aligned(p.Y, 16);
+}
+
+cci_status to_status(cudaError_t e) { return e == cudaSuccess ? CCI_OK : CCI_ERR_CUDA; }
+
+cci_status forward(const FwdParams &p, int dtype, int G, int K, cci_algo algo, cudaStream_t stream)
+{
+    if (p.N == 0) return CCI_OK;
+    if (algo == CCI_ALGO_DENSE_TC) return CCI_ERR_UNSUPPORTED;
+    if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE) {
+        const RegtileEntry *e = find_regtile(dtype, G, K);
+        if (e && regtile_shape_ok(dtype, p.Cin, p.R, K) && regtile_ptr_ok(p)) return to_status(e->launch(p, stream));
+        if (algo == CCI_ALGO_REGTILE) return CCI_ERR_UNSUPPORTED;
+    } else if (algo != CCI_ALGO_GENERIC) {
+        return CCI_ERR_UNSUPPORTED;
+    }
+    return to_status(launch_generic(p, dtype, G, K, stream));
+}
+
+cci_status check_common(const void *X, int dtype, const void *values, const uint8_t *idx, float *Y,
+                        int64_t N, int64_t Cout, int64_t R, int G, int K)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!values || !idx) return CCI_ERR_NULL;
+    if (N > 0 && (!X || !Y)) return CCI_ERR_NULL;
+    if (N < 0 || Cout < 1 || R < 1) return CCI_ERR_SHAPE;
+    const cci_status g = check_group(Cout, G, K);
+    if (g != CCI_OK) return g;
+    if (!mul_ok(N, Cout) || !mul_ok(R, K) || !mul_ok(R * K, Cout / G) || R >= (int64_t(1) << 40))
+        return CCI_ERR_SHAPE;
+    const size_t es = elem_size(dtype);
+    if (!aligned(values, es) || (X && !aligned(X, es)) || (Y && !aligned(Y, 4))) return CCI_ERR_ALIGN;
+    return CCI_OK;
+}
+
+}  // namespace
+
+int regtile_wc(int64_t groups, int MG)
+{
+    // 8 channel-warps when the layer has enough groups, else 4 (fewer would
+    // widen the column tile past the shared-memory budget)
+    return static_cast<int64_t>(8) * MG <= groups ? 8 : 4;
+}
+
+}  // namespace cci
+
+using namespace cci;
+
+extern "C" {
+
+int cci_version(void) { return 1 * 10000 + 0 * 100 + 0; }
+
+const char *cci_status_string(cci_status s)
+{
+    switch (s) {
+        case CCI_OK: return "ok";
+        case CCI_ERR_NULL: return "a required pointer is NULL";
+        case CCI_ERR_SHAPE: return "invalid or too large shape";
+        case CCI_ERR_GROUP: return "invalid group: need 1 <= K <= G <= 256 and Cout % G == 0";
+        case CCI_ERR_DTYPE: return "unknown dtype";
+        case CCI_ERR_ALIGN: return "pointer not aligned to its element size";
+        case CCI_ERR_VALUE: return "NaN among the weights given to cci_pack";
+        case CCI_ERR_CUDA: return "CUDA launch or runtime error";
+        case CCI_ERR_TIMEOUT: return "a bounded wait inside a kernel expired";
+        case CCI_ERR_UNSUPPORTED: return "request not supported by this build";
+        case CCI_ERR_INDEX: return "a packed index >= G";
+    }
+    return "unknown status";
+}
+
+cci_status cci_decode_device_status(uint32_t word)
+{
+    for (int b = 1; b < 32; ++b)
+        if (word & (1u << b)) return static_cast<cci_status>(b);
+    return CCI_OK;
+}
+
+cci_status cci_pack(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K, void *values,
+                    uint8_t *idx, uint32_t *dev_status, cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!W || !values || !idx) return CCI_ERR_NULL;
+    if (Cout < 1 || R < 1 || !mul_ok(Cout, R)) return CCI_ERR_SHAPE;
+    const cci_status g = check_group(Cout, G, K);
+    if (g != CCI_OK) return g;
+    const size_t es = elem_size(dtype);
+    if (!aligned(W, es) || !aligned(values, es)) return CCI_ERR_ALIGN;
+    return to_status(launch_pack(W, dtype, Cout, R, G, K, values, idx, dev_status,
+                                 reinterpret_cast<cudaStream_t>(stream)));
+}
+
+cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+                         const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
+                         cci_algo algo, cci_stream_t stream)
+{
+    const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, Cin, G, K);
+    if (st != CCI_OK) return st;
+    if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
+    FwdParams p{};
+    p.X = X;
+    p.values = values;
+    p.idx = idx;
+    p.Y = Y;
+    p.status = dev_status;
+    p.N = N;
+    p.Cout = Cout;
+    p.R = Cin;
+    p.Cin = Cin;
+    p.H = p.W = p.P = p.Q = 1;
+    p.KH = p.KW = p.sh = p.sw = 1;
+    p.ph = p.pw = 0;
+    p.is_conv = 0;
+    return forward(p, dtype, G, K, algo, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cci_status cci_linear(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+                      const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
+                      cci_stream_t stream)
+{
+    return cci_linear_ex(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, CCI_ALGO_AUTO, stream);
+}
+
+cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
+                         const void *values, const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h,
+                         int stride_w, int pad_h, int pad_w, int G, int K, float *Y, uint32_t *dev_status,
+                         cci_algo algo, cci_stream_t stream)
+{
+    if (B < 0 || H < 1 || W < 1 || Cin < 1 || KH < 1 || KW < 1 || stride_h < 1 || stride_w < 1 || pad_h < 0 ||
+        pad_w < 0)
+        return valid_dtype(dtype) ? CCI_ERR_SHAPE : CCI_ERR_DTYPE;
+    const int64_t lim = int64_t(1) << 30;
+    if (H >= lim || W >= lim || pad_h >= lim || pad_w >= lim) return CCI_ERR_SHAPE;
+    if (H + 2 * pad_h < KH || W + 2 * pad_w < KW) return CCI_ERR_SHAPE;
+    const int64_t P = (H + 2 * pad_h - KH) / stride_h + 1;
+    const int64_t Q = (W + 2 * pad_w - KW) / stride_w + 1;
+    if (!mul_ok(P, Q) || !mul_ok(B, P * Q) || !mul_ok(H, W) || !mul_ok(H * W, Cin) || !mul_ok(B, H * W * Cin) ||
+        !mul_ok(static_cast<int64_t>(KH) * KW, Cin))
+        return CCI_ERR_SHAPE;
+    const int64_t N = B * P * Q;
+    const int64_t R = static_cast<int64_t>(KH) * KW * Cin;
+    const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, R, G, K);
+    if (st != CCI_OK) return st;
+    FwdParams p{};
+    p.X = X;
+    p.values = values;
+    p.idx = idx;
+    p.Y = Y;
+    p.status = dev_status;
+    p.N = N;
+    p.Cout = Cout;
+    p.R = R;
+    p.Cin = Cin;
+    p.H = H;
+    p.W = W;
+    p.P = P;
+    p.Q = Q;
+    p.KH = KH;
+    p.KW = KW;
+    p.sh = stride_h;
+    p.sw = stride_w;
+    p.ph = pad_h;
+    p.pw = pad_w;
+    p.is_conv = 1;
+    return forward(p, dtype, G, K, algo, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
+                      const void *values, const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h,
+                      int stride_w, int pad_h, int pad_w, int G, int K, float *Y, uint32_t *dev_status,
+                      cci_stream_t stream)
+{
+    return cci_conv2d_ex(X, dtype, B, H, W, Cin, values, idx, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, G, K,
+                         Y, dev_status, CCI_ALGO_AUTO, stream);
+}
+
+const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K, cci_algo algo)
+{
+    if (!valid_dtype(dtype) || Cin < 1 || R < Cin || check_group(Cout, G, K) != CCI_OK) return "";
+    if (algo == CCI_ALGO_DENSE_TC) return "";
+    if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE) {
+        const RegtileEntry *e = find_regtile(dtype, G, K);
+        if (e && regtile_shape_ok(dtype, Cin, R, K)) return e->name;
+        if (algo == CCI_ALGO_REGTILE) return "";
+    }
+    return dtype == CCI_F32 ? "generic_f32" : "generic_bf16";
+}
+
+cci_status cci_fma_probe(float *out, int blocks, int threads, int iters, cci_stream_t stream)
+{
+    if (!out) return CCI_ERR_NULL;
+    if (blocks < 1 || threads < 1 || threads > 1024 || iters < 0) return CCI_ERR_SHAPE;
+    return to_status(launch_fma_probe(out, blocks, threads, iters, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+}  // extern "C"

@@ -1,0 +1,172 @@
+// cci_basic.cu -- the pack kernel, the generic product kernel and the FMA probe.
+#include "cci_kernels.h"
+
+namespace cci {
+
+// ---------------------------------------------------------------------------
+// pack: one thread per (group gi, input feature r).  Sec. 3.1 / Sec. 5.1:
+// the K weights of largest |w| in W[gi*G .. gi*G+G)[r] survive, ties to the
+// lower index, and are written in increasing index.  |w| is compared on the
+// storage bits with the sign cleared (an order-preserving integer compare for
+// every non-NaN value; NaN bit patterns rank above +inf and are reported).
+// ---------------------------------------------------------------------------
+template <typename TB>  // uint32_t for fp32, uint16_t for bf16 (raw bits)
+__global__ void pack_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, int G, int K,
+                            TB *__restrict__ values, uint8_t *__restrict__ idx, uint32_t *status)
+{
+    constexpr uint32_t kAbs = sizeof(TB) == 4 ? 0x7fffffffu : 0x7fffu;
+    constexpr uint32_t kInf = sizeof(TB) == 4 ? 0x7f800000u : 0x7f80u;
+    const int64_t total = (Cout / G) * R;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gi = t / R;
+        const int64_t r = t - gi * R;
+        const TB *col = W + gi * G * R + r;
+        bool nan = false;
+        int s = 0;
+        for (int j = 0; j < G && s < K; ++j) {
+            const TB wj = col[static_cast<int64_t>(j) * R];
+            const uint32_t a = static_cast<uint32_t>(wj) & kAbs;
+            nan |= a > kInf;
+            int rank = 0;  // number of entries ranked ahead of j
+            for (int j2 = 0; j2 < G && rank < K; ++j2) {
+                const uint32_t b = static_cast<uint32_t>(col[static_cast<int64_t>(j2) * R]) & kAbs;
+                rank += (b > a) || (b == a && j2 < j);
+            }
+            if (rank < K) {
+                values[t * K + s] = wj;
+                idx[t * K + s] = static_cast<uint8_t>(j);
+                ++s;
+            }
+        }
+        // entries after the K-th survivor were not scanned; check them for NaN too
+        for (int j = 0; j < G; ++j)
+            nan |= (static_cast<uint32_t>(col[static_cast<int64_t>(j) * R]) & kAbs) > kInf;
+        if (nan) report(status, CCI_ERR_VALUE);
+    }
+}
+
+cudaError_t launch_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K, void *values,
+                        uint8_t *idx, uint32_t *status, cudaStream_t stream)
+{
+    const int64_t total = (Cout / G) * R;
+    const int threads = 256;
+    const int64_t blocks = (total + threads - 1) / threads;
+    const int grid = static_cast<int>(blocks < 65536 * 16 ? blocks : 65536 * 16);
+    if (dtype == CCI_F32)
+        pack_kernel<uint32_t><<<grid, threads, 0, stream>>>(static_cast<const uint32_t *>(W), Cout, R, G, K,
+                                                            static_cast<uint32_t *>(values), idx, status);
+    else
+        pack_kernel<uint16_t><<<grid, threads, 0, stream>>>(static_cast<const uint16_t *>(W), Cout, R, G, K,
+                                                            static_cast<uint16_t *>(values), idx, status);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// generic product: any G <= 256, any K, any alignment.  A CTA of 128 threads
+// owns one group and 128 columns; thread = column; the G accumulators of the
+// column live in shared memory acc[G][128] (the thread's own column only).
+// Contributions arrive in ascending r, then slot, each one fused multiply-add
+// from +0 -- the same order as the register-tiled kernel.
+// ---------------------------------------------------------------------------
+template <typename TB>
+__device__ __forceinline__ float load_elem(const TB *p, int64_t off);
+template <>
+__device__ __forceinline__ float load_elem<uint32_t>(const uint32_t *p, int64_t off)
+{
+    return __uint_as_float(__ldg(p + off));
+}
+template <>
+__device__ __forceinline__ float load_elem<uint16_t>(const uint16_t *p, int64_t off)
+{
+    return bf16_bits_to_f32(__ldg(p + off));
+}
+
+template <typename TB>
+__global__ void __launch_bounds__(128) generic_kernel(FwdParams p, int G, int K, int64_t n_col_tiles)
+{
+    extern __shared__ float acc[];  // [G][128]
+    const int tid = threadIdx.x;
+    const int64_t tile = blockIdx.x;
+    const int64_t gi = tile / n_col_tiles;
+    const int64_t n = (tile - gi * n_col_tiles) * 128 + tid;
+    const bool col_ok = n < p.N;
+    for (int i = 0; i < G; ++i) acc[i * 128 + tid] = 0.0f;
+    ColumnSite site{0, 0, 0};
+    if (col_ok) site = column_site(p, n);
+    const TB *X = static_cast<const TB *>(p.X);
+    const TB *V = static_cast<const TB *>(p.values) + gi * p.R * K;
+    const uint8_t *I = p.idx + gi * p.R * K;
+    bool bad = false;
+    for (int64_t r = 0; r < p.R; ++r) {
+        float x = 0.0f;
+        if (col_ok) {
+            const int64_t off = x_offset(p, site, r);
+            if (off >= 0) x = load_elem<TB>(X, off);
+        }
+        for (int s = 0; s < K; ++s) {
+            const int i = I[r * K + s];
+            const float v = load_elem<TB>(V, r * K + s);
+            if (i >= G) {
+                bad = true;
+                continue;
+            }
+            acc[i * 128 + tid] = fmaf(v, x, acc[i * 128 + tid]);
+        }
+    }
+    if (bad && tid == 0) report(p.status, CCI_ERR_INDEX);
+    if (col_ok) {
+        float *y = p.Y + n * p.Cout + gi * G;
+        for (int i = 0; i < G; ++i) y[i] = acc[i * 128 + tid];
+    }
+}
+
+cudaError_t launch_generic(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream)
+{
+    const int64_t n_col_tiles = (p.N + 127) / 128;
+    const int64_t tiles = n_col_tiles * (p.Cout / G);
+    const size_t smem = static_cast<size_t>(G) * 128 * sizeof(float);
+    static const bool attr = [] {
+        cudaFuncSetAttribute(generic_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             256 * 128 * 4);
+        cudaFuncSetAttribute(generic_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             256 * 128 * 4);
+        return true;
+    }();
+    (void)attr;
+    if (tiles > 0x7fffffffll) return cudaErrorInvalidConfiguration;
+    if (dtype == CCI_F32)
+        generic_kernel<uint32_t><<<static_cast<unsigned>(tiles), 128, smem, stream>>>(p, G, K, n_col_tiles);
+    else
+        generic_kernel<uint16_t><<<static_cast<unsigned>(tiles), 128, smem, stream>>>(p, G, K, n_col_tiles);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// FMA probe: 16 independent packed-FMA chains per thread
+// ---------------------------------------------------------------------------
+__global__ void fma_probe_kernel(float *out, int iters)
+{
+    unsigned long long acc[16];
+    const float seed = static_cast<float>(threadIdx.x) * 1e-3f;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) acc[k] = pack2(seed + k, seed - k);
+    const unsigned long long a = pack2(1.0e-3f, -1.0e-3f);
+    const unsigned long long b = pack2(0.5f, 0.25f);
+    for (int it = 0; it < iters; ++it) {
+#pragma unroll
+        for (int k = 0; k < 16; ++k) ffma2(acc[k], a, b);
+    }
+    float s = 0.0f;
+#pragma unroll
+    for (int k = 0; k < 16; ++k) s += lo_of(acc[k]) + hi_of(acc[k]);
+    out[blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x] = s;
+}
+
+cudaError_t launch_fma_probe(float *out, int blocks, int threads, int iters, cudaStream_t stream)
+{
+    fma_probe_kernel<<<blocks, threads, 0, stream>>>(out, iters);
+    return cudaGetLastError();
+}
+
+}  // namespace cci

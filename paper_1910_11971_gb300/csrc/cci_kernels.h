@@ -1,0 +1,28 @@
+// cci_kernels.h -- launchers shared between the libcci translation units.
+#pragma once
+
+#include "cci_common.cuh"
+
+namespace cci {
+
+cudaError_t launch_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K, void *values,
+                        uint8_t *idx, uint32_t *status, cudaStream_t stream);
+cudaError_t launch_generic(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);
+cudaError_t launch_fma_probe(float *out, int blocks, int threads, int iters, cudaStream_t stream);
+
+// One register-tiled instantiation: (dtype, G, K) -> tile shape and launcher.
+struct RegtileEntry {
+    int dtype, G, K, MG, T;
+    const char *name;
+    cudaError_t (*launch)(const FwdParams &p, cudaStream_t stream);
+};
+
+// all instantiations, terminated by an entry with launch == nullptr
+const RegtileEntry *regtile_table();
+
+// channel-warps per CTA (4 or 8) for a layer with this many groups
+int regtile_wc(int64_t groups, int MG);
+
+constexpr size_t kMaxSmemPerBlock = 227 * 1024;
+
+}  // namespace cci

@@ -1,0 +1,141 @@
+"""The C ABI without a GPU: libcci.so builds, loads, exports every entry point
+that include/cci.h declares, and rejects bad arguments with the documented
+status before anything is enqueued (these paths never touch the device)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_1910_11971_gb300 as cci
+from paper_1910_11971_gb300 import build as cci_build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "cci.h")
+
+OK, NULL, SHAPE, GROUP, DTYPE, ALIGN, VALUE, CUDA, TIMEOUT, UNSUP, INDEX = range(11)
+FAKE = 0x10000  # a 256-byte-aligned non-null address; never dereferenced on these paths
+
+
+@pytest.fixture(scope="module")
+def lib():
+    cci_build.build()
+    return cci.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(cci_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("cci_pack", "cci_linear", "cci_conv2d", "cci_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing
+    assert set(declared_functions()) == set(cci.SIGNATURES)
+
+
+def test_version_and_strings(lib):
+    assert lib.cci_version() >= 10000
+    for code in range(11):
+        assert lib.cci_status_string(code)
+    assert lib.cci_status_string(OK) == b"ok"
+
+
+def test_decode_device_status(lib):
+    assert cci.decode_status(0) == OK
+    assert cci.decode_status(1 << INDEX) == INDEX
+    assert cci.decode_status((1 << INDEX) | (1 << VALUE)) == VALUE
+    assert cci.decode_status(1 << TIMEOUT) == TIMEOUT
+
+
+def linear(lib, X=FAKE, dt=0, N=16, Cin=16, V=FAKE, I=FAKE, Cout=16, G=8, K=2, Y=FAKE, algo=0):
+    return lib.cci_linear_ex(X, dt, N, Cin, V, I, Cout, G, K, Y, None, algo, None)
+
+
+def conv(lib, X=FAKE, dt=1, B=1, H=4, W=4, Cin=8, V=FAKE, I=FAKE, Cout=8, KH=3, KW=3, sh=1, sw=1,
+         ph=1, pw=1, G=8, K=2, Y=FAKE, algo=0):
+    return lib.cci_conv2d_ex(X, dt, B, H, W, Cin, V, I, Cout, KH, KW, sh, sw, ph, pw, G, K, Y, None,
+                             algo, None)
+
+
+def test_linear_rejects(lib):
+    assert linear(lib, X=None) == NULL
+    assert linear(lib, Y=None) == NULL
+    assert linear(lib, V=None) == NULL
+    assert linear(lib, I=None) == NULL
+    assert linear(lib, dt=7) == DTYPE
+    assert linear(lib, N=-1) == SHAPE
+    assert linear(lib, Cin=0) == SHAPE
+    assert linear(lib, Cout=0) == SHAPE
+    assert linear(lib, G=0) == GROUP
+    assert linear(lib, G=257, Cout=257) == GROUP
+    assert linear(lib, K=0) == GROUP
+    assert linear(lib, K=9) == GROUP
+    assert linear(lib, Cout=12) == GROUP  # 12 % 8
+    assert linear(lib, X=FAKE + 2) == ALIGN  # fp32 needs 4-byte alignment
+    assert linear(lib, Y=FAKE + 2) == ALIGN
+    assert linear(lib, N=1 << 40, Cout=1 << 30) == SHAPE  # N*Cout overflows the limit
+
+
+def test_empty_input_is_ok_without_device(lib):
+    # N = 0 enqueues nothing, so it succeeds even with no GPU (and NULL X / Y)
+    assert linear(lib, N=0, X=None, Y=None) == OK
+    assert conv(lib, B=0, X=None, Y=None) == OK
+
+
+def test_conv_rejects(lib):
+    assert conv(lib, H=0) == SHAPE
+    assert conv(lib, KH=0) == SHAPE
+    assert conv(lib, sh=0) == SHAPE
+    assert conv(lib, ph=-1) == SHAPE
+    assert conv(lib, H=2, KH=5, ph=1) == SHAPE  # no output row
+    assert conv(lib, dt=3) == DTYPE
+    assert conv(lib, G=3) == GROUP
+    assert conv(lib, X=FAKE + 1) == ALIGN  # bf16 needs 2-byte alignment
+    assert conv(lib, I=None) == NULL
+
+
+def test_pack_rejects(lib):
+    p = lib.cci_pack
+    assert p(None, 0, 8, 4, 4, 2, FAKE, FAKE, None, None) == NULL
+    assert p(FAKE, 0, 8, 4, 4, 2, None, FAKE, None, None) == NULL
+    assert p(FAKE, 2, 8, 4, 4, 2, FAKE, FAKE, None, None) == DTYPE
+    assert p(FAKE, 0, 0, 4, 4, 2, FAKE, FAKE, None, None) == SHAPE
+    assert p(FAKE, 0, 8, 0, 4, 2, FAKE, FAKE, None, None) == SHAPE
+    assert p(FAKE, 0, 8, 4, 3, 2, FAKE, FAKE, None, None) == GROUP
+    assert p(FAKE, 0, 8, 4, 4, 5, FAKE, FAKE, None, None) == GROUP
+    assert p(FAKE + 2, 0, 8, 4, 4, 2, FAKE, FAKE, None, None) == ALIGN
+
+
+def test_algo_dense_tc_without_bf16_is_unsupported_name(lib):
+    assert cci.kernel_name(__import__("torch").float32, 16, 16, 16, 8, 2, cci.ALGO_DENSE_TC) == ""
+
+
+def test_kernel_names(lib):
+    import torch
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2) == "regtile_float_G8_K2_MG2_T8"
+    assert cci.kernel_name(torch.bfloat16, 128, 1152, 128, 16, 4).startswith("regtile_uint16_t_G16_K4")
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 3) == "generic_f32"  # no tile for K=3
+    assert cci.kernel_name(torch.bfloat16, 12, 12, 16, 8, 2) == "generic_bf16"  # Cin % 8 != 0
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 3, cci.ALGO_REGTILE) == ""
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2, cci.ALGO_GENERIC) == "generic_f32"
+
+
+def test_fma_probe_rejects(lib):
+    assert lib.cci_fma_probe(None, 1, 32, 1, None) == NULL
+    assert lib.cci_fma_probe(FAKE, 0, 32, 1, None) == SHAPE
+    assert lib.cci_fma_probe(FAKE, 1, 2048, 1, None) == SHAPE
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(cci, "_lib", None)
+    monkeypatch.setattr(cci, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        cci.lib()

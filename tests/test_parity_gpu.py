@@ -1,0 +1,327 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+* cci_pack: indices exact, values bit for bit, including ties, signed zeros and
+  infinities (Sec. 5.1 selection, ties to the lower index).
+* cci_linear / cci_conv2d: |y - y_oracle| <= 1e-5 * sum |w||x| per output, on
+  small ragged shapes (all outputs) and at the full workload sizes in the
+  launch configuration the benchmark times (sampled outputs: the first and
+  last rows -- tile edges and the ragged tail -- and random ones).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_1910_11971_gb300 as cci
+from paper_1910_11971_gb300 import build as cci_build
+from paper_1910_11971_gb300 import workloads as wl
+from parity_util import assert_pack_equal, assert_within_tol, f64, oracle_reference, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+F32, BF16 = torch.float32, torch.bfloat16
+
+
+@pytest.fixture(scope="module")
+def dev():
+    cci_build.build()
+    assert torch.cuda.is_available(), "GPU tests need CUDA"
+    return torch.device("cuda:0")
+
+
+def _dt(name):
+    return F32 if name == "f32" else BF16
+
+
+# ---------------------------------------------------------------------------
+# pack
+# ---------------------------------------------------------------------------
+PACK_GK = [(1, 1), (2, 1), (3, 2), (4, 1), (4, 2), (4, 4), (5, 3), (8, 1), (8, 2), (8, 3), (8, 4),
+           (16, 4), (16, 8), (32, 4), (32, 16), (64, 5), (256, 7), (256, 256)]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("G,K", PACK_GK)
+def test_pack_random(dev, dtype, G, K):
+    Cout, R = 2 * G, 37
+    W = wl.draw_w(Cout, R, 1.0, dtype, seed=G * 100 + K).to(dev)
+    v, i = cci.pack(W, G, K)
+    vo, io, _, _ = oracle_reference(W, G, K)
+    assert_pack_equal(v, i, vo, io)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("G,K", [(4, 2), (8, 3), (16, 5), (3, 1)])
+def test_pack_ties_signed_zero_inf(dev, dtype, G, K):
+    Cout, R = 4 * G, 29
+    W = wl.integer_valued((Cout, R), -3, 3, seed=G + K)  # many equal magnitudes
+    W[0, :5] = -0.0
+    W[1, 5] = float("inf")
+    W[2 % Cout, 6] = float("-inf")
+    W[:, 7] = 0.0
+    W[:, 8] = -0.0
+    W = W.to(_dt(dtype)).to(dev)
+    v, i = cci.pack(W, G, K)
+    vo, io, _, _ = oracle_reference(W, G, K)
+    assert_pack_equal(v, i, vo, io)
+
+
+def test_pack_nan_reported(dev):
+    W = torch.randn(16, 9, device=dev)
+    W[5, 3] = float("nan")
+    with pytest.raises(cci.CCIError) as e:
+        cci.pack(W, 8, 2)
+    assert e.value.status == 6
+    st = cci.new_status(dev)
+    cci.pack(W.to(BF16), 8, 2, status=st, check=False)
+    assert cci.read_status(st) == 6
+
+
+@pytest.mark.parametrize("name", ["bottleneck_1x1", "conv3x3_28", "sweep_G32_K8", "resnet_l01"])
+def test_pack_full_workloads(dev, name):
+    if name == "bottleneck_1x1":
+        case = wl.BOTTLENECK_1X1
+        W = wl.draw_w(case.Cout, case.R, case.w_std, case.dtype, case.seed)
+    elif name == "conv3x3_28":
+        case = wl.CONV3X3_28
+        W = wl.draw_w(case.Cout, case.R, case.w_std, case.dtype, case.seed)
+    elif name == "sweep_G32_K8":
+        case = wl.sweep_case(32, 8)
+        W = wl.draw_w(case.Cout, case.R, case.w_std, case.dtype, case.seed)
+    else:
+        case = wl.resnet50_layers(K=2)[1]
+        W = wl.draw_w(case.Cout, case.R, case.w_std, case.dtype, case.seed)
+    v, i = cci.pack(W.to(dev), case.G, case.K)
+    vo, io, _, _ = oracle_reference(W, case.G, case.K)
+    assert_pack_equal(v, i, vo, io)
+
+
+# ---------------------------------------------------------------------------
+# products
+# ---------------------------------------------------------------------------
+def run_linear(dev, X, W, G, K, algo=cci.ALGO_AUTO):
+    Xd, Wd_ = X.to(dev), W.to(dev)
+    v, i = cci.pack(Wd_, G, K)
+    Y = torch.full((X.shape[0], W.shape[0]), float("nan"), device=dev)  # poison: all must be written
+    st = cci.new_status(dev)
+    cci.linear(Xd, v, i, W.shape[0], G, K, out=Y, status=st, algo=algo)
+    assert cci.read_status(st) == 0
+    return Y
+
+
+# (N, Cin, Cout, G, K, dtype): ragged N, N < tile, Cout = G, tiny Cin, and G / K
+# without a register tile (generic kernel)
+SMALL = [
+    (1, 16, 8, 8, 2, "f32"), (33, 64, 64, 4, 2, "f32"), (257, 32, 16, 8, 1, "f32"),
+    (300, 48, 24, 8, 4, "f32"), (1000, 16, 32, 16, 4, "f32"), (77, 64, 64, 32, 8, "f32"),
+    (513, 256, 1024, 8, 2, "f32"), (130, 16, 64, 4, 1, "bf16"), (257, 64, 128, 16, 8, "bf16"),
+    (96, 32, 64, 32, 16, "bf16"), (600, 128, 256, 8, 2, "bf16"), (45, 24, 16, 16, 2, "bf16"),
+    (50, 20, 12, 3, 2, "f32"), (70, 12, 128, 64, 5, "bf16"), (9, 7, 256, 256, 3, "f32"),
+    (65, 40, 16, 2, 1, "bf16"), (31, 64, 32, 8, 8, "f32"), (31, 64, 32, 8, 3, "bf16"),
+]
+
+
+@pytest.mark.parametrize("case", SMALL, ids=lambda c: "N{}_C{}x{}_G{}K{}_{}".format(*c))
+def test_linear_small(dev, case):
+    N, Cin, Cout, G, K, dtype = case
+    X, W = wl.random_small(N + Cin, dtype, N, Cin, Cout)
+    Y = run_linear(dev, X, W, G, K)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, str(case))
+
+
+@pytest.mark.parametrize("case", [c for c in SMALL if c[0] > 1], ids=lambda c: "N{}_C{}x{}_G{}K{}_{}".format(*c))
+def test_regtile_matches_generic_bitwise(dev, case):
+    """Both kernels add the contributions of an output in the same order (ascending
+    r, then slot, one FMA each, from +0), so they agree bit for bit."""
+    N, Cin, Cout, G, K, dtype = case
+    X, W = wl.random_small(N + 7 * Cin, dtype, N, Cin, Cout)
+    Ya = run_linear(dev, X, W, G, K, cci.ALGO_AUTO)
+    Yg = run_linear(dev, X, W, G, K, cci.ALGO_GENERIC)
+    assert torch.equal(Ya.view(torch.int32), Yg.view(torch.int32))
+
+
+def test_linear_tiny_workload(dev):
+    case = wl.TINY_LINEAR
+    X, W = wl.linear_inputs(case)
+    Y = run_linear(dev, X, W, case.G, case.K)
+    _, _, Wd, mask = oracle_reference(W, case.G, case.K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, case.name)
+
+
+def test_linear_bottleneck_full(dev):
+    """N = 100352 columns, 256 -> 1024, G=8, K=2, fp32: every output written;
+    2048 sampled rows against the oracle."""
+    case = wl.BOTTLENECK_1X1
+    X, W = wl.linear_inputs(case)
+    assert cci.kernel_name(F32, case.Cin, case.R, case.Cout, case.G, case.K).startswith("regtile")
+    Y = run_linear(dev, X, W, case.G, case.K)
+    assert torch.isfinite(Y).all()
+    rows = sample_rows(case.N, 2048)
+    _, _, Wd, mask = oracle_reference(W, case.G, case.K)
+    Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name)
+
+
+@pytest.mark.parametrize("G,K", wl.SWEEP_POINTS)
+def test_linear_sweep_full(dev, G, K):
+    """4096 -> 4096, N = 8192, bf16: 192 sampled rows per (G, K) against the oracle."""
+    case = wl.sweep_case(G, K)
+    X, W = wl.linear_inputs(case, device="cpu")
+    Y = run_linear(dev, X, W, G, K)
+    assert torch.isfinite(Y).all()
+    rows = sample_rows(case.N, 192, seed=G * 31 + K)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name)
+
+
+@pytest.mark.parametrize("algo", [cci.ALGO_AUTO, cci.ALGO_GENERIC])
+def test_linear_bad_index_reported(dev, algo):
+    G, K, Cout, Cin, N = 8, 2, 16, 32, 40
+    v = torch.ones((Cout // G, Cin, K), device=dev)
+    i = torch.zeros((Cout // G, Cin, K), dtype=torch.uint8, device=dev)
+    i[..., 1] = 1
+    i[1, 5, 0] = 9  # >= G
+    X = torch.randn(N, Cin, device=dev)
+    st = cci.new_status(dev)
+    cci.linear(X, v, i, Cout, G, K, status=st, algo=algo)
+    assert cci.read_status(st) == 10
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("algo", [cci.ALGO_AUTO, cci.ALGO_GENERIC])
+def test_linear_repeated_and_unordered_indices(dev, dtype, algo):
+    """Packed input not produced by cci_pack: repeated and descending indices are
+    summed as Alg. 2 does (the oracle's decompression sums them too)."""
+    G, K, Cout, Cin, N = 8, 2, 32, 64, 300
+    g = torch.Generator().manual_seed(3)
+    v = torch.randn((Cout // G, Cin, K), generator=g).to(_dt(dtype))
+    i = torch.randint(0, G, (Cout // G, Cin, K), generator=g, dtype=torch.uint8)
+    X = torch.randn((N, Cin), generator=g).to(_dt(dtype))
+    Y = cci.linear(X.to(dev), v.to(dev), i.to(dev), Cout, G, K, algo=algo)
+    Wd, mask = oracle.decompress(f64(v), i.numpy(), Cout, G)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, "repeated indices")
+    Y2 = oracle.linear_alg2(f64(X), f64(v), i.numpy(), Cout, G)
+    assert_within_tol(f64(Y), Y2, S, "repeated indices vs Alg. 2")
+
+
+def test_linear_empty(dev):
+    v, i = cci.pack(torch.randn(16, 32, device=dev), 8, 2)
+    Y = cci.linear(torch.empty((0, 32), device=dev), v, i, 16, 8, 2)
+    assert Y.shape == (0, 16)
+
+
+def test_linear_unaligned_views(dev):
+    """Pointers off the 16-byte grid go to the generic kernel, with the same result."""
+    G, K, Cout, Cin, N = 8, 2, 64, 32, 200
+    X, W = wl.random_small(5, "f32", N + 1, Cin + 1, Cout)
+    Xv = X.to(dev)[1:, 1:]  # not contiguous: make a contiguous copy shifted by one element
+    base = torch.empty(N * Cin + 1, device=dev)
+    base[1:].copy_(Xv.reshape(-1))
+    Xs = base[1:].view(N, Cin)
+    W = W[:, :Cin].contiguous()
+    v, i = cci.pack(W.to(dev), G, K)
+    Y = cci.linear(Xs, v, i, Cout, G, K)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(Xv), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, "unaligned")
+
+
+# ---------------------------------------------------------------------------
+# convolutions
+# ---------------------------------------------------------------------------
+def run_conv(dev, X, W, case_geom, G, K, algo=cci.ALGO_AUTO):
+    KH, KW, stride, pad, Cout = case_geom
+    v, i = cci.pack(W.to(dev), G, K)
+    B, H, Wi, Cin = X.shape
+    P, Q = cci.conv_out_hw(H, Wi, KH, KW, stride, pad)
+    Y = torch.full((B, P, Q, Cout), float("nan"), device=dev)
+    st = cci.new_status(dev)
+    cci.conv2d(X.to(dev), v, i, Cout, G, K, KH, KW, stride, pad, out=Y, status=st, algo=algo)
+    assert cci.read_status(st) == 0
+    return Y
+
+
+# (B, H, W, Cin, Cout, KH, KW, stride, pad, G, K, dtype)
+CONV_SMALL = [
+    (2, 9, 7, 16, 32, 3, 3, (1, 1), (1, 1), 8, 2, "bf16"),
+    (1, 11, 10, 8, 16, 3, 3, (2, 2), (1, 1), 16, 4, "bf16"),
+    (3, 6, 6, 32, 64, 1, 1, (2, 2), (0, 0), 8, 1, "bf16"),
+    (2, 8, 5, 4, 16, 5, 3, (1, 2), (2, 1), 4, 2, "f32"),
+    (1, 7, 7, 64, 128, 3, 3, (1, 1), (0, 0), 32, 8, "f32"),
+    (2, 5, 5, 8, 8, 3, 3, (1, 1), (1, 1), 8, 4, "f32"),
+    (1, 6, 9, 6, 12, 3, 2, (1, 1), (1, 0), 3, 2, "bf16"),  # generic kernel
+    (4, 3, 3, 16, 64, 3, 3, (1, 1), (1, 1), 4, 1, "f32"),
+]
+
+
+@pytest.mark.parametrize("case", CONV_SMALL, ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
+def test_conv_small(dev, case):
+    B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
+    g = torch.Generator().manual_seed(B * 7 + Cin)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(_dt(dtype))
+    W = torch.randn((Cout, KH * KW * Cin), generator=g).to(_dt(dtype))
+    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
+
+
+def test_conv_1x1_equals_linear_bitwise(dev):
+    B, H, Wi, Cin, Cout, G, K = 2, 14, 14, 64, 128, 8, 2
+    X = torch.randn((B, H, Wi, Cin)).to(BF16)
+    W = torch.randn((Cout, Cin)).to(BF16)
+    Yc = run_conv(dev, X, W, (1, 1, (1, 1), (0, 0), Cout), G, K)
+    Yl = run_linear(dev, X.reshape(-1, Cin), W, G, K)
+    assert torch.equal(Yc.reshape(-1, Cout).view(torch.int32), Yl.view(torch.int32))
+
+
+def conv_points(case, k: int, seed: int):
+    """Sampled output positions from the first and last image of the batch."""
+    P, Q = case.P, case.Q
+    per = P * Q
+    rng = np.random.default_rng(seed)
+    first = np.concatenate([np.arange(min(per, k // 4)), rng.choice(per, size=k // 4)])
+    last = (case.B - 1) * per + np.concatenate([np.arange(per - min(per, k // 4), per),
+                                                rng.choice(per, size=k // 4)])
+    return np.unique(np.concatenate([first, last]))
+
+
+def check_conv_case(dev, case, npts=1024, seed=0):
+    X, W = wl.conv_inputs(case, device="cpu")
+    Y = run_conv(dev, X, W, (case.KH, case.KW, (case.stride,) * 2, (case.pad,) * 2, case.Cout),
+                 case.G, case.K)
+    assert torch.isfinite(Y).all()
+    pts = conv_points(case, npts, seed)
+    # oracle on the two images the points come from
+    imgs = [0, case.B - 1] if case.B > 1 else [0]
+    Xs = f64(X[imgs])
+    per = case.P * case.Q
+    local = np.where(pts < per, pts, pts - (case.B - 1) * per + (per if case.B > 1 else 0))
+    _, _, Wd, mask = oracle_reference(W, case.G, case.K)
+    Yo, S = oracle.conv2d(Xs, Wd, mask, case.KH, case.KW, (case.stride,) * 2, (case.pad,) * 2, pts=local)
+    Yg = f64(Y.reshape(-1, case.Cout)[torch.from_numpy(pts).to(dev)])
+    assert_within_tol(Yg, Yo, S, case.name)
+
+
+def test_conv3x3_full(dev):
+    """Batch 64, 28x28, 128 -> 128, 3x3 s1 p1, G=16, K=4, bf16."""
+    case = wl.CONV3X3_28
+    assert cci.kernel_name(BF16, case.Cin, case.R, case.Cout, case.G, case.K).startswith("regtile")
+    check_conv_case(dev, case, npts=2048)
+
+
+RESNET_PICK = [0, 1, 3, 4, 11, 13, 24, 25, 42, 44, 49, 51]
+
+
+@pytest.mark.parametrize("K", [1, 2, 4])
+@pytest.mark.parametrize("li", RESNET_PICK)
+def test_resnet50_layer(dev, li, K):
+    """Layers of the ResNet-50 stack (batch 128), G=8: first/last 1x1, 3x3 s1 and
+    s2, strided downsample 1x1, 14x14 and 7x7 stages."""
+    case = wl.resnet50_layers(K=K)[li]
+    check_conv_case(dev, case, npts=512, seed=li)
