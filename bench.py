@@ -55,6 +55,8 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--extras", type=int, default=1, help="also measure the sweep / conv workloads")
     ap.add_argument("--cpu-sample-seconds", type=float, default=12.0)
+    ap.add_argument("--profile", type=int, default=0,
+                    help="only the warm-up and timed steps of the main path (for ncu)")
     return ap.parse_args()
 
 
@@ -320,6 +322,8 @@ def run_ours(args, rank, world, local):
         torch.cuda.synchronize(dev)
         t_wall = time.perf_counter() - t_wall0
     barrier(world)
+    if args.profile:
+        return 0
     step_ms = [a.elapsed_time(c) for a, b, c in ev]
     lin_ms = [b.elapsed_time(c) for a, b, c in ev]
     pack_ms = [a.elapsed_time(b) for a, b, c in ev]
