@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--cpu-sample-seconds", type=float, default=12.0)
     ap.add_argument("--profile", type=int, default=0,
                     help="only the warm-up and timed steps of the main path (for ncu)")
+    ap.add_argument("--workload", default="bottleneck_1x1",
+                    help="bottleneck_1x1 (default) or sweep_4096_G<G>_K<K>: the product timed")
     return ap.parse_args()
 
 
@@ -271,6 +273,15 @@ def time_device(fn, reps, flush, stream):
     return out
 
 
+def workload_case(name: str) -> wl.LinearCase:
+    if name == wl.BOTTLENECK_1X1.name:
+        return wl.BOTTLENECK_1X1
+    for G, K in wl.SWEEP_POINTS:
+        if name == wl.sweep_case(G, K).name:
+            return wl.sweep_case(G, K)
+    raise SystemExit(f"unknown workload {name}")
+
+
 def run_ours(args, rank, world, local):
     import paper_1910_11971_gb300 as cci
     from paper_1910_11971_gb300 import build as cci_build
@@ -281,7 +292,7 @@ def run_ours(args, rank, world, local):
     stream = torch.cuda.current_stream(dev)
     torch.backends.cuda.matmul.allow_tf32 = False
     torch.backends.cudnn.allow_tf32 = False
-    case = wl.BOTTLENECK_1X1
+    case = workload_case(args.workload)
     X, W = wl.linear_inputs(case, device="cpu")
     X_host = X.pin_memory()
     W_host = W.pin_memory()
@@ -332,15 +343,15 @@ def run_ours(args, rank, world, local):
     nzf = case.nz_flops()
     value = world * nzf / (ms_step * 1e-3) / 1e12
     lin_avg = statistics.mean(lin_ms)
-    kname = cci.kernel_name(torch.float32, case.Cin, case.R, case.Cout, case.G, case.K)
+    kname = cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K)
     achieved = nzf / (lin_avg * 1e-3) / 1e12
     roofline = {"bound": "alu", "achieved": achieved, "peak": ALU_PEAK_TFLOPS, "unit": "TFLOP/s",
                 "frac": achieved / ALU_PEAK_TFLOPS, "traffic": measured_traffic(kname),
                 "kernel": kname,
                 "peak_source": "derived: 152 SMs x 128 FP32 FMA lanes x 2 flop x 2.070 GHz max clock",
                 "algorithmic_flops_per_launch": nzf,
-                "hbm_bytes_per_launch": case.N * case.Cin * 4 + case.N * case.Cout * 4
-                + (case.Cout // case.G) * case.R * case.K * 5}
+                "hbm_bytes_per_launch": case.N * case.Cin * X.element_size() + case.N * case.Cout * 4
+                + (case.Cout // case.G) * case.R * case.K * (X.element_size() + 1)}
 
     # ---- end to end through the public API: host X,W -> device, step, Y -> host ----
     Y_host = torch.empty((case.N, case.Cout), dtype=torch.float32).pin_memory()
@@ -358,7 +369,7 @@ def run_ours(args, rank, world, local):
     e2e_ms = statistics.mean(time_device(e2e_step, max(3, args.steps // 4), flush, stream))
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
     e2e = {"value": world * nzf / (e2e_ms * 1e-3) / 1e12, "unit": UNIT,
-           "h2d_bytes_per_step": X_host.numel() * 4 + W_host.numel() * 4,
+           "h2d_bytes_per_step": X_host.numel() * X_host.element_size() + W_host.numel() * W_host.element_size(),
            "d2h_bytes_per_step": Y_host.numel() * 4, "ms_per_step": e2e_ms}
 
     # ---- dense reference line: cuBLAS fp32 (TF32 off) on the masked dense weights ----
