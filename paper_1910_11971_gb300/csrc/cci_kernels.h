@@ -12,7 +12,7 @@ cudaError_t launch_fma_probe(float *out, int blocks, int threads, int iters, cud
 
 // One register-tiled instantiation: (dtype, G, K) -> tile shape and launcher.
 struct RegtileEntry {
-    int dtype, G, K, MG, T;
+    int dtype, G, K, MG, T, D;
     const char *name;
     cudaError_t (*launch)(const FwdParams &p, cudaStream_t stream);
 };

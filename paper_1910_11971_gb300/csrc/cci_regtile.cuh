@@ -4,55 +4,32 @@
 // loop for K > 1) for a product or an implicit convolution.
 //
 // Work split (the group-boundary split of Sec. 3.2: a CTA owns whole groups):
-//   * a CTA of 8 warps owns CH = WC*MG*G output channels (WC warps across
-//     channels, each owning MG whole groups) and NTC = WN*32*T columns (WN = 8/WC
-//     warps across columns);
+//   * a CTA of 8 warps owns WC*MG whole groups (WC warps across channels, each
+//     owning MG groups) and NTC = (8/WC)*32*T columns (8/WC warps across columns);
 //   * lane l of a warp owns T columns: 4-column runs at l*4 + q*128, q < T/4;
-//   * every lane of a warp sees the same (value, index) pair at the same time
-//     (the index depends on (group, r, slot), not on the column), so the index
-//     choice of Alg. 2 is a warp-uniform branch, and the MG*G x T accumulator
-//     block stays in registers ("load a whole group of elements of H onto
+//   * the index of a slot depends on (group, r, slot), not on the column, so all
+//     lanes of a warp take the same index at the same time: the choice of the
+//     output row in Alg. 2 is one warp-uniform jump (generated PTX brx.idx, see
+//     cci_dispatch.cuh) into straight-line packed FMAs, and the MG*G x T block of
+//     outputs stays in registers ("load a whole group of elements of H onto
 //     on-chip registers", Sec. 3.2);
-//   * two columns share one packed FMA (fma.rn.f32x2), so a slot costs T/2 FMA
-//     instructions per lane.
+//   * two columns share one packed FMA (fma.rn.f32x2).
 //
-// Pipeline per chunk of RC reduction indices:
+// Pipeline per chunk of RC = 16 reduction indices:
 //   raw X tile [NTC][RC] and raw (value, index) runs are copied global->shared
 //   with cp.async one chunk ahead (no registers held); the chunk is then
-//   transposed to an fp32 [RC][NTC] tile (bf16 widened exactly) and the slots are
-//   decoded into {v, v} pairs plus one dispatch code per (group, r): the colex
-//   rank of the ascending index set among all K-subsets of [0, G) when there are
-//   at most 128 subsets, else the raw indices.  A non-ascending or repeated index
-//   set takes a per-slot path, so any index set is summed as Alg. 2 does.
-//   Per output channel the contributions arrive in ascending r (then slot), each
-//   one fused multiply-add, starting from +0.
+//   transposed to an fp32 [RC][NTC] tile (bf16 widened exactly) and each
+//   (group, r) gets a record of 16-byte units: K fp32 values, then the dispatch
+//   words (D = 1: the indices, 4 per word; D = 2: per slot pair the colex rank
+//   of the ascending pair in bits 0-7 and the raw indices in bits 8-23).
+//   Per output channel the contributions arrive in ascending r (then slot), one
+//   fused multiply-add each, starting from +0.
 #pragma once
 
 #include "cci_common.cuh"
+#include "cci_dispatch.cuh"
 
 namespace cci {
-
-__host__ __device__ constexpr int binom(int n, int k)
-{
-    if (k < 0 || k > n) return 0;
-    long long r = 1;
-    for (int i = 1; i <= k; ++i) r = r * (n - k + i) / i;
-    return static_cast<int>(r);
-}
-
-// Element s (ascending) of the K-subset of [0, G) whose colex rank is c, where
-// rank(i_0 < ... < i_{K-1}) = sum_s binom(i_s, s + 1).
-__host__ __device__ constexpr int colex_element(int c, int K, int s)
-{
-    int out = 0;
-    for (int t = K - 1; t >= 0; --t) {
-        int i = t;
-        while (binom(i + 1, t + 1) <= c) ++i;
-        c -= binom(i, t + 1);
-        if (t == s) out = i;
-    }
-    return out;
-}
 
 template <typename TS>
 struct Elem;
@@ -83,183 +60,73 @@ __device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool va
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;\n" ::: "memory"); }
 
-template <typename TS, int G, int K, int MG, int T>
+__host__ __device__ constexpr size_t round16(size_t b) { return (b + 15) / 16 * 16; }
+
+template <typename TS, int G, int K, int MG, int T, int D, int WC>
 struct RegTile {
     static constexpr int kThreads = 256;
-    static constexpr int kWarps = 8;
-    static constexpr int kRC = 16;          // reduction indices per chunk
+    static constexpr int kRC = 16;                        // reduction indices per chunk
     static constexpr int kVec = Elem<TS>::kVec;
-    static constexpr int kNC = binom(G, K);
-    static constexpr bool kCombo = kNC <= 128;
-    static constexpr int kSlotsRC = kRC * K;  // slots of one group in a chunk
+    static constexpr int kWN = 8 / WC;                    // column-warps
+    static constexpr int kNTC = kWN * 32 * T;             // columns per CTA
+    static constexpr int kNGR = WC * MG;                  // groups per CTA
+    static constexpr int kSlots = kRC * K;                // slots of one group in a chunk
+    static constexpr int kDisp = K / D;                   // jumps per (group, r)
+    static constexpr int kWords = D > 1 ? kDisp : (K + 3) / 4;
+    static constexpr int kRecVec = static_cast<int>(round16(4 * K + 4 * kWords) / 16);
+    static constexpr int kXPitch = kRC + 16 / static_cast<int>(sizeof(TS));
+    static_assert(WC == 4 || WC == 8, "4 or 8 channel-warps");
+    static_assert(D == 1 || (D == 2 && K % 2 == 0), "one or two slots per jump");
     static_assert(T % 4 == 0, "T must be a multiple of 4");
     static_assert(kRC % kVec == 0, "a chunk must hold whole 16-byte vectors");
-    static_assert((kSlotsRC * static_cast<int>(sizeof(TS))) % 16 == 0, "value runs must be 16-byte multiples");
-    static_assert(kSlotsRC % 16 == 0, "index runs must be 16-byte multiples");
+    static_assert((kSlots * static_cast<int>(sizeof(TS))) % 16 == 0, "value runs must be 16-byte multiples");
+    static_assert(kSlots % 16 == 0, "index runs must be 16-byte multiples");
     static_assert((MG * G) % 4 == 0, "output rows are stored as float4");
 
     // shared-memory layout (byte offsets; every part 16-byte aligned)
-    struct Layout {
-        int ntc;         // columns per CTA
-        int ngroups;     // groups per CTA = WC * MG
-        int xpitch;      // elements per raw X row (RC + 16 bytes of padding)
-        size_t xraw, xs, vraw, iraw, vv, code, sidx, sites, total;
-    };
-
-    __host__ __device__ static Layout layout(int wc)
-    {
-        Layout L{};
-        L.ntc = (kWarps / wc) * 32 * T;
-        L.ngroups = wc * MG;
-        L.xpitch = kRC + 16 / static_cast<int>(sizeof(TS));
-        size_t off = 0;
-        auto take = [&off](size_t bytes) {
-            const size_t o = off;
-            off += (bytes + 15) / 16 * 16;
-            return o;
-        };
-        L.xraw = take(2ull * L.ntc * L.xpitch * sizeof(TS));
-        L.xs = take(2ull * kRC * L.ntc * sizeof(float));
-        L.vraw = take(2ull * L.ngroups * kSlotsRC * sizeof(TS));
-        L.iraw = take(2ull * L.ngroups * kSlotsRC);
-        L.vv = take(2ull * L.ngroups * kSlotsRC * sizeof(unsigned long long));
-        L.code = take(2ull * L.ngroups * kRC);
-        L.sidx = take(2ull * L.ngroups * kSlotsRC);
-        L.sites = take(static_cast<size_t>(L.ntc) * sizeof(int4));
-        L.total = off;
-        return L;
-    }
+    static constexpr size_t kXraw = 0;
+    static constexpr size_t kXs = kXraw + round16(2ull * kNTC * kXPitch * sizeof(TS));
+    static constexpr size_t kVraw = kXs + round16(2ull * kRC * kNTC * sizeof(float));
+    static constexpr size_t kIraw = kVraw + round16(2ull * kNGR * kSlots * sizeof(TS));
+    static constexpr size_t kRec = kIraw + round16(2ull * kNGR * kSlots);
+    static constexpr size_t kSites = kRec + round16(2ull * kNGR * kRC * kRecVec * 16);
+    static constexpr size_t kTotal = kSites + round16(static_cast<size_t>(kNTC) * sizeof(int4));
 };
 
-// ---------------------------------------------------------------------------
-// slot application: acc[g][i][*] += x * v for a compile-time index i
-// ---------------------------------------------------------------------------
-template <int T, int G, int MG>
-struct Acc {
-    unsigned long long a[MG][G][T / 2];
-};
-
-template <int T, int G, int MG, int g, int i>
-__device__ __forceinline__ void apply_slot(Acc<T, G, MG> &acc, const unsigned long long (&xx)[T / 2],
-                                           unsigned long long v)
+__device__ __forceinline__ uint32_t word_of(const uint4 &u, int k)
 {
-#pragma unroll
-    for (int t = 0; t < T / 2; ++t) ffma2(acc.a[g][i][t], xx[t], v);
-}
-
-template <int T, int G, int MG, int g, int K, int c, int s = 0>
-__device__ __forceinline__ void apply_combo(Acc<T, G, MG> &acc, const unsigned long long (&xx)[T / 2],
-                                            const unsigned long long (&vv)[K])
-{
-    if constexpr (s < K) {
-        constexpr int i = colex_element(c, K, s);
-        apply_slot<T, G, MG, g, i>(acc, xx, vv[s]);
-        apply_combo<T, G, MG, g, K, c, s + 1>(acc, xx, vv);
-    }
-}
-
-#define CCI_CASE(c, BODY) \
-    case (c):             \
-        BODY(c);          \
-        break;
-#define CCI_CASES4(b, BODY) CCI_CASE(b, BODY) CCI_CASE(b + 1, BODY) CCI_CASE(b + 2, BODY) CCI_CASE(b + 3, BODY)
-#define CCI_CASES16(b, BODY) \
-    CCI_CASES4(b, BODY) CCI_CASES4(b + 4, BODY) CCI_CASES4(b + 8, BODY) CCI_CASES4(b + 12, BODY)
-#define CCI_CASES64(b, BODY) \
-    CCI_CASES16(b, BODY) CCI_CASES16(b + 16, BODY) CCI_CASES16(b + 32, BODY) CCI_CASES16(b + 48, BODY)
-#define CCI_CASES128(b, BODY) CCI_CASES64(b, BODY) CCI_CASES64(b + 64, BODY)
-
-// one slot with a run-time (warp-uniform) index: a G-way branch
-template <int T, int G, int MG, int g>
-__device__ __forceinline__ void apply_single(Acc<T, G, MG> &acc, const unsigned long long (&xx)[T / 2],
-                                             unsigned long long v, int i)
-{
-#define CCI_SINGLE_BODY(c)                                         \
-    if constexpr ((c) < G) {                                       \
-        apply_slot<T, G, MG, g, ((c) < G ? (c) : 0)>(acc, xx, v); \
-    }
-    switch (i) {
-        CCI_CASES128(0, CCI_SINGLE_BODY)
-        default:
-            break;
-    }
-#undef CCI_SINGLE_BODY
-}
-
-template <int T, int G, int MG, int g, int K>
-__device__ __forceinline__ void apply_group(Acc<T, G, MG> &acc, const unsigned long long (&xx)[T / 2],
-                                            const unsigned long long (&vv)[K], int code,
-                                            const uint8_t *sidx)
-{
-    constexpr int NC = binom(G, K);
-    if constexpr (NC <= 128) {
-#define CCI_COMBO_BODY(c)                                               \
-    if constexpr ((c) < NC) {                                           \
-        apply_combo<T, G, MG, g, K, ((c) < NC ? (c) : 0)>(acc, xx, vv); \
-    } else if constexpr ((c) == NC) {                                   \
-        _Pragma("unroll") for (int s = 0; s < K; ++s)                   \
-            apply_single<T, G, MG, g>(acc, xx, vv[s], sidx[s]);         \
-    }
-        switch (code) {
-            CCI_CASES128(0, CCI_COMBO_BODY)
-            CCI_CASE(128, CCI_COMBO_BODY)
-            default:
-                break;
-        }
-#undef CCI_COMBO_BODY
-    } else {
-#pragma unroll
-        for (int s = 0; s < K; ++s) apply_single<T, G, MG, g>(acc, xx, vv[s], sidx[s]);
-    }
-}
-
-// all MG groups of the warp at one reduction index r; the pointers are at
-// (group 0, r) and advance by `gstride_*` per group
-template <int T, int G, int MG, int K, int g = 0>
-__device__ __forceinline__ void apply_all_groups(Acc<T, G, MG> &acc, const unsigned long long (&xx)[T / 2],
-                                                 const unsigned long long *vv_r, const uint8_t *code_r,
-                                                 const uint8_t *sidx_r, int gstride_code, int gstride_slot)
-{
-    if constexpr (g < MG) {
-        unsigned long long vv[K];
-#pragma unroll
-        for (int s = 0; s < K; ++s) vv[s] = vv_r[g * gstride_slot + s];
-        const int code = code_r[g * gstride_code];
-        apply_group<T, G, MG, g, K>(acc, xx, vv, code, sidx_r + g * gstride_slot);
-        apply_all_groups<T, G, MG, K, g + 1>(acc, xx, vv_r, code_r, sidx_r, gstride_code, gstride_slot);
-    }
+    return k == 0 ? u.x : k == 1 ? u.y : k == 2 ? u.z : u.w;
 }
 
 // ---------------------------------------------------------------------------
 // the kernel: persistent over tiles (tile = channel tile fastest, so the CTAs
 // running at the same time share column tiles and X is reused through L2)
 // ---------------------------------------------------------------------------
-template <typename TS, int G, int K, int MG, int T>
-__global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, int64_t n_ct, int64_t n_tiles)
+template <typename TS, int G, int K, int MG, int T, int D, int WC>
+__global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_ct, int64_t n_tiles)
 {
-    using RT = RegTile<TS, G, K, MG, T>;
+    using RT = RegTile<TS, G, K, MG, T, D, WC>;
     constexpr int RC = RT::kRC;
     constexpr int VEC = RT::kVec;
-    constexpr int SLOTS = RT::kSlotsRC;
+    constexpr int NTC = RT::kNTC;
+    constexpr int NGR = RT::kNGR;
+    constexpr int SLOTS = RT::kSlots;
+    constexpr int XP = RT::kXPitch;
+    constexpr int RV = RT::kRecVec;
+    constexpr int H = T / 2;
     extern __shared__ __align__(16) unsigned char smem[];
-    const auto L = RT::layout(wc);
-    TS *xraw = reinterpret_cast<TS *>(smem + L.xraw);
-    float *xs = reinterpret_cast<float *>(smem + L.xs);
-    TS *vraw = reinterpret_cast<TS *>(smem + L.vraw);
-    uint8_t *iraw = smem + L.iraw;
-    unsigned long long *vvs = reinterpret_cast<unsigned long long *>(smem + L.vv);
-    uint8_t *codes = smem + L.code;
-    uint8_t *sidx = smem + L.sidx;
-    int4 *sites = reinterpret_cast<int4 *>(smem + L.sites);
+    TS *xraw = reinterpret_cast<TS *>(smem + RT::kXraw);
+    float *xs = reinterpret_cast<float *>(smem + RT::kXs);
+    TS *vraw = reinterpret_cast<TS *>(smem + RT::kVraw);
+    uint8_t *iraw = smem + RT::kIraw;
+    uint4 *rec = reinterpret_cast<uint4 *>(smem + RT::kRec);
+    int4 *sites = reinterpret_cast<int4 *>(smem + RT::kSites);
 
     const int tid = threadIdx.x;
     const int lane = tid & 31;
     const int warp = tid >> 5;
-    const int wcw = warp % wc;  // channel-warp index
-    const int wnw = warp / wc;  // column-warp index
-    const int ntc = L.ntc;
-    const int ngr = L.ngroups;
-    const int xpitch = L.xpitch;
+    const int wcw = warp % WC;  // channel-warp index
+    const int wnw = warp / WC;  // column-warp index
     const int64_t total_groups = p.Cout / G;
     const int nchunks = static_cast<int>((p.R + RC - 1) / RC);
     const TS *X = static_cast<const TS *>(p.X);
@@ -267,11 +134,11 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, in
 
     for (int64_t tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
         const int64_t ct = tile % n_ct;
-        const int64_t n0 = (tile / n_ct) * ntc;
-        const int64_t g0 = ct * ngr;  // first group of the CTA
+        const int64_t n0 = (tile / n_ct) * NTC;
+        const int64_t g0 = ct * NGR;  // first group of the CTA
 
         // column sites: {img lo, img hi (-1: column past N), hb, wb}
-        for (int c = tid; c < ntc; c += RT::kThreads) {
+        for (int c = tid; c < NTC; c += RT::kThreads) {
             const int64_t n = n0 + c;
             int4 s = make_int4(0, -1, 0, 0);
             if (n < p.N) {
@@ -286,38 +153,40 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, in
         auto issue_chunk = [&](int chunk) {
             const int buf = chunk & 1;
             const int64_t r0 = static_cast<int64_t>(chunk) * RC;
-            TS *xr = xraw + static_cast<size_t>(buf) * ntc * xpitch;
-            const int nvec = ntc * (RC / VEC);
-            for (int v = tid; v < nvec; v += RT::kThreads) {
-                const int col = v % ntc;
-                const int rv = v / ntc;
-                const int64_t r = r0 + rv * VEC;
-                const int4 s = sites[col];
-                bool ok = (s.y >= 0) && (r < p.R);
-                const TS *src = X;
-                if (ok) {
-                    const int64_t img = (static_cast<int64_t>(s.y) << 32) | static_cast<uint32_t>(s.x);
-                    if (!p.is_conv) {
-                        src = X + img + r;
-                    } else {
-                        const int64_t tap = r / p.Cin;
-                        const int64_t ci = r - tap * p.Cin;
-                        const int kh = static_cast<int>(tap / p.KW);
-                        const int kw = static_cast<int>(tap - static_cast<int64_t>(kh) * p.KW);
-                        const int h = s.z + kh, w = s.w + kw;
-                        ok = (h >= 0) && (h < p.H) && (w >= 0) && (w < p.W);
-                        if (ok) src = X + img + (static_cast<int64_t>(h) * p.W + w) * p.Cin + ci;
+            TS *xr = xraw + buf * (NTC * XP);
+#pragma unroll
+            for (int it = 0; it < (NTC * (RC / VEC) + RT::kThreads - 1) / RT::kThreads; ++it) {
+                const int v = it * RT::kThreads + tid;
+                if (v < NTC * (RC / VEC)) {
+                    const int col = v % NTC;
+                    const int rv = v / NTC;
+                    const int64_t r = r0 + rv * VEC;
+                    const int4 s = sites[col];
+                    bool ok = (s.y >= 0) && (r < p.R);
+                    const TS *src = X;
+                    if (ok) {
+                        const int64_t img = (static_cast<int64_t>(s.y) << 32) | static_cast<uint32_t>(s.x);
+                        if (!p.is_conv) {
+                            src = X + img + r;
+                        } else {
+                            const int64_t tap = r / p.Cin;
+                            const int64_t ci = r - tap * p.Cin;
+                            const int kh = static_cast<int>(tap / p.KW);
+                            const int kw = static_cast<int>(tap - static_cast<int64_t>(kh) * p.KW);
+                            const int h = s.z + kh, w = s.w + kw;
+                            ok = (h >= 0) && (h < p.H) && (w >= 0) && (w < p.W);
+                            if (ok) src = X + img + (static_cast<int64_t>(h) * p.W + w) * p.Cin + ci;
+                        }
                     }
+                    cp_async16(xr + col * XP + rv * VEC, src, ok);
                 }
-                cp_async16(xr + static_cast<size_t>(col) * xpitch + rv * VEC, src, ok);
             }
-            TS *vr = vraw + static_cast<size_t>(buf) * ngr * SLOTS;
-            uint8_t *ir = iraw + static_cast<size_t>(buf) * ngr * SLOTS;
-            constexpr int VPG = SLOTS * static_cast<int>(sizeof(TS)) / 16;  // value vectors per group
-            constexpr int EPV = 16 / static_cast<int>(sizeof(TS));          // values per vector
-            constexpr int IPG = SLOTS / 16;                                 // index vectors per group
-            const int nsv = ngr * (VPG + IPG);
-            for (int v = tid; v < nsv; v += RT::kThreads) {
+            TS *vr = vraw + buf * (NGR * SLOTS);
+            uint8_t *ir = iraw + buf * (NGR * SLOTS);
+            constexpr int EPV = 16 / static_cast<int>(sizeof(TS));  // values per 16 bytes
+            constexpr int VPG = SLOTS / EPV;                          // value vectors per group
+            constexpr int IPG = SLOTS / 16;                           // index vectors per group
+            for (int v = tid; v < NGR * (VPG + IPG); v += RT::kThreads) {
                 const int gl = v / (VPG + IPG);
                 const int part = v % (VPG + IPG);
                 const int64_t gg = g0 + gl;
@@ -337,34 +206,35 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, in
         auto transform_chunk = [&](int chunk) {
             const int buf = chunk & 1;
             const int64_t r0 = static_cast<int64_t>(chunk) * RC;
-            const TS *xr = xraw + static_cast<size_t>(buf) * ntc * xpitch;
-            float *xo = xs + static_cast<size_t>(buf) * RC * ntc;
-            const int nvec = ntc * (RC / VEC);
-            for (int v = tid; v < nvec; v += RT::kThreads) {
-                const int col = v % ntc;
-                const int rv = v / ntc;
-                const uint4 w4 = *reinterpret_cast<const uint4 *>(xr + static_cast<size_t>(col) * xpitch + rv * VEC);
-                const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
+            const TS *xr = xraw + buf * (NTC * XP);
+            float *xo = xs + buf * (RC * NTC);
 #pragma unroll
-                for (int e = 0; e < VEC; ++e)
-                    xo[static_cast<size_t>(rv * VEC + e) * ntc + col] = Elem<TS>::widen(w, e);
+            for (int it = 0; it < (NTC * (RC / VEC) + RT::kThreads - 1) / RT::kThreads; ++it) {
+                const int v = it * RT::kThreads + tid;
+                if (v < NTC * (RC / VEC)) {
+                    const int col = v % NTC;
+                    const int rv = v / NTC;
+                    const uint4 w4 = *reinterpret_cast<const uint4 *>(xr + col * XP + rv * VEC);
+                    const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e) xo[(rv * VEC + e) * NTC + col] = Elem<TS>::widen(w, e);
+                }
             }
-            const TS *vr = vraw + static_cast<size_t>(buf) * ngr * SLOTS;
-            const uint8_t *ir = iraw + static_cast<size_t>(buf) * ngr * SLOTS;
-            unsigned long long *vo = vvs + static_cast<size_t>(buf) * ngr * SLOTS;
-            uint8_t *co = codes + static_cast<size_t>(buf) * ngr * RC;
-            uint8_t *so = sidx + static_cast<size_t>(buf) * ngr * SLOTS;
-            const int nitems = ngr * RC;
-            for (int it = tid; it < nitems; it += RT::kThreads) {
-                const int gl = it / RC;
-                const int r = it % RC;
+            const TS *vr = vraw + buf * (NGR * SLOTS);
+            const uint8_t *ir = iraw + buf * (NGR * SLOTS);
+            uint4 *ro = rec + buf * (NGR * RC * RV);
+            for (int item = tid; item < NGR * RC; item += RT::kThreads) {
+                const int gl = item / RC;
+                const int r = item % RC;
                 const bool live = (g0 + gl < total_groups) && (r0 + r < p.R);
-                int code = 0, prev = -1;
-                bool canon = true;
+                uint32_t words[RV * 4];
+#pragma unroll
+                for (int k = 0; k < RV * 4; ++k) words[k] = 0;
+                int idxs[K];
 #pragma unroll
                 for (int s = 0; s < K; ++s) {
                     float v = 0.0f;
-                    int i = s;  // padding: value 0 on the index set {0..K-1}
+                    int i = s % G;  // padding: value 0 on an ascending index set
                     if (live) {
                         v = Elem<TS>::to_f32(vr[gl * SLOTS + r * K + s]);
                         i = ir[gl * SLOTS + r * K + s];
@@ -374,30 +244,42 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, in
                             i = 0;
                         }
                     }
-                    canon = canon && (i > prev);
-                    prev = i;
-                    code += binom(i, s + 1);
-                    vo[gl * SLOTS + r * K + s] = pack2(v, v);
-                    so[gl * SLOTS + r * K + s] = static_cast<uint8_t>(i);
+                    words[s] = __float_as_uint(v);
+                    idxs[s] = i;
                 }
-                co[gl * RC + r] = static_cast<uint8_t>(canon ? code : RT::kNC);
+                if constexpr (D == 1) {
+#pragma unroll
+                    for (int s = 0; s < K; ++s) words[K + s / 4] |= static_cast<uint32_t>(idxs[s]) << (8 * (s % 4));
+                } else {
+#pragma unroll
+                    for (int d = 0; d < K / 2; ++d) {
+                        const int i0 = idxs[2 * d], i1 = idxs[2 * d + 1];
+                        const uint32_t code = (i0 < i1) ? static_cast<uint32_t>(i0 + i1 * (i1 - 1) / 2)
+                                                        : static_cast<uint32_t>(G * (G - 1) / 2);
+                        words[K + d] = code | (static_cast<uint32_t>(i0) << 8) | (static_cast<uint32_t>(i1) << 16);
+                    }
+                }
+                uint4 *dst = ro + (gl * RC + r) * RV;
+#pragma unroll
+                for (int q = 0; q < RV; ++q)
+                    dst[q] = make_uint4(words[4 * q], words[4 * q + 1], words[4 * q + 2], words[4 * q + 3]);
             }
         };
 
-        Acc<T, G, MG> acc;
+        unsigned long long acc[MG][G][H];
 #pragma unroll
         for (int g = 0; g < MG; ++g)
 #pragma unroll
             for (int i = 0; i < G; ++i)
 #pragma unroll
-                for (int t = 0; t < T / 2; ++t) acc.a[g][i][t] = 0ull;
+                for (int t = 0; t < H; ++t) acc[g][i][t] = 0ull;
 
         // Buffer safety (b = chunk parity):
         //  * issue(c+1) writes raw[b'] last read by transform(c-1): separated by the
         //    barriers of iteration c-1;
-        //  * transform(c+1) writes proc[b'] last read by compute(c-1): separated by
+        //  * transform(c+1) writes xs/rec[b'] last read by compute(c-1): separated by
         //    the barrier before compute(c);
-        //  * compute(c) reads proc[b] written by transform(c): barrier before compute.
+        //  * compute(c) reads xs/rec[b] written by transform(c): barrier before compute.
         issue_chunk(0);
         cp_async_wait_all();
         __syncthreads();
@@ -406,21 +288,54 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, in
             if (c + 1 < nchunks) issue_chunk(c + 1);
             __syncthreads();
             const int buf = c & 1;
-            const float *xo = xs + static_cast<size_t>(buf) * RC * ntc + wnw * (32 * T) + lane * 4;
-            const int gw0 = wcw * MG;  // first CTA-local group of this warp
-            const unsigned long long *vo = vvs + static_cast<size_t>(buf) * ngr * SLOTS + gw0 * SLOTS;
-            const uint8_t *co = codes + static_cast<size_t>(buf) * ngr * RC + gw0 * RC;
-            const uint8_t *so = sidx + static_cast<size_t>(buf) * ngr * SLOTS + gw0 * SLOTS;
-#pragma unroll 1
-            for (int r = 0; r < RC; ++r) {
-                unsigned long long xx[T / 2];
+            const float *xw = xs + buf * (RC * NTC) + wnw * (32 * T) + lane * 4;
+            const uint4 *rw = rec + buf * (NGR * RC * RV) + wcw * MG * RC * RV;
+
+            unsigned long long xx[H];
+            uint4 rc[MG][RV];
+            auto load_r = [&](int r, unsigned long long (&xo)[H], uint4 (&ro)[MG][RV]) {
 #pragma unroll
                 for (int q = 0; q < T / 4; ++q) {
-                    const ulonglong2 u = *reinterpret_cast<const ulonglong2 *>(xo + r * ntc + q * 128);
-                    xx[2 * q] = u.x;
-                    xx[2 * q + 1] = u.y;
+                    const ulonglong2 u = *reinterpret_cast<const ulonglong2 *>(xw + r * NTC + q * 128);
+                    xo[2 * q] = u.x;
+                    xo[2 * q + 1] = u.y;
                 }
-                apply_all_groups<T, G, MG, K>(acc, xx, vo + r * K, co + r, so + r * K, RC, SLOTS);
+#pragma unroll
+                for (int g = 0; g < MG; ++g)
+#pragma unroll
+                    for (int q = 0; q < RV; ++q) ro[g][q] = rw[(g * RC + r) * RV + q];
+            };
+            load_r(0, xx, rc);
+#pragma unroll 1
+            for (int r = 0; r < RC; ++r) {
+                unsigned long long xn[H];
+                uint4 rn[MG][RV];
+                load_r(r + 1 < RC ? r + 1 : r, xn, rn);  // prefetch the next reduction index
+#pragma unroll
+                for (int g = 0; g < MG; ++g) {
+#pragma unroll
+                    for (int d = 0; d < K / D; ++d) {
+                        unsigned long long vv[D];
+#pragma unroll
+                        for (int s = 0; s < D; ++s) {
+                            const float v = __uint_as_float(word_of(rc[g][(d * D + s) / 4], (d * D + s) % 4));
+                            vv[s] = pack2(v, v);
+                        }
+                        uint32_t word;
+                        if constexpr (D == 1) {
+                            word = (word_of(rc[g][(K + d / 4) / 4], (K + d / 4) % 4) >> (8 * (d % 4))) & 0xffu;
+                        } else {
+                            word = word_of(rc[g][(K + d) / 4], (K + d) % 4);
+                        }
+                        Dispatch<G, D, T>::run(acc[g], xx, vv, word);
+                    }
+                }
+#pragma unroll
+                for (int t = 0; t < H; ++t) xx[t] = xn[t];
+#pragma unroll
+                for (int g = 0; g < MG; ++g)
+#pragma unroll
+                    for (int q = 0; q < RV; ++q) rc[g][q] = rn[g][q];
             }
             if (c + 1 < nchunks) {
                 cp_async_wait_all();
@@ -432,7 +347,7 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, in
         // epilogue: Y[n][c0 .. c0 + MG*G) for this lane's T columns
         const int64_t gfirst = g0 + wcw * MG;
 #pragma unroll
-        for (int t2 = 0; t2 < T / 2; ++t2) {
+        for (int t2 = 0; t2 < H; ++t2) {
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
                 const int col = wnw * (32 * T) + (t2 >> 1) * 128 + lane * 4 + (t2 & 1) * 2 + e;
@@ -446,10 +361,10 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int wc, in
 #pragma unroll
                     for (int i4 = 0; i4 < G / 4; ++i4) {
                         float4 o;
-                        o.x = e ? hi_of(acc.a[g][4 * i4 + 0][t2]) : lo_of(acc.a[g][4 * i4 + 0][t2]);
-                        o.y = e ? hi_of(acc.a[g][4 * i4 + 1][t2]) : lo_of(acc.a[g][4 * i4 + 1][t2]);
-                        o.z = e ? hi_of(acc.a[g][4 * i4 + 2][t2]) : lo_of(acc.a[g][4 * i4 + 2][t2]);
-                        o.w = e ? hi_of(acc.a[g][4 * i4 + 3][t2]) : lo_of(acc.a[g][4 * i4 + 3][t2]);
+                        o.x = e ? hi_of(acc[g][4 * i4 + 0][t2]) : lo_of(acc[g][4 * i4 + 0][t2]);
+                        o.y = e ? hi_of(acc[g][4 * i4 + 1][t2]) : lo_of(acc[g][4 * i4 + 1][t2]);
+                        o.z = e ? hi_of(acc[g][4 * i4 + 2][t2]) : lo_of(acc[g][4 * i4 + 2][t2]);
+                        o.w = e ? hi_of(acc[g][4 * i4 + 3][t2]) : lo_of(acc[g][4 * i4 + 3][t2]);
                         __stcs(yg + i4, o);
                     }
                 }

@@ -14,38 +14,39 @@ inline int device_sm_count()
     return sms > 0 ? sms : 1;
 }
 
-template <typename TS, int G, int K, int MG, int T>
-cudaError_t launch_regtile(const FwdParams &p, cudaStream_t stream)
+template <typename TS, int G, int K, int MG, int T, int D, int WC>
+cudaError_t launch_regtile_wc(const FwdParams &p, cudaStream_t stream)
 {
-    using RT = RegTile<TS, G, K, MG, T>;
-    auto kern = regtile_kernel<TS, G, K, MG, T>;
-    // opt in to the largest layout any channel split uses, once per process
-    static const cudaError_t attr = [kern] {
-        const size_t most = RT::layout(4).total > RT::layout(8).total ? RT::layout(4).total : RT::layout(8).total;
-        if (most > kMaxSmemPerBlock) return cudaErrorInvalidConfiguration;
-        return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(most));
-    }();
+    using RT = RegTile<TS, G, K, MG, T, D, WC>;
+    static_assert(RT::kTotal <= kMaxSmemPerBlock, "shared-memory layout over the per-block limit");
+    auto kern = regtile_kernel<TS, G, K, MG, T, D, WC>;
+    static const cudaError_t attr =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(RT::kTotal));
     if (attr != cudaSuccess) return attr;
     const int64_t groups = p.Cout / G;
-    const int wc = regtile_wc(groups, MG);
-    const auto L = RT::layout(wc);
-    if (L.total > kMaxSmemPerBlock) return cudaErrorInvalidConfiguration;
-    const int64_t n_ct = (groups + L.ngroups - 1) / L.ngroups;
-    const int64_t n_nt = (p.N + L.ntc - 1) / L.ntc;
+    const int64_t n_ct = (groups + RT::kNGR - 1) / RT::kNGR;
+    const int64_t n_nt = (p.N + RT::kNTC - 1) / RT::kNTC;
     const int64_t n_tiles = n_ct * n_nt;
     int per_sm = 0;
-    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, RT::kThreads, L.total);
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, RT::kThreads, RT::kTotal);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) per_sm = 1;
     const int64_t resident = static_cast<int64_t>(device_sm_count()) * per_sm;
     const unsigned grid = static_cast<unsigned>(n_tiles < resident ? n_tiles : resident);
-    kern<<<grid, RT::kThreads, L.total, stream>>>(p, wc, n_ct, n_tiles);
+    kern<<<grid, RT::kThreads, RT::kTotal, stream>>>(p, n_ct, n_tiles);
     return cudaGetLastError();
+}
+
+template <typename TS, int G, int K, int MG, int T, int D>
+cudaError_t launch_regtile(const FwdParams &p, cudaStream_t stream)
+{
+    if (regtile_wc(p.Cout / G, MG) == 8) return launch_regtile_wc<TS, G, K, MG, T, D, 8>(p, stream);
+    return launch_regtile_wc<TS, G, K, MG, T, D, 4>(p, stream);
 }
 
 }  // namespace cci
 
-// table row for one instantiation (dtype tag, storage type, G, K, MG, T)
-#define CCI_REGTILE_ROW(DT, TS, G, K, MG, T)                                                       \
-    {DT, G, K, MG, T, "regtile_" #TS "_G" #G "_K" #K "_MG" #MG "_T" #T,                             \
-     &cci::launch_regtile<TS, G, K, MG, T>},
+// table row for one instantiation (dtype tag, storage type, G, K, MG, T, D)
+#define CCI_REGTILE_ROW(DT, TS, G, K, MG, T, D)                                                    \
+    {DT, G, K, MG, T, D, "regtile_" #TS "_G" #G "_K" #K "_MG" #MG "_T" #T "_D" #D,                  \
+     &cci::launch_regtile<TS, G, K, MG, T, D>},
