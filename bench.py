@@ -381,6 +381,18 @@ def run_ours(args, rank, world, local):
              "dense_tflops": case.dense_flops() / (dense_ms * 1e-3) / 1e12,
              "speedup_cci_over_dense": dense_ms / lin_avg}
 
+    # the CUDA-core kernel families on the same product (same inputs, same output)
+    families = {}
+    for name, algo in (("regtile_jump_dispatch", cci.ALGO_REGTILE), ("expand_branch_free", cci.ALGO_EXPAND)):
+        kn = cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, algo)
+        if not kn:
+            continue
+        fn = lambda a=algo: cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, algo=a)  # noqa: E731
+        fn()
+        ms = statistics.median(time_device(fn, 10, flush, stream))
+        families[name] = {"kernel": kn, "ms": ms, "nz_tflops": nzf / (ms * 1e-3) / 1e12,
+                          "roofline_frac": nzf / (ms * 1e-3) / 1e12 / ALU_PEAK_TFLOPS}
+
     extras = {}
     if args.extras and rank == 0:
         extras = run_extras(cci, dev, stream, flush)
@@ -401,7 +413,7 @@ def run_ours(args, rank, world, local):
             "gpu_launches": 2 * args.steps, "clocks": clk.summary(),
             "breakdown_ms": {"pack": statistics.mean(pack_ms), "linear": lin_avg,
                              "wall_per_step_incl_flush": t_wall * 1e3 / args.steps},
-            "dense_reference": dense, **extras,
+            "dense_reference": dense, "cuda_core_families": families, **extras,
         }
         print(json.dumps(line), flush=True)
     return 0
@@ -419,6 +431,9 @@ def run_extras(cci, dev, stream, flush):
         fn = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y)  # noqa: E731
         fn()
         ms = statistics.median(time_device(fn, 10, flush, stream))
+        fr = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_REGTILE)  # noqa: E731
+        fr()
+        ms_jump = statistics.median(time_device(fr, 5, flush, stream))
         Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
         Wm.view(case.Cout // G, G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
         dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), 10, flush, stream))
@@ -427,6 +442,7 @@ def run_extras(cci, dev, stream, flush):
                                   "dense_equiv_tflops": case.dense_flops() / (ms * 1e-3) / 1e12,
                                   "roofline_frac": tf / ALU_PEAK_TFLOPS,
                                   "dense_bf16_ms": dms, "speedup_over_dense": dms / ms,
+                                  "regtile_jump_dispatch_ms": ms_jump,
                                   "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R,
                                                             case.Cout, G, K)})
         del X, W, v, i, Y, Wm

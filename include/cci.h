@@ -75,14 +75,18 @@ typedef enum cci_dtype {
 
 /* Kernel family for cci_linear_ex / cci_conv2d_ex. */
 typedef enum cci_algo {
-    CCI_ALGO_AUTO = 0,      /* register-tiled scatter kernel when (G, K, dtype, shape)
-                               has one, else the generic kernel */
+    CCI_ALGO_AUTO = 0,      /* the fastest family this build has for (G, K, dtype, shape) */
     CCI_ALGO_GENERIC = 1,   /* generic kernel: any G <= 256, any K, any alignment */
-    CCI_ALGO_REGTILE = 2,   /* register-tiled scatter kernel only; CCI_ERR_UNSUPPORTED
-                               when (G, K, dtype, shape) has none */
-    CCI_ALGO_DENSE_TC = 3   /* comparison only: decompress to bf16 tiles in shared
+    CCI_ALGO_REGTILE = 2,   /* register-tiled scatter on CUDA cores: Alg. 2 with the output
+                               row chosen per (group, r) by a warp-uniform jump;
+                               CCI_ERR_UNSUPPORTED when (G, K, dtype, shape) has no tile */
+    CCI_ALGO_DENSE_TC = 3,  /* comparison only: decompress to bf16 tiles in shared
                                memory and multiply densely on the tensor cores
                                (tcgen05); bf16 only */
+    CCI_ALGO_EXPAND = 4     /* register-tiled on CUDA cores without jumps: each (group, r)
+                               is expanded to its G weights (pruned ones zero) in shared
+                               memory and all G rows are updated; same shape rules as
+                               CCI_ALGO_REGTILE */
 } cci_algo;
 
 /*

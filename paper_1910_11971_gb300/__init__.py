@@ -24,7 +24,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libcci.so")
 
 F32, BF16 = 0, 1
-ALGO_AUTO, ALGO_GENERIC, ALGO_REGTILE, ALGO_DENSE_TC = 0, 1, 2, 3
+ALGO_AUTO, ALGO_GENERIC, ALGO_REGTILE, ALGO_DENSE_TC, ALGO_EXPAND = 0, 1, 2, 3, 4
 
 STATUS_NAMES = {
     0: "CCI_OK", 1: "CCI_ERR_NULL", 2: "CCI_ERR_SHAPE", 3: "CCI_ERR_GROUP", 4: "CCI_ERR_DTYPE",

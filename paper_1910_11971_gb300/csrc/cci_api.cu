@@ -38,13 +38,24 @@ cci_status check_group(int64_t Cout, int G, int K)
     return CCI_OK;
 }
 
-const RegtileEntry *find_regtile(int dtype, int G, int K)
+// expand = true: the branch-free kernel (D == 0); false: the jump-dispatch kernel
+const RegtileEntry *find_regtile(int dtype, int G, int K, bool expand)
 {
     const RegtileEntry *tables[] = {kRegtile_f32_a, kRegtile_f32_b, kRegtile_bf16_a, kRegtile_bf16_b};
     for (const RegtileEntry *t : tables)
         for (; t->launch; ++t)
-            if (t->dtype == dtype && t->G == G && t->K == K) return t;
+            if (t->dtype == dtype && t->G == G && t->K == K && (t->D == 0) == expand) return t;
     return nullptr;
+}
+
+// the register-tiled family AUTO uses (measured on GB300: the branch-free kernel
+// is faster than the jump dispatch at every (G, K) of the workloads)
+bool auto_prefers_expand(int dtype, int G, int K)
+{
+    (void)dtype;
+    (void)G;
+    (void)K;
+    return true;
 }
 
 // shape conditions of the register-tiled kernel (16-byte vector copies)
@@ -65,10 +76,11 @@ cci_status forward(const FwdParams &p, int dtype, int G, int K, cci_algo algo, c
 {
     if (p.N == 0) return CCI_OK;
     if (algo == CCI_ALGO_DENSE_TC) return CCI_ERR_UNSUPPORTED;
-    if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE) {
-        const RegtileEntry *e = find_regtile(dtype, G, K);
+    if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
+        const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
+        const RegtileEntry *e = find_regtile(dtype, G, K, expand);
         if (e && regtile_shape_ok(dtype, p.Cin, p.R, K) && regtile_ptr_ok(p)) return to_status(e->launch(p, stream));
-        if (algo == CCI_ALGO_REGTILE) return CCI_ERR_UNSUPPORTED;
+        if (algo != CCI_ALGO_AUTO) return CCI_ERR_UNSUPPORTED;
     } else if (algo != CCI_ALGO_GENERIC) {
         return CCI_ERR_UNSUPPORTED;
     }
@@ -235,10 +247,13 @@ const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cou
 {
     if (!valid_dtype(dtype) || Cin < 1 || R < Cin || check_group(Cout, G, K) != CCI_OK) return "";
     if (algo == CCI_ALGO_DENSE_TC) return "";
-    if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE) {
-        const RegtileEntry *e = find_regtile(dtype, G, K);
+    if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
+        const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
+        const RegtileEntry *e = find_regtile(dtype, G, K, expand);
         if (e && regtile_shape_ok(dtype, Cin, R, K)) return e->name;
-        if (algo == CCI_ALGO_REGTILE) return "";
+        if (algo != CCI_ALGO_AUTO) return "";
+    } else if (algo != CCI_ALGO_GENERIC) {
+        return "";
     }
     return dtype == CCI_F32 ? "generic_f32" : "generic_bf16";
 }

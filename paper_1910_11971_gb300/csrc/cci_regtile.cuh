@@ -13,7 +13,11 @@
 //     cci_dispatch.cuh) into straight-line packed FMAs, and the MG*G x T block of
 //     outputs stays in registers ("load a whole group of elements of H onto
 //     on-chip registers", Sec. 3.2);
-//   * two columns share one packed FMA (fma.rn.f32x2).
+//   * two columns share one packed FMA (fma.rn.f32x2);
+//   * expand mode (D = 0) takes no jump: each record holds the G weights of the
+//     (group, r) with the pruned ones zero and the lane runs G straight-line
+//     packed FMAs per column pair -- G/K times the useful work, but no
+//     warp-uniform jumps, which cost far more than an FMA on this GPU.
 //
 // Pipeline per chunk of RC = 16 reduction indices:
 //   raw X tile [NTC][RC] and raw (value, index) runs are copied global->shared
@@ -71,12 +75,15 @@ struct RegTile {
     static constexpr int kNTC = kWN * 32 * T;             // columns per CTA
     static constexpr int kNGR = WC * MG;                  // groups per CTA
     static constexpr int kSlots = kRC * K;                // slots of one group in a chunk
-    static constexpr int kDisp = K / D;                   // jumps per (group, r)
-    static constexpr int kWords = D > 1 ? kDisp : (K + 3) / 4;
-    static constexpr int kRecVec = static_cast<int>(round16(4 * K + 4 * kWords) / 16);
+    static constexpr bool kExpand = D == 0;               // branch-free: G decompressed weights
+    static constexpr int kDisp = kExpand ? 0 : K / D;     // jumps per (group, r)
+    static constexpr int kWords = D > 1 ? K / D : (K + 3) / 4;
+    static constexpr int kRecVec =
+        kExpand ? G / 4 : static_cast<int>(round16(4 * K + 4 * kWords) / 16);
     static constexpr int kXPitch = kRC + 16 / static_cast<int>(sizeof(TS));
     static_assert(WC == 4 || WC == 8, "4 or 8 channel-warps");
-    static_assert(D == 1 || (D == 2 && K % 2 == 0), "one or two slots per jump");
+    static_assert(D == 0 || D == 1 || (D == 2 && K % 2 == 0), "expand, or one or two slots per jump");
+    static_assert(D != 0 || G % 4 == 0, "expanded records are whole 16-byte units");
     static_assert(T % 4 == 0, "T must be a multiple of 4");
     static_assert(kRC % kVec == 0, "a chunk must hold whole 16-byte vectors");
     static_assert((kSlots * static_cast<int>(sizeof(TS))) % 16 == 0, "value runs must be 16-byte multiples");
@@ -223,6 +230,31 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
             const TS *vr = vraw + buf * (NGR * SLOTS);
             const uint8_t *ir = iraw + buf * (NGR * SLOTS);
             uint4 *ro = rec + buf * (NGR * RC * RV);
+            if constexpr (RT::kExpand) {
+                // record = the G weights of (group, r) with the pruned ones zero;
+                // the thread owns the record, so the zero fill and the adds need no sync
+                for (int item = tid; item < NGR * RC; item += RT::kThreads) {
+                    const int gl = item / RC;
+                    const int r = item % RC;
+                    const bool live = (g0 + gl < total_groups) && (r0 + r < p.R);
+                    uint4 *dst = ro + (gl * RC + r) * RV;
+#pragma unroll
+                    for (int q = 0; q < RV; ++q) dst[q] = make_uint4(0, 0, 0, 0);
+                    if (!live) continue;
+                    float *w = reinterpret_cast<float *>(dst);
+#pragma unroll
+                    for (int s = 0; s < K; ++s) {
+                        const float v = Elem<TS>::to_f32(vr[gl * SLOTS + r * K + s]);
+                        const int i = ir[gl * SLOTS + r * K + s];
+                        if (i >= G) {
+                            report(p.status, CCI_ERR_INDEX);
+                            continue;
+                        }
+                        w[i] += v;  // a repeated index adds both values
+                    }
+                }
+                return;
+            }
             for (int item = tid; item < NGR * RC; item += RT::kThreads) {
                 const int gl = item / RC;
                 const int r = item % RC;
@@ -311,23 +343,35 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
                 unsigned long long xn[H];
                 uint4 rn[MG][RV];
                 load_r(r + 1 < RC ? r + 1 : r, xn, rn);  // prefetch the next reduction index
+                if constexpr (RT::kExpand) {
+#pragma unroll
+                    for (int g = 0; g < MG; ++g)
+#pragma unroll
+                        for (int j = 0; j < G; ++j) {
+                            const float w = __uint_as_float(word_of(rc[g][j / 4], j % 4));
+                            const unsigned long long ww = pack2(w, w);
+#pragma unroll
+                            for (int t = 0; t < H; ++t) ffma2(acc[g][j][t], xx[t], ww);
+                        }
+                } else
 #pragma unroll
                 for (int g = 0; g < MG; ++g) {
 #pragma unroll
-                    for (int d = 0; d < K / D; ++d) {
-                        unsigned long long vv[D];
+                    for (int d = 0; d < RT::kDisp; ++d) {
+                        constexpr int DD = D > 0 ? D : 1;
+                        unsigned long long vv[DD];
 #pragma unroll
-                        for (int s = 0; s < D; ++s) {
-                            const float v = __uint_as_float(word_of(rc[g][(d * D + s) / 4], (d * D + s) % 4));
+                        for (int s = 0; s < DD; ++s) {
+                            const float v = __uint_as_float(word_of(rc[g][(d * DD + s) / 4], (d * DD + s) % 4));
                             vv[s] = pack2(v, v);
                         }
                         uint32_t word;
-                        if constexpr (D == 1) {
+                        if constexpr (DD == 1) {
                             word = (word_of(rc[g][(K + d / 4) / 4], (K + d / 4) % 4) >> (8 * (d % 4))) & 0xffu;
                         } else {
                             word = word_of(rc[g][(K + d) / 4], (K + d) % 4);
                         }
-                        Dispatch<G, D, T>::run(acc[g], xx, vv, word);
+                        Dispatch<G, (D > 0 ? D : 1), T>::run(acc[g], xx, vv, word);
                     }
                 }
 #pragma unroll

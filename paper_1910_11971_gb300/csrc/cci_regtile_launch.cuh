@@ -48,5 +48,6 @@ cudaError_t launch_regtile(const FwdParams &p, cudaStream_t stream)
 
 // table row for one instantiation (dtype tag, storage type, G, K, MG, T, D)
 #define CCI_REGTILE_ROW(DT, TS, G, K, MG, T, D)                                                    \
-    {DT, G, K, MG, T, D, "regtile_" #TS "_G" #G "_K" #K "_MG" #MG "_T" #T "_D" #D,                  \
+    {DT, G, K, MG, T, D, (D == 0 ? "expand_" #TS "_G" #G "_K" #K "_MG" #MG "_T" #T                  \
+                                 : "regtile_" #TS "_G" #G "_K" #K "_MG" #MG "_T" #T "_D" #D),       \
      &cci::launch_regtile<TS, G, K, MG, T, D>},

@@ -120,8 +120,10 @@ def test_algo_dense_tc_without_bf16_is_unsupported_name(lib):
 
 def test_kernel_names(lib):
     import torch
-    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2).startswith("regtile_float_G8_K2_")
-    assert cci.kernel_name(torch.bfloat16, 128, 1152, 128, 16, 4).startswith("regtile_uint16_t_G16_K4")
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2, cci.ALGO_REGTILE).startswith("regtile_float_G8_K2_")
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2, cci.ALGO_EXPAND).startswith("expand_float_G8_K2_")
+    assert cci.kernel_name(torch.bfloat16, 128, 1152, 128, 16, 4, cci.ALGO_REGTILE).startswith("regtile_uint16_t_G16_K4")
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2) != ""
     assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 3) == "generic_f32"  # no tile for K=3
     assert cci.kernel_name(torch.bfloat16, 12, 12, 16, 8, 2) == "generic_bf16"  # Cin % 8 != 0
     assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 3, cci.ALGO_REGTILE) == ""

@@ -131,13 +131,21 @@ def test_linear_small(dev, case):
     assert_within_tol(f64(Y), Yo, S, str(case))
 
 
+REGTILE_ALGOS = [cci.ALGO_REGTILE, cci.ALGO_EXPAND]
+
+
+@pytest.mark.parametrize("algo", REGTILE_ALGOS, ids=["regtile", "expand"])
 @pytest.mark.parametrize("case", [c for c in SMALL if c[0] > 1], ids=lambda c: "N{}_C{}x{}_G{}K{}_{}".format(*c))
-def test_regtile_matches_generic_bitwise(dev, case):
-    """Both kernels add the contributions of an output in the same order (ascending
-    r, then slot, one FMA each, from +0), so they agree bit for bit."""
+def test_regtile_matches_generic_bitwise(dev, case, algo):
+    """The kernels add the contributions of an output in the same order (ascending
+    r, then slot, one FMA each, from +0); the expand kernel's extra terms are
+    fma(0, x, acc) = acc exactly (acc is never -0), so all agree bit for bit."""
     N, Cin, Cout, G, K, dtype = case
     X, W = wl.random_small(N + 7 * Cin, dtype, N, Cin, Cout)
-    Ya = run_linear(dev, X, W, G, K, cci.ALGO_AUTO)
+    name = cci.kernel_name(_dt(dtype), Cin, Cin, Cout, G, K, algo)
+    if not name:
+        pytest.skip("no register tile for this (G, K, dtype, shape)")
+    Ya = run_linear(dev, X, W, G, K, algo)
     Yg = run_linear(dev, X, W, G, K, cci.ALGO_GENERIC)
     assert torch.equal(Ya.view(torch.int32), Yg.view(torch.int32))
 
@@ -178,7 +186,7 @@ def test_linear_sweep_full(dev, G, K):
     assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name)
 
 
-@pytest.mark.parametrize("algo", [cci.ALGO_AUTO, cci.ALGO_GENERIC])
+@pytest.mark.parametrize("algo", [cci.ALGO_GENERIC] + REGTILE_ALGOS)
 def test_linear_bad_index_reported(dev, algo):
     G, K, Cout, Cin, N = 8, 2, 16, 32, 40
     v = torch.ones((Cout // G, Cin, K), device=dev)
@@ -192,7 +200,7 @@ def test_linear_bad_index_reported(dev, algo):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("algo", [cci.ALGO_AUTO, cci.ALGO_GENERIC])
+@pytest.mark.parametrize("algo", [cci.ALGO_GENERIC] + REGTILE_ALGOS)
 def test_linear_repeated_and_unordered_indices(dev, dtype, algo):
     """Packed input not produced by cci_pack: repeated and descending indices are
     summed as Alg. 2 does (the oracle's decompression sums them too)."""
@@ -259,13 +267,16 @@ CONV_SMALL = [
 ]
 
 
+@pytest.mark.parametrize("algo", [cci.ALGO_AUTO] + REGTILE_ALGOS, ids=["auto", "regtile", "expand"])
 @pytest.mark.parametrize("case", CONV_SMALL, ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
-def test_conv_small(dev, case):
+def test_conv_small(dev, case, algo):
     B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
+    if not cci.kernel_name(_dt(dtype), Cin, KH * KW * Cin, Cout, G, K, algo):
+        pytest.skip("no register tile for this (G, K, dtype, shape)")
     g = torch.Generator().manual_seed(B * 7 + Cin)
     X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(_dt(dtype))
     W = torch.randn((Cout, KH * KW * Cin), generator=g).to(_dt(dtype))
-    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K)
+    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K, algo)
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
     assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
