@@ -237,11 +237,13 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
                     const int gl = item / RC;
                     const int r = item % RC;
                     const bool live = (g0 + gl < total_groups) && (r0 + r < p.R);
-                    uint4 *dst = ro + (gl * RC + r) * RV;
+                    // every write of the record goes through float (one type for the
+                    // zero fill and the adds, so no aliasing reordering between them)
+                    float *w = reinterpret_cast<float *>(ro + (gl * RC + r) * RV);
 #pragma unroll
-                    for (int q = 0; q < RV; ++q) dst[q] = make_uint4(0, 0, 0, 0);
+                    for (int q = 0; q < RV; ++q)
+                        reinterpret_cast<float4 *>(w)[q] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
                     if (!live) continue;
-                    float *w = reinterpret_cast<float *>(dst);
 #pragma unroll
                     for (int s = 0; s < K; ++s) {
                         const float v = Elem<TS>::to_f32(vr[gl * SLOTS + r * K + s]);
@@ -353,7 +355,7 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
 #pragma unroll
                             for (int t = 0; t < H; ++t) ffma2(acc[g][j][t], xx[t], ww);
                         }
-                } else
+                } else {
 #pragma unroll
                 for (int g = 0; g < MG; ++g) {
 #pragma unroll
@@ -373,6 +375,7 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
                         }
                         Dispatch<G, (D > 0 ? D : 1), T>::run(acc[g], xx, vv, word);
                     }
+                }
                 }
 #pragma unroll
                 for (int t = 0; t < H; ++t) xx[t] = xn[t];
