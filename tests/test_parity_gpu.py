@@ -164,7 +164,7 @@ def test_linear_bottleneck_full(dev):
     2048 sampled rows against the oracle."""
     case = wl.BOTTLENECK_1X1
     X, W = wl.linear_inputs(case)
-    assert cci.kernel_name(F32, case.Cin, case.R, case.Cout, case.G, case.K).startswith("regtile")
+    assert cci.kernel_name(F32, case.Cin, case.R, case.Cout, case.G, case.K).startswith(("regtile", "expand"))
     Y = run_linear(dev, X, W, case.G, case.K)
     assert torch.isfinite(Y).all()
     rows = sample_rows(case.N, 2048)
@@ -322,7 +322,7 @@ def check_conv_case(dev, case, npts=1024, seed=0):
 def test_conv3x3_full(dev):
     """Batch 64, 28x28, 128 -> 128, 3x3 s1 p1, G=16, K=4, bf16."""
     case = wl.CONV3X3_28
-    assert cci.kernel_name(BF16, case.Cin, case.R, case.Cout, case.G, case.K).startswith("regtile")
+    assert cci.kernel_name(BF16, case.Cin, case.R, case.Cout, case.G, case.K).startswith(("regtile", "expand"))
     check_conv_case(dev, case, npts=2048)
 
 
