@@ -325,6 +325,34 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
             const float *xw = xs + buf * (RC * NTC) + wnw * (32 * T) + lane * 4;
             const uint4 *rw = rec + buf * (NGR * RC * RV) + wcw * MG * RC * RV;
 
+            if constexpr (RT::kExpand) {
+                // straight-line code: unrolled so the compiler schedules the shared
+                // loads of later reduction indices under the FMAs of earlier ones
+#pragma unroll 4
+                for (int r = 0; r < RC; ++r) {
+                    unsigned long long xx[H];
+#pragma unroll
+                    for (int q = 0; q < T / 4; ++q) {
+                        const ulonglong2 u = *reinterpret_cast<const ulonglong2 *>(xw + r * NTC + q * 128);
+                        xx[2 * q] = u.x;
+                        xx[2 * q + 1] = u.y;
+                    }
+#pragma unroll
+                    for (int g = 0; g < MG; ++g) {
+#pragma unroll
+                        for (int q = 0; q < RV; ++q) {
+                            const float4 w4 = reinterpret_cast<const float4 *>(rw)[(g * RC + r) * RV + q];
+                            const float w[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                const unsigned long long ww = pack2(w[e], w[e]);
+#pragma unroll
+                                for (int t = 0; t < H; ++t) ffma2(acc[g][4 * q + e][t], xx[t], ww);
+                            }
+                        }
+                    }
+                }
+            } else {
             unsigned long long xx[H];
             uint4 rc[MG][RV];
             auto load_r = [&](int r, unsigned long long (&xo)[H], uint4 (&ro)[MG][RV]) {
@@ -345,17 +373,7 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
                 unsigned long long xn[H];
                 uint4 rn[MG][RV];
                 load_r(r + 1 < RC ? r + 1 : r, xn, rn);  // prefetch the next reduction index
-                if constexpr (RT::kExpand) {
-#pragma unroll
-                    for (int g = 0; g < MG; ++g)
-#pragma unroll
-                        for (int j = 0; j < G; ++j) {
-                            const float w = __uint_as_float(word_of(rc[g][j / 4], j % 4));
-                            const unsigned long long ww = pack2(w, w);
-#pragma unroll
-                            for (int t = 0; t < H; ++t) ffma2(acc[g][j][t], xx[t], ww);
-                        }
-                } else {
+                {
 #pragma unroll
                 for (int g = 0; g < MG; ++g) {
 #pragma unroll
@@ -384,6 +402,7 @@ __global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_
 #pragma unroll
                     for (int q = 0; q < RV; ++q) rc[g][q] = rn[g][q];
             }
+            }  // jump-dispatch path
             if (c + 1 < nchunks) {
                 cp_async_wait_all();
                 __syncthreads();
