@@ -109,8 +109,15 @@ __device__ __forceinline__ uint32_t word_of(const uint4 &u, int k)
 // the kernel: persistent over tiles (tile = channel tile fastest, so the CTAs
 // running at the same time share column tiles and X is reused through L2)
 // ---------------------------------------------------------------------------
+// CTAs per SM the kernel is compiled for: two when the accumulator tile is at
+// most 64 fp32 registers per lane (16 resident warps hide the shared-load and
+// barrier latencies), else one
+template <int MG, int G, int T>
+constexpr int regtile_min_blocks() { return MG * G * T <= 64 ? 2 : 1; }
+
 template <typename TS, int G, int K, int MG, int T, int D, int WC>
-__global__ void __launch_bounds__(256, 1) regtile_kernel(FwdParams p, int64_t n_ct, int64_t n_tiles)
+__global__ void __launch_bounds__(256, regtile_min_blocks<MG, G, T>())
+    regtile_kernel(FwdParams p, int64_t n_ct, int64_t n_tiles)
 {
     using RT = RegTile<TS, G, K, MG, T, D, WC>;
     constexpr int RC = RT::kRC;
