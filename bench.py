@@ -192,7 +192,7 @@ def run_reference(args, rank, world):
     t0 = time.perf_counter()
     oracle.linear(Xf[:rows], Wd, mask)
     dt = time.perf_counter() - t0
-    budget = 120.0 / max(1, args.steps + args.warmup)
+    budget = 90.0 / max(1, args.steps + args.warmup)
     rows = max(16, min(Xf.shape[0], int(rows * budget / max(dt, 1e-4))))
     for _ in range(args.warmup):
         oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
