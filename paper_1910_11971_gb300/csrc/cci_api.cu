@@ -75,7 +75,11 @@ cci_status to_status(cudaError_t e) { return e == cudaSuccess ? CCI_OK : CCI_ERR
 cci_status forward(const FwdParams &p, int dtype, int G, int K, cci_algo algo, cudaStream_t stream)
 {
     if (p.N == 0) return CCI_OK;
-    if (algo == CCI_ALGO_DENSE_TC) return CCI_ERR_UNSUPPORTED;
+    if (algo == CCI_ALGO_DENSE_TC) {
+        if (!dense_tc_supported(dtype, G, K) || p.Cin % 8 != 0 || !aligned(p.X, 16) || !aligned(p.Y, 16))
+            return CCI_ERR_UNSUPPORTED;
+        return to_status(launch_dense_tc(p, G, K, stream));
+    }
     if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
         const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
         const RegtileEntry *e = find_regtile(dtype, G, K, expand);
@@ -246,7 +250,19 @@ cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int6
 const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K, cci_algo algo)
 {
     if (!valid_dtype(dtype) || Cin < 1 || R < Cin || check_group(Cout, G, K) != CCI_OK) return "";
-    if (algo == CCI_ALGO_DENSE_TC) return "";
+    if (algo == CCI_ALGO_DENSE_TC) {
+        static const char *names[] = {"dense_tc_bf16_G4_K1", "dense_tc_bf16_G4_K2", "dense_tc_bf16_G8_K1",
+                                      "dense_tc_bf16_G8_K2", "dense_tc_bf16_G8_K4", "dense_tc_bf16_G16_K1",
+                                      "dense_tc_bf16_G16_K2", "dense_tc_bf16_G16_K4", "dense_tc_bf16_G16_K8",
+                                      "dense_tc_bf16_G32_K1", "dense_tc_bf16_G32_K2", "dense_tc_bf16_G32_K4",
+                                      "dense_tc_bf16_G32_K8", "dense_tc_bf16_G32_K16"};
+        if (!dense_tc_supported(dtype, G, K) || Cin % 8 != 0) return "";
+        int i = 0;
+        for (int g = 4; g <= 32; g *= 2)
+            for (int k = 1; k <= g / 2; k *= 2, ++i)
+                if (g == G && k == K) return names[i];
+        return "";
+    }
     if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
         const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
         const RegtileEntry *e = find_regtile(dtype, G, K, expand);

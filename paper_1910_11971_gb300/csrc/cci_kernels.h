@@ -10,6 +10,10 @@ cudaError_t launch_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G
 cudaError_t launch_generic(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);
 cudaError_t launch_fma_probe(float *out, int blocks, int threads, int iters, cudaStream_t stream);
 
+// dense tensor-core comparison kernel (tcgen05, bf16 only)
+bool dense_tc_supported(int dtype, int G, int K);
+cudaError_t launch_dense_tc(const FwdParams &p, int G, int K, cudaStream_t stream);
+
 // One register-tiled instantiation: (dtype, G, K) -> tile shape and launcher.
 struct RegtileEntry {
     int dtype, G, K, MG, T, D;

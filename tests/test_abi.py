@@ -114,8 +114,13 @@ def test_pack_rejects(lib):
     assert p(FAKE + 2, 0, 8, 4, 4, 2, FAKE, FAKE, None, None) == ALIGN
 
 
-def test_algo_dense_tc_without_bf16_is_unsupported_name(lib):
-    assert cci.kernel_name(__import__("torch").float32, 16, 16, 16, 8, 2, cci.ALGO_DENSE_TC) == ""
+def test_algo_dense_tc_names(lib):
+    import torch
+    assert cci.kernel_name(torch.float32, 16, 16, 16, 8, 2, cci.ALGO_DENSE_TC) == ""  # bf16 only
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 16, 8, 2, cci.ALGO_DENSE_TC) == "dense_tc_bf16_G8_K2"
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 64, 32, 16, cci.ALGO_DENSE_TC) == "dense_tc_bf16_G32_K16"
+    assert cci.kernel_name(torch.bfloat16, 12, 12, 16, 8, 2, cci.ALGO_DENSE_TC) == ""  # Cin % 8
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 24, 8, 3, cci.ALGO_DENSE_TC) == ""  # K not a power of 2
 
 
 def test_kernel_names(lib):

@@ -336,3 +336,66 @@ def test_resnet50_layer(dev, li, K):
     s2, strided downsample 1x1, 14x14 and 7x7 stages."""
     case = wl.resnet50_layers(K=K)[li]
     check_conv_case(dev, case, npts=512, seed=li)
+
+
+# ---------------------------------------------------------------------------
+# dense tensor-core comparison kernel (tcgen05, bf16)
+# ---------------------------------------------------------------------------
+# (N, Cin, Cout, G, K): one tile, ragged N and Cout, several tiles per CTA, every (G, K) family
+DENSE_SMALL = [
+    (128, 64, 256, 8, 2), (1, 64, 256, 8, 2), (200, 64, 256, 8, 2), (300, 128, 512, 8, 2),
+    (130, 72, 40, 4, 1), (257, 136, 96, 4, 2), (64, 64, 64, 16, 4), (515, 192, 384, 16, 8),
+    (129, 80, 64, 32, 16), (100, 256, 320, 32, 4), (1000, 64, 256, 8, 4), (77, 8, 32, 16, 1),
+]
+
+
+@pytest.mark.parametrize("case", DENSE_SMALL, ids=lambda c: "N{}_C{}x{}_G{}K{}".format(*c))
+def test_dense_tc_small(dev, case):
+    N, Cin, Cout, G, K = case
+    X, W = wl.random_small(N * 3 + Cin, "bf16", N, Cin, Cout)
+    assert cci.kernel_name(BF16, Cin, Cin, Cout, G, K, cci.ALGO_DENSE_TC).startswith("dense_tc")
+    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, str(case))
+
+
+@pytest.mark.parametrize("G,K", wl.SWEEP_POINTS)
+def test_dense_tc_sweep_full(dev, G, K):
+    case = wl.sweep_case(G, K)
+    X, W = wl.linear_inputs(case, device="cpu")
+    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC)
+    assert torch.isfinite(Y).all()
+    rows = sample_rows(case.N, 192, seed=G * 37 + K)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name + " dense_tc")
+
+
+@pytest.mark.parametrize("case", [c for c in CONV_SMALL if c[-1] == "bf16" and c[3] % 8 == 0 and c[9] in (4, 8, 16, 32)
+                                  and (c[10] & (c[10] - 1)) == 0 and c[10] <= c[9] // 2],
+                         ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
+def test_dense_tc_conv_small(dev, case):
+    B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
+    g = torch.Generator().manual_seed(B * 11 + Cin)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, KH * KW * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K, cci.ALGO_DENSE_TC)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
+
+
+def test_dense_tc_conv3x3_full(dev):
+    case = wl.CONV3X3_28
+    X, W = wl.conv_inputs(case, device="cpu")
+    Y = run_conv(dev, X, W, (case.KH, case.KW, (case.stride,) * 2, (case.pad,) * 2, case.Cout),
+                 case.G, case.K, cci.ALGO_DENSE_TC)
+    assert torch.isfinite(Y).all()
+    pts = conv_points(case, 1024, 5)
+    Xs = f64(X[[0, case.B - 1]])
+    per = case.P * case.Q
+    local = np.where(pts < per, pts, pts - (case.B - 1) * per + per)
+    _, _, Wd, mask = oracle_reference(W, case.G, case.K)
+    Yo, S = oracle.conv2d(Xs, Wd, mask, 3, 3, (1, 1), (1, 1), pts=local)
+    assert_within_tol(f64(Y.reshape(-1, case.Cout)[torch.from_numpy(pts).to(dev)]), Yo, S, "conv3x3 dense_tc")
