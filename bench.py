@@ -434,6 +434,9 @@ def run_extras(cci, dev, stream, flush):
         fr = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_REGTILE)  # noqa: E731
         fr()
         ms_jump = statistics.median(time_device(fr, 5, flush, stream))
+        ft = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_DENSE_TC)  # noqa: E731
+        ft()
+        ms_tc = statistics.median(time_device(ft, 10, flush, stream))
         Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
         Wm.view(case.Cout // G, G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
         dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), 10, flush, stream))
@@ -443,6 +446,9 @@ def run_extras(cci, dev, stream, flush):
                                   "roofline_frac": tf / ALU_PEAK_TFLOPS,
                                   "dense_bf16_ms": dms, "speedup_over_dense": dms / ms,
                                   "regtile_jump_dispatch_ms": ms_jump,
+                                  "dense_tc_ms": ms_tc,
+                                  "dense_tc_nz_tflops": case.nz_flops() / (ms_tc * 1e-3) / 1e12,
+                                  "dense_tc_dense_equiv_tflops": case.dense_flops() / (ms_tc * 1e-3) / 1e12,
                                   "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R,
                                                             case.Cout, G, K)})
         del X, W, v, i, Y, Wm
@@ -458,8 +464,14 @@ def run_extras(cci, dev, stream, flush):
     x4 = X.permute(0, 3, 1, 2)  # NHWC memory, NCHW view = channels_last
     dms = statistics.median(time_device(
         lambda: torch.nn.functional.conv2d(x4, w4, padding=1), 10, flush, stream))
+    ft = lambda: cci.conv2d(X, v, i, case.Cout, case.G, case.K, 3, 3, (1, 1), (1, 1),  # noqa: E731
+                            algo=cci.ALGO_DENSE_TC)
+    ft()
+    ms_tc = statistics.median(time_device(ft, 10, flush, stream))
     tf = case.nz_flops() / (ms * 1e-3) / 1e12
     out["conv3x3_28"] = {"ms": ms, "nz_tflops": tf, "roofline_frac": tf / ALU_PEAK_TFLOPS,
+                         "dense_tc_ms": ms_tc, "dense_tc_nz_tflops": case.nz_flops() / (ms_tc * 1e-3) / 1e12,
+                         "dense_tc_dense_equiv_tflops": case.dense_flops() / (ms_tc * 1e-3) / 1e12,
                          "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
                          "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R, case.Cout,
                                                    case.G, case.K)}
