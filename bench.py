@@ -437,6 +437,11 @@ def run_extras(cci, dev, stream, flush):
         ft = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_DENSE_TC)  # noqa: E731
         ft()
         ms_tc = statistics.median(time_device(ft, 10, flush, stream))
+        ws = cci.new_workspace(cci.ALGO_DENSE_TC_WS, X.dtype, case.Cout, case.R, dev)
+        fw = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_DENSE_TC_WS,  # noqa: E731
+                                workspace=ws)
+        fw()
+        ms_ws = statistics.median(time_device(fw, 10, flush, stream))
         Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
         Wm.view(case.Cout // G, G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
         dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), 10, flush, stream))
@@ -449,9 +454,14 @@ def run_extras(cci, dev, stream, flush):
                                   "dense_tc_ms": ms_tc,
                                   "dense_tc_nz_tflops": case.nz_flops() / (ms_tc * 1e-3) / 1e12,
                                   "dense_tc_dense_equiv_tflops": case.dense_flops() / (ms_tc * 1e-3) / 1e12,
+                         "dense_tc_ws_ms": ms_ws, "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
+                         "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
+                                  "dense_tc_ws_ms": ms_ws,
+                                  "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
+                                  "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
                                   "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R,
                                                             case.Cout, G, K)})
-        del X, W, v, i, Y, Wm
+        del X, W, v, i, Y, Wm, ws
     case = wl.CONV3X3_28
     X, W = wl.conv_inputs(case, device=str(dev))
     v, i = cci.pack(W, case.G, case.K)
@@ -468,10 +478,17 @@ def run_extras(cci, dev, stream, flush):
                             algo=cci.ALGO_DENSE_TC)
     ft()
     ms_tc = statistics.median(time_device(ft, 10, flush, stream))
+    ws = cci.new_workspace(cci.ALGO_DENSE_TC_WS, X.dtype, case.Cout, case.R, dev)
+    fw = lambda: cci.conv2d(X, v, i, case.Cout, case.G, case.K, 3, 3, (1, 1), (1, 1),  # noqa: E731
+                            algo=cci.ALGO_DENSE_TC_WS, workspace=ws)
+    fw()
+    ms_ws = statistics.median(time_device(fw, 10, flush, stream))
     tf = case.nz_flops() / (ms * 1e-3) / 1e12
     out["conv3x3_28"] = {"ms": ms, "nz_tflops": tf, "roofline_frac": tf / ALU_PEAK_TFLOPS,
                          "dense_tc_ms": ms_tc, "dense_tc_nz_tflops": case.nz_flops() / (ms_tc * 1e-3) / 1e12,
                          "dense_tc_dense_equiv_tflops": case.dense_flops() / (ms_tc * 1e-3) / 1e12,
+                         "dense_tc_ws_ms": ms_ws, "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
+                         "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
                          "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
                          "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R, case.Cout,
                                                    case.G, case.K)}

@@ -44,6 +44,7 @@
 #ifndef CCI_H_
 #define CCI_H_
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -65,7 +66,10 @@ typedef enum cci_status {
     CCI_ERR_CUDA = 7,         /* a CUDA launch or runtime call failed */
     CCI_ERR_TIMEOUT = 8,      /* device: a bounded wait inside a kernel expired */
     CCI_ERR_UNSUPPORTED = 9,  /* valid request this build does not implement */
-    CCI_ERR_INDEX = 10        /* device: a packed index >= G given to a product */
+    CCI_ERR_INDEX = 10,       /* device: a packed index >= G given to a product (dense
+                                 kernels: also an index set not strictly increasing) */
+    CCI_ERR_WORKSPACE = 11    /* the kernel family needs a workspace: missing, too small
+                                 or not 16-byte aligned (see cci_workspace_size) */
 } cci_status;
 
 typedef enum cci_dtype {
@@ -83,10 +87,15 @@ typedef enum cci_algo {
     CCI_ALGO_DENSE_TC = 3,  /* comparison only: decompress to bf16 tiles in shared
                                memory and multiply densely on the tensor cores
                                (tcgen05); bf16 only */
-    CCI_ALGO_EXPAND = 4     /* register-tiled on CUDA cores without jumps: each (group, r)
+    CCI_ALGO_EXPAND = 4,    /* register-tiled on CUDA cores without jumps: each (group, r)
                                is expanded to its G weights (pruned ones zero) in shared
                                memory and all G rows are updated; same shape rules as
                                CCI_ALGO_REGTILE */
+    CCI_ALGO_DENSE_TC_WS = 5  /* decompress the packed weights once per call into a caller
+                               workspace (dense bf16 [Cout][R]) and multiply densely on the
+                               tensor cores (tcgen05), operands streamed by cp.async;
+                               bf16 only, Cin % 8 == 0, R % 8 == 0; needs
+                               cci_workspace_size() bytes */
 } cci_algo;
 
 /*
@@ -149,7 +158,8 @@ cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int6
                       int KH, int KW, int stride_h, int stride_w, int pad_h, int pad_w, int G,
                       int K, float *Y, uint32_t *dev_status, cci_stream_t stream);
 
-/* As cci_linear / cci_conv2d, with the kernel family chosen by `algo`. */
+/* As cci_linear / cci_conv2d, with the kernel family chosen by `algo` and no
+ * workspace (CCI_ALGO_DENSE_TC_WS returns CCI_ERR_WORKSPACE; AUTO does not pick it). */
 cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
                          const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
                          float *Y, uint32_t *dev_status, cci_algo algo, cci_stream_t stream);
@@ -158,6 +168,32 @@ cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
                          int KH, int KW, int stride_h, int stride_w, int pad_h, int pad_w,
                          int G, int K, float *Y, uint32_t *dev_status, cci_algo algo,
                          cci_stream_t stream);
+
+/*
+ * cci_workspace_size -- bytes of device workspace that cci_linear_ws /
+ * cci_conv2d_ws need for this kernel family and layer (R = Cin for a product,
+ * Cin*KH*KW for a convolution): Cout*R*2 for CCI_ALGO_DENSE_TC_WS, 0 for the
+ * families that need none.  For CCI_ALGO_AUTO: the bytes that let AUTO pick its
+ * fastest family for a bf16 layer (0 for fp32).
+ */
+size_t cci_workspace_size(cci_algo algo, cci_dtype dtype, int64_t Cout, int64_t R);
+
+/*
+ * As cci_linear_ex / cci_conv2d_ex with a caller workspace (device, 16-byte
+ * aligned, `workspace_bytes` long; NULL / 0 allowed for families that need
+ * none).  The call overwrites the workspace; calls that overlap on the GPU must
+ * use different workspaces.  CCI_ALGO_AUTO uses the dense tensor-core family
+ * for bf16 layers when the workspace is large enough, else the CUDA-core family.
+ */
+cci_status cci_linear_ws(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
+                         const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
+                         float *Y, uint32_t *dev_status, cci_algo algo, void *workspace,
+                         size_t workspace_bytes, cci_stream_t stream);
+cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W,
+                         int64_t Cin, const void *values, const uint8_t *idx, int64_t Cout,
+                         int KH, int KW, int stride_h, int stride_w, int pad_h, int pad_w,
+                         int G, int K, float *Y, uint32_t *dev_status, cci_algo algo,
+                         void *workspace, size_t workspace_bytes, cci_stream_t stream);
 
 /*
  * cci_kernel_name -- the name of the kernel that cci_linear_ex / cci_conv2d_ex

@@ -24,12 +24,12 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "libcci.so")
 
 F32, BF16 = 0, 1
-ALGO_AUTO, ALGO_GENERIC, ALGO_REGTILE, ALGO_DENSE_TC, ALGO_EXPAND = 0, 1, 2, 3, 4
+ALGO_AUTO, ALGO_GENERIC, ALGO_REGTILE, ALGO_DENSE_TC, ALGO_EXPAND, ALGO_DENSE_TC_WS = 0, 1, 2, 3, 4, 5
 
 STATUS_NAMES = {
     0: "CCI_OK", 1: "CCI_ERR_NULL", 2: "CCI_ERR_SHAPE", 3: "CCI_ERR_GROUP", 4: "CCI_ERR_DTYPE",
     5: "CCI_ERR_ALIGN", 6: "CCI_ERR_VALUE", 7: "CCI_ERR_CUDA", 8: "CCI_ERR_TIMEOUT",
-    9: "CCI_ERR_UNSUPPORTED", 10: "CCI_ERR_INDEX",
+    9: "CCI_ERR_UNSUPPORTED", 10: "CCI_ERR_INDEX", 11: "CCI_ERR_WORKSPACE",
 }
 
 # exported symbols with their ctypes signatures (the declarations of cci.h)
@@ -42,6 +42,11 @@ SIGNATURES = {
                           _I32, _I32, _I32, _I32, _P, _U32P, _P]),
     "cci_conv2d_ex": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32, _I32,
                              _I32, _I32, _I32, _I32, _P, _U32P, _I32, _P]),
+    "cci_linear_ws": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P, _I32, _P,
+                             ctypes.c_size_t, _P]),
+    "cci_conv2d_ws": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32, _I32,
+                             _I32, _I32, _I32, _I32, _P, _U32P, _I32, _P, ctypes.c_size_t, _P]),
+    "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
     "cci_kernel_name": (ctypes.c_char_p, [_I32, _I64, _I64, _I64, _I32, _I32, _I32]),
     "cci_status_string": (ctypes.c_char_p, [_I32]),
     "cci_decode_device_status": (_I32, [ctypes.c_uint32]),
@@ -147,16 +152,39 @@ def pack(W: torch.Tensor, G: int, K: int, *, status: Optional[torch.Tensor] = No
     return values, idx
 
 
+def workspace_size(algo: int, dtype: torch.dtype, Cout: int, R: int) -> int:
+    """Bytes of workspace the kernel family needs for a layer (0: none)."""
+    return int(lib().cci_workspace_size(algo, F32 if dtype == torch.float32 else BF16, Cout, R))
+
+
+def new_workspace(algo: int, dtype: torch.dtype, Cout: int, R: int, device) -> Optional[torch.Tensor]:
+    n = workspace_size(algo, dtype, Cout, R)
+    return torch.empty(n, dtype=torch.uint8, device=device) if n else None
+
+
+def _ws(workspace: Optional[torch.Tensor]):
+    if workspace is None:
+        return None, 0
+    return workspace.data_ptr(), workspace.numel() * workspace.element_size()
+
+
 def linear(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int, *,
            out: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
-           algo: int = ALGO_AUTO) -> torch.Tensor:
-    """Y[N][Cout] (fp32) = the CCI-sparse product of X[N][Cin] (Alg. 2)."""
+           algo: int = ALGO_AUTO, workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Y[N][Cout] (fp32) = the CCI-sparse product of X[N][Cin] (Alg. 2).
+
+    ``workspace``: device buffer for the families that need one (see
+    ``workspace_size``); with ``algo=ALGO_DENSE_TC_WS`` and none given, one is
+    allocated here (PyTorch memory, not by the library)."""
     _cuda_contig(X, "X")
     N, Cin = X.shape
+    if workspace is None and algo == ALGO_DENSE_TC_WS:
+        workspace = new_workspace(algo, X.dtype, Cout, Cin, X.device)
     Y = out if out is not None else torch.empty((N, Cout), dtype=torch.float32, device=X.device)
-    code = lib().cci_linear_ex(X.data_ptr(), _dtype_code(X), N, Cin, values.data_ptr(),
+    wp, wb = _ws(workspace)
+    code = lib().cci_linear_ws(X.data_ptr(), _dtype_code(X), N, Cin, values.data_ptr(),
                                idx.data_ptr(), Cout, G, K, Y.data_ptr(),
-                               status.data_ptr() if status is not None else None, algo,
+                               status.data_ptr() if status is not None else None, algo, wp, wb,
                                _stream(X.device))
     _check(code, "cci_linear")
     return Y
@@ -168,17 +196,21 @@ def conv_out_hw(H: int, W: int, KH: int, KW: int, stride: Sequence[int], pad: Se
 
 def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int,
            KH: int, KW: int, stride=(1, 1), pad=(0, 0), *, out: Optional[torch.Tensor] = None,
-           status: Optional[torch.Tensor] = None, algo: int = ALGO_AUTO) -> torch.Tensor:
+           status: Optional[torch.Tensor] = None, algo: int = ALGO_AUTO,
+           workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
     """Y NHWC [B][P][Q][Cout] (fp32) = CCI-sparse convolution of X NHWC [B][H][W][Cin]."""
     _cuda_contig(X, "X")
     B, H, W, Cin = X.shape
     P, Q = conv_out_hw(H, W, KH, KW, stride, pad)
     Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=torch.float32,
                                                 device=X.device)
-    code = lib().cci_conv2d_ex(X.data_ptr(), _dtype_code(X), B, H, W, Cin, values.data_ptr(),
+    if workspace is None and algo == ALGO_DENSE_TC_WS:
+        workspace = new_workspace(algo, X.dtype, Cout, KH * KW * Cin, X.device)
+    wp, wb = _ws(workspace)
+    code = lib().cci_conv2d_ws(X.data_ptr(), _dtype_code(X), B, H, W, Cin, values.data_ptr(),
                                idx.data_ptr(), Cout, KH, KW, stride[0], stride[1], pad[0], pad[1],
                                G, K, Y.data_ptr(), status.data_ptr() if status is not None else None,
-                               algo, _stream(X.device))
+                               algo, wp, wb, _stream(X.device))
     _check(code, "cci_conv2d")
     return Y
 

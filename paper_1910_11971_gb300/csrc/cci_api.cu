@@ -72,13 +72,29 @@ bool regtile_ptr_ok(const FwdParams &p)
 
 cci_status to_status(cudaError_t e) { return e == cudaSuccess ? CCI_OK : CCI_ERR_CUDA; }
 
-cci_status forward(const FwdParams &p, int dtype, int G, int K, cci_algo algo, cudaStream_t stream)
+size_t dense_ws_bytes(int64_t Cout, int64_t R) { return static_cast<size_t>(Cout) * static_cast<size_t>(R) * 2; }
+
+bool dense_tc_shape_ok(int dtype, int G, int K, int64_t Cin, int64_t R)
+{
+    return dense_tc_supported(dtype, G, K) && Cin % 8 == 0 && R % 8 == 0;
+}
+
+cci_status forward(FwdParams p, int dtype, int G, int K, cci_algo algo, void *ws, size_t ws_bytes,
+                   cudaStream_t stream)
 {
     if (p.N == 0) return CCI_OK;
-    if (algo == CCI_ALGO_DENSE_TC) {
-        if (!dense_tc_supported(dtype, G, K) || p.Cin % 8 != 0 || !aligned(p.X, 16) || !aligned(p.Y, 16))
+    if (algo == CCI_ALGO_AUTO && dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) && ws &&
+        ws_bytes >= dense_ws_bytes(p.Cout, p.R) && aligned(ws, 16) && aligned(p.X, 16) && aligned(p.Y, 16))
+        algo = CCI_ALGO_DENSE_TC_WS;
+    if (algo == CCI_ALGO_DENSE_TC || algo == CCI_ALGO_DENSE_TC_WS) {
+        const bool use_ws = algo == CCI_ALGO_DENSE_TC_WS;
+        if (!dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) || !aligned(p.X, 16) || !aligned(p.Y, 16))
             return CCI_ERR_UNSUPPORTED;
-        return to_status(launch_dense_tc(p, G, K, stream));
+        if (use_ws) {
+            if (!ws || ws_bytes < dense_ws_bytes(p.Cout, p.R) || !aligned(ws, 16)) return CCI_ERR_WORKSPACE;
+            p.wdense = ws;
+        }
+        return to_status(launch_dense_tc(p, G, K, use_ws, stream));
     }
     if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
         const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
@@ -137,7 +153,8 @@ const char *cci_status_string(cci_status s)
         case CCI_ERR_CUDA: return "CUDA launch or runtime error";
         case CCI_ERR_TIMEOUT: return "a bounded wait inside a kernel expired";
         case CCI_ERR_UNSUPPORTED: return "request not supported by this build";
-        case CCI_ERR_INDEX: return "a packed index >= G";
+        case CCI_ERR_INDEX: return "a packed index >= G (dense kernels: or not strictly increasing)";
+        case CCI_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
     }
     return "unknown status";
 }
@@ -163,9 +180,9 @@ cci_status cci_pack(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int
                                  reinterpret_cast<cudaStream_t>(stream)));
 }
 
-cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+cci_status cci_linear_ws(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
                          const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
-                         cci_algo algo, cci_stream_t stream)
+                         cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream)
 {
     const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, Cin, G, K);
     if (st != CCI_OK) return st;
@@ -184,7 +201,14 @@ cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
     p.KH = p.KW = p.sh = p.sw = 1;
     p.ph = p.pw = 0;
     p.is_conv = 0;
-    return forward(p, dtype, G, K, algo, reinterpret_cast<cudaStream_t>(stream));
+    return forward(p, dtype, G, K, algo, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+                         const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
+                         cci_algo algo, cci_stream_t stream)
+{
+    return cci_linear_ws(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, algo, nullptr, 0, stream);
 }
 
 cci_status cci_linear(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
@@ -194,10 +218,10 @@ cci_status cci_linear(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, co
     return cci_linear_ex(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, CCI_ALGO_AUTO, stream);
 }
 
-cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
+cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
                          const void *values, const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h,
                          int stride_w, int pad_h, int pad_w, int G, int K, float *Y, uint32_t *dev_status,
-                         cci_algo algo, cci_stream_t stream)
+                         cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream)
 {
     if (B < 0 || H < 1 || W < 1 || Cin < 1 || KH < 1 || KW < 1 || stride_h < 1 || stride_w < 1 || pad_h < 0 ||
         pad_w < 0)
@@ -235,7 +259,23 @@ cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
     p.ph = pad_h;
     p.pw = pad_w;
     p.is_conv = 1;
-    return forward(p, dtype, G, K, algo, reinterpret_cast<cudaStream_t>(stream));
+    return forward(p, dtype, G, K, algo, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
+                         const void *values, const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h,
+                         int stride_w, int pad_h, int pad_w, int G, int K, float *Y, uint32_t *dev_status,
+                         cci_algo algo, cci_stream_t stream)
+{
+    return cci_conv2d_ws(X, dtype, B, H, W, Cin, values, idx, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, G, K,
+                         Y, dev_status, algo, nullptr, 0, stream);
+}
+
+size_t cci_workspace_size(cci_algo algo, cci_dtype dtype, int64_t Cout, int64_t R)
+{
+    if (Cout < 1 || R < 1 || !mul_ok(Cout, R)) return 0;
+    if (algo == CCI_ALGO_DENSE_TC_WS || (algo == CCI_ALGO_AUTO && dtype == CCI_BF16)) return dense_ws_bytes(Cout, R);
+    return 0;
 }
 
 cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
@@ -250,13 +290,26 @@ cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int6
 const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K, cci_algo algo)
 {
     if (!valid_dtype(dtype) || Cin < 1 || R < Cin || check_group(Cout, G, K) != CCI_OK) return "";
+    if (algo == CCI_ALGO_DENSE_TC_WS) {
+        static const char *names_ws[] = {"dense_tc_ws_bf16_G4_K1", "dense_tc_ws_bf16_G4_K2", "dense_tc_ws_bf16_G8_K1",
+                                         "dense_tc_ws_bf16_G8_K2", "dense_tc_ws_bf16_G8_K4", "dense_tc_ws_bf16_G16_K1",
+                                         "dense_tc_ws_bf16_G16_K2", "dense_tc_ws_bf16_G16_K4", "dense_tc_ws_bf16_G16_K8",
+                                         "dense_tc_ws_bf16_G32_K1", "dense_tc_ws_bf16_G32_K2", "dense_tc_ws_bf16_G32_K4",
+                                         "dense_tc_ws_bf16_G32_K8", "dense_tc_ws_bf16_G32_K16"};
+        if (!dense_tc_shape_ok(dtype, G, K, Cin, R)) return "";
+        int i = 0;
+        for (int g = 4; g <= 32; g *= 2)
+            for (int k = 1; k <= g / 2; k *= 2, ++i)
+                if (g == G && k == K) return names_ws[i];
+        return "";
+    }
     if (algo == CCI_ALGO_DENSE_TC) {
         static const char *names[] = {"dense_tc_bf16_G4_K1", "dense_tc_bf16_G4_K2", "dense_tc_bf16_G8_K1",
                                       "dense_tc_bf16_G8_K2", "dense_tc_bf16_G8_K4", "dense_tc_bf16_G16_K1",
                                       "dense_tc_bf16_G16_K2", "dense_tc_bf16_G16_K4", "dense_tc_bf16_G16_K8",
                                       "dense_tc_bf16_G32_K1", "dense_tc_bf16_G32_K2", "dense_tc_bf16_G32_K4",
                                       "dense_tc_bf16_G32_K8", "dense_tc_bf16_G32_K16"};
-        if (!dense_tc_supported(dtype, G, K) || Cin % 8 != 0) return "";
+        if (!dense_tc_shape_ok(dtype, G, K, Cin, R)) return "";
         int i = 0;
         for (int g = 4; g <= 32; g *= 2)
             for (int k = 1; k <= g / 2; k *= 2, ++i)

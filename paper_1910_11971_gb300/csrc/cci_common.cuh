@@ -25,6 +25,7 @@ struct FwdParams {
     int64_t P, Q;   // output image (1 x 1 for a product)
     int KH, KW, sh, sw, ph, pw;
     int is_conv;
+    const void *wdense;  // dense decompressed weights [Cout][R] (workspace kernels only)
 };
 
 __device__ __forceinline__ void report(uint32_t *status, cci_status code)

@@ -158,7 +158,9 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32])
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-template <int G, int K>
+// WS = false: the producers decompress the CTA's packed groups into the B tile;
+// WS = true: B is copied (cp.async) from the dense workspace p.wdense [Cout][R]
+template <int G, int K, bool WS>
 __global__ void __launch_bounds__(kThreads, 1) dense_tc_kernel(FwdParams p, int64_t n_ct, int64_t n_tiles)
 {
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -253,10 +255,22 @@ __global__ void __launch_bounds__(kThreads, 1) dense_tc_kernel(FwdParams p, int6
                     }
                     cp_async16(a_smem + s * kATile + sw128(row, chunk * 8), src, valid);
                 }
+                const uint32_t bt = b_smem + s * kBTile;
+                if constexpr (WS) {
+                    // B: 256 rows x 8 chunks of the dense weights; rows rowb + 16 i, chunk `chunk`
+                    const uint16_t *Wd = static_cast<const uint16_t *>(p.wdense);
+                    const int64_t co0 = ct * kN;
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        const int row = rowb + 16 * i;
+                        const bool valid = co0 + row < p.Cout && rok;
+                        cp_async16(bt + sw128(row, chunk * 8), valid ? Wd + (co0 + row) * p.R + r : Wd, valid);
+                    }
+                }
                 asm volatile("cp.async.commit_group;" ::: "memory");
+                if constexpr (!WS) {
                 // B: units (group, 8-index chunk): zero the group's G rows of the
                 // chunk, then write the K kept values of each of the 8 indices
-                const uint32_t bt = b_smem + s * kBTile;
                 for (int u = pt; u < (kN / G) * 8; u += 128) {
                     const int gl = u >> 3, chunk = u & 7;
 #pragma unroll
@@ -268,17 +282,20 @@ __global__ void __launch_bounds__(kThreads, 1) dense_tc_kernel(FwdParams p, int6
                         const int64_t r = r0 + chunk * 8 + e;
                         if (r >= p.R) break;
                         const int64_t o = (gg * p.R + r) * K;
+                        int prev = -1;
 #pragma unroll
                         for (int sl = 0; sl < K; ++sl) {
                             const int i = __ldg(p.idx + o + sl);
-                            if (i >= G) {
+                            if (i >= G || i <= prev) {  // index sets must be strictly increasing
                                 report(p.status, CCI_ERR_INDEX);
                                 continue;
                             }
+                            prev = i;
                             const uint16_t val = __ldg(V + o + sl);
                             st_shared_b16(bt + sw128(gl * G + i, chunk * 8 + e), val);
                         }
                     }
+                }
                 }
                 // stage it - kLag is complete for this thread: its copies landed
                 if (it >= kLag) {
@@ -370,10 +387,10 @@ __global__ void __launch_bounds__(kThreads, 1) dense_tc_kernel(FwdParams p, int6
     }
 }
 
-template <int G, int K>
+template <int G, int K, bool WS>
 cudaError_t launch(const FwdParams &p, cudaStream_t stream)
 {
-    auto kern = dense_tc_kernel<G, K>;
+    auto kern = dense_tc_kernel<G, K, WS>;
     static const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmemBytes));
     if (attr != cudaSuccess) return attr;
@@ -390,11 +407,52 @@ cudaError_t launch(const FwdParams &p, cudaStream_t stream)
 
 }  // namespace tc
 
-// (G, K) pairs with a dense tensor-core instantiation (G divides the 256-channel tile)
-cudaError_t launch_dense_tc(const FwdParams &p, int G, int K, cudaStream_t stream)
+// one thread per (group gi, r): the G weights W[gi*G + j][r] of the dense
+// matrix, zero except the K kept ones (bf16 copied bit for bit); index sets
+// must be strictly increasing (as cci_pack writes them)
+template <int G, int K>
+__global__ void decompress_bf16_kernel(const uint16_t *__restrict__ values, const uint8_t *__restrict__ idx,
+                                       int64_t Cout, int64_t R, uint16_t *__restrict__ wd, uint32_t *status)
 {
-#define CCI_TC_CASE(g, k) \
-    if (G == g && K == k) return tc::launch<g, k>(p, stream);
+    const int64_t total = (Cout / G) * R;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gi = t / R, r = t - gi * R;
+        uint16_t v[K];
+        int ix[K];
+        bool bad = false;
+#pragma unroll
+        for (int s = 0; s < K; ++s) {
+            v[s] = values[t * K + s];
+            ix[s] = idx[t * K + s];
+            bad |= ix[s] >= G || (s > 0 && ix[s] <= ix[s - 1]);
+        }
+        if (bad) report(status, CCI_ERR_INDEX);
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+            uint16_t o = 0;
+#pragma unroll
+            for (int s = 0; s < K; ++s) o = (ix[s] == j) ? v[s] : o;
+            wd[(gi * G + j) * R + r] = o;
+        }
+    }
+}
+
+// (G, K) pairs with a dense tensor-core instantiation (G divides the 256-channel tile)
+cudaError_t launch_dense_tc(const FwdParams &p, int G, int K, bool ws, cudaStream_t stream)
+{
+#define CCI_TC_CASE(g, k)                                                                          \
+    if (G == g && K == k) {                                                                        \
+        if (!ws) return tc::launch<g, k, false>(p, stream);                                        \
+        const int64_t total = (p.Cout / g) * p.R;                                                  \
+        const int64_t blocks = (total + 255) / 256;                                                \
+        decompress_bf16_kernel<g, k><<<static_cast<unsigned>(blocks < 65536 * 8 ? blocks : 65536 * 8), 256, 0, \
+                                       stream>>>(static_cast<const uint16_t *>(p.values), p.idx, p.Cout, p.R, \
+                                                 static_cast<uint16_t *>(const_cast<void *>(p.wdense)), p.status); \
+        const cudaError_t e = cudaGetLastError();                                                  \
+        if (e != cudaSuccess) return e;                                                            \
+        return tc::launch<g, k, true>(p, stream);                                                  \
+    }
     CCI_TC_CASE(4, 1) CCI_TC_CASE(4, 2)
     CCI_TC_CASE(8, 1) CCI_TC_CASE(8, 2) CCI_TC_CASE(8, 4)
     CCI_TC_CASE(16, 1) CCI_TC_CASE(16, 2) CCI_TC_CASE(16, 4) CCI_TC_CASE(16, 8)

@@ -135,6 +135,21 @@ def test_kernel_names(lib):
     assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2, cci.ALGO_GENERIC) == "generic_f32"
 
 
+def test_workspace_rules(lib):
+    import torch
+    ws = cci.ALGO_DENSE_TC_WS
+    assert cci.workspace_size(ws, torch.bfloat16, 256, 64) == 256 * 64 * 2
+    assert cci.workspace_size(cci.ALGO_EXPAND, torch.bfloat16, 256, 64) == 0
+    assert cci.workspace_size(cci.ALGO_AUTO, torch.float32, 256, 64) == 0
+    assert cci.workspace_size(cci.ALGO_AUTO, torch.bfloat16, 256, 64) == 256 * 64 * 2
+    # the family needs a workspace: rejected before any launch (no device needed)
+    assert linear(lib, dt=1, algo=ws) == 11
+    assert lib.cci_linear_ws(FAKE, 1, 16, 16, FAKE, FAKE, 16, 8, 2, FAKE, None, ws, FAKE, 16, None) == 11
+    assert lib.cci_linear_ws(FAKE, 1, 16, 16, FAKE, FAKE, 16, 8, 2, FAKE, None, ws, FAKE + 8, 4096, None) == 11
+    assert cci.kernel_name(torch.bfloat16, 64, 64, 256, 8, 2, ws) == "dense_tc_ws_bf16_G8_K2"
+    assert cci.kernel_name(torch.bfloat16, 8, 36, 256, 8, 2, ws) == ""  # R % 8 != 0
+
+
 def test_fma_probe_rejects(lib):
     assert lib.cci_fma_probe(None, 1, 32, 1, None) == NULL
     assert lib.cci_fma_probe(FAKE, 0, 32, 1, None) == SHAPE

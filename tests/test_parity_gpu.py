@@ -349,22 +349,28 @@ DENSE_SMALL = [
 ]
 
 
+DENSE_ALGOS = [cci.ALGO_DENSE_TC, cci.ALGO_DENSE_TC_WS]
+DENSE_IDS = ["smem", "ws"]
+
+
+@pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
 @pytest.mark.parametrize("case", DENSE_SMALL, ids=lambda c: "N{}_C{}x{}_G{}K{}".format(*c))
-def test_dense_tc_small(dev, case):
+def test_dense_tc_small(dev, case, algo):
     N, Cin, Cout, G, K = case
     X, W = wl.random_small(N * 3 + Cin, "bf16", N, Cin, Cout)
-    assert cci.kernel_name(BF16, Cin, Cin, Cout, G, K, cci.ALGO_DENSE_TC).startswith("dense_tc")
-    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC)
+    assert cci.kernel_name(BF16, Cin, Cin, Cout, G, K, algo).startswith("dense_tc")
+    Y = run_linear(dev, X, W, G, K, algo)
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.linear(f64(X), Wd, mask)
     assert_within_tol(f64(Y), Yo, S, str(case))
 
 
+@pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
 @pytest.mark.parametrize("G,K", wl.SWEEP_POINTS)
-def test_dense_tc_sweep_full(dev, G, K):
+def test_dense_tc_sweep_full(dev, G, K, algo):
     case = wl.sweep_case(G, K)
     X, W = wl.linear_inputs(case, device="cpu")
-    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC)
+    Y = run_linear(dev, X, W, G, K, algo)
     assert torch.isfinite(Y).all()
     rows = sample_rows(case.N, 192, seed=G * 37 + K)
     _, _, Wd, mask = oracle_reference(W, G, K)
@@ -375,22 +381,24 @@ def test_dense_tc_sweep_full(dev, G, K):
 @pytest.mark.parametrize("case", [c for c in CONV_SMALL if c[-1] == "bf16" and c[3] % 8 == 0 and c[9] in (4, 8, 16, 32)
                                   and (c[10] & (c[10] - 1)) == 0 and c[10] <= c[9] // 2],
                          ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
-def test_dense_tc_conv_small(dev, case):
+@pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
+def test_dense_tc_conv_small(dev, case, algo):
     B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
     g = torch.Generator().manual_seed(B * 11 + Cin)
     X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(BF16)
     W = torch.randn((Cout, KH * KW * Cin), generator=g).to(BF16)
-    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K, cci.ALGO_DENSE_TC)
+    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K, algo)
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
     assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
 
 
-def test_dense_tc_conv3x3_full(dev):
+@pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
+def test_dense_tc_conv3x3_full(dev, algo):
     case = wl.CONV3X3_28
     X, W = wl.conv_inputs(case, device="cpu")
     Y = run_conv(dev, X, W, (case.KH, case.KW, (case.stride,) * 2, (case.pad,) * 2, case.Cout),
-                 case.G, case.K, cci.ALGO_DENSE_TC)
+                 case.G, case.K, algo)
     assert torch.isfinite(Y).all()
     pts = conv_points(case, 1024, 5)
     Xs = f64(X[[0, case.B - 1]])
@@ -399,3 +407,31 @@ def test_dense_tc_conv3x3_full(dev):
     _, _, Wd, mask = oracle_reference(W, case.G, case.K)
     Yo, S = oracle.conv2d(Xs, Wd, mask, 3, 3, (1, 1), (1, 1), pts=local)
     assert_within_tol(f64(Y.reshape(-1, case.Cout)[torch.from_numpy(pts).to(dev)]), Yo, S, "conv3x3 dense_tc")
+
+
+@pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
+def test_dense_tc_rejects_repeated_indices(dev, algo):
+    """A dense tile holds one weight per (channel, r): index sets must be strictly
+    increasing (cci_pack's output); anything else is reported."""
+    G, K, Cout, Cin, N = 8, 2, 256, 64, 128
+    v = torch.ones((Cout // G, Cin, K), dtype=BF16, device=dev)
+    i = torch.zeros((Cout // G, Cin, K), dtype=torch.uint8, device=dev)
+    i[..., 1] = 3
+    i[2, 7, 1] = 0  # repeated index
+    X = torch.randn(N, Cin, device=dev).to(BF16)
+    st = cci.new_status(dev)
+    cci.linear(X, v, i, Cout, G, K, status=st, algo=algo)
+    assert cci.read_status(st) == 10
+
+
+def test_auto_with_workspace_uses_dense_tc_ws(dev):
+    """AUTO picks the dense tensor-core family for bf16 when given a workspace."""
+    N, Cin, Cout, G, K = 300, 64, 256, 8, 2
+    X, W = wl.random_small(4, "bf16", N, Cin, Cout)
+    Xd = X.to(dev)
+    v, i = cci.pack(W.to(dev), G, K)
+    ws = cci.new_workspace(cci.ALGO_AUTO, BF16, Cout, Cin, dev)
+    assert ws is not None and ws.numel() == Cout * Cin * 2
+    Ya = cci.linear(Xd, v, i, Cout, G, K, workspace=ws)
+    Yw = cci.linear(Xd, v, i, Cout, G, K, algo=cci.ALGO_DENSE_TC_WS)
+    assert torch.equal(Ya.view(torch.int32), Yw.view(torch.int32))
