@@ -195,6 +195,38 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
                          int G, int K, float *Y, uint32_t *dev_status, cci_algo algo,
                          void *workspace, size_t workspace_bytes, cci_stream_t stream);
 
+/* Largest dense-weight size (Cout*R*2 bytes) that cci_linear_dense_tc_static accepts. */
+#define CCI_STATIC_WORKSPACE_BYTES (16u * 1024u * 1024u)
+
+/*
+ * cci_linear_dense_tc_static -- the product of cci_linear_ws with
+ * CCI_ALGO_DENSE_TC_WS, for callers that cannot allocate device memory
+ * themselves: for example a plug-in called by a host framework that owns all
+ * device memory and hands it no allocator, or a latency-bound serving loop that
+ * forbids allocations after start-up.  Such a caller still passes X, the packed
+ * weights and Y, but no workspace: the dense weights are decompressed into a
+ * scratch array that lives in the library itself (a static device array of
+ * CCI_STATIC_WORKSPACE_BYTES, held by every GPU that loads the library until the
+ * process exits).  This entry point calls no allocation routine.  (The paper
+ * has no counterpart: this is a deployment convenience of this library.)
+ *
+ *   arguments  as cci_linear (bf16 only, Cin % 8 == 0, 16-byte aligned X and Y)
+ * Rules:
+ *   - Cout*Cin*2 > CCI_STATIC_WORKSPACE_BYTES is rejected with CCI_ERR_WORKSPACE;
+ *   - the first call on a device looks up the array's device address on that
+ *     device (the device current at the call); make that first call before any
+ *     stream capture;
+ *   - every call shares the one array per device and leaves it holding the last
+ *     call's dense weights; each call rewrites the part it reads, so nothing
+ *     needs clearing, but calls that overlap on the GPU (other streams, other
+ *     threads) race on the array and must be serialised by the caller.
+ * Errors: as cci_linear; CCI_ERR_UNSUPPORTED for shapes the dense kernel lacks;
+ *         CCI_ERR_CUDA if the address lookup fails.
+ */
+cci_status cci_linear_dense_tc_static(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
+                                      const void *values, const uint8_t *idx, int64_t Cout, int G,
+                                      int K, float *Y, uint32_t *dev_status, cci_stream_t stream);
+
 /*
  * cci_kernel_name -- the name of the kernel that cci_linear_ex / cci_conv2d_ex
  * would launch for a layer with these sizes (R = Cin for a product, Cin*KH*KW

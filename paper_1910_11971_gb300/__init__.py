@@ -47,6 +47,8 @@ SIGNATURES = {
     "cci_conv2d_ws": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32, _I32,
                              _I32, _I32, _I32, _I32, _P, _U32P, _I32, _P, ctypes.c_size_t, _P]),
     "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
+    "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
+                                          _P]),
     "cci_kernel_name": (ctypes.c_char_p, [_I32, _I64, _I64, _I64, _I32, _I32, _I32]),
     "cci_status_string": (ctypes.c_char_p, [_I32]),
     "cci_decode_device_status": (_I32, [ctypes.c_uint32]),

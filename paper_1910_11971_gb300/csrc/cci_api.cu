@@ -4,6 +4,7 @@
 // kernel, launch on the caller's stream.  The library allocates nothing.
 #include <cstdint>
 #include <cstring>
+#include <mutex>
 
 #include "cci_kernels.h"
 
@@ -335,3 +336,51 @@ cci_status cci_fma_probe(float *out, int blocks, int threads, int iters, cci_str
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Static-scratch product for callers that cannot allocate device memory.
+// The dense-weight scratch is this file-scope device array; host code here
+// looks up its device address once per device (cudaGetSymbolAddress, with that
+// device current) and passes the address to the kernels as their workspace.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kStaticWsBytes = CCI_STATIC_WORKSPACE_BYTES;
+static __device__ __align__(256) unsigned char g_static_ws[kStaticWsBytes];
+
+constexpr int kMaxDevices = 64;
+std::mutex g_static_ws_mutex;
+void *g_static_ws_ptr[kMaxDevices] = {};
+
+// device address of g_static_ws on the current device (looked up on first use)
+cci_status static_ws_address(void **out)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return CCI_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_static_ws_mutex);
+    if (!g_static_ws_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_static_ws) != cudaSuccess || !p) return CCI_ERR_CUDA;
+        g_static_ws_ptr[dev] = p;
+    }
+    *out = g_static_ws_ptr[dev];
+    return CCI_OK;
+}
+
+}  // namespace
+
+extern "C" cci_status cci_linear_dense_tc_static(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
+                                                 const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
+                                                 float *Y, uint32_t *dev_status, cci_stream_t stream)
+{
+    const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, Cin, G, K);
+    if (st != CCI_OK) return st;
+    if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
+    if (dense_ws_bytes(Cout, Cin) > kStaticWsBytes) return CCI_ERR_WORKSPACE;
+    if (N == 0) return CCI_OK;
+    void *ws = nullptr;
+    const cci_status a = static_ws_address(&ws);
+    if (a != CCI_OK) return a;
+    return cci_linear_ws(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, CCI_ALGO_DENSE_TC_WS, ws,
+                         kStaticWsBytes, stream);
+}
