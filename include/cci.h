@@ -92,10 +92,12 @@ typedef enum cci_algo {
                                memory and all G rows are updated; same shape rules as
                                CCI_ALGO_REGTILE */
     CCI_ALGO_DENSE_TC_WS = 5  /* decompress the packed weights once per call into a caller
-                               workspace (dense bf16 [Cout][R]) and multiply densely on the
-                               tensor cores (tcgen05), operands streamed by cp.async;
-                               bf16 only, Cin % 8 == 0, R % 8 == 0; needs
-                               cci_workspace_size() bytes */
+                               workspace and multiply densely on the tensor cores (tcgen05),
+                               operands streamed by cp.async.  bf16: dense bf16 [Cout][R],
+                               Cin % 8 == 0, R % 8 == 0.  fp32: hi and lo tf32 planes
+                               [2][Cout][R] and a three-pass tf32 product (hi*hi + hi*lo +
+                               lo*hi, |error| below 2^-21 of sum |w||x|), Cin % 4 == 0,
+                               R % 4 == 0.  Needs cci_workspace_size() bytes */
 } cci_algo;
 
 /*
@@ -172,9 +174,9 @@ cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
 /*
  * cci_workspace_size -- bytes of device workspace that cci_linear_ws /
  * cci_conv2d_ws need for this kernel family and layer (R = Cin for a product,
- * Cin*KH*KW for a convolution): Cout*R*2 for CCI_ALGO_DENSE_TC_WS, 0 for the
- * families that need none.  For CCI_ALGO_AUTO: the bytes that let AUTO pick its
- * fastest family for a bf16 layer (0 for fp32).
+ * Cin*KH*KW for a convolution): for CCI_ALGO_DENSE_TC_WS Cout*R*2 (bf16) or
+ * Cout*R*8 (fp32), 0 for the families that need none.  For CCI_ALGO_AUTO: the
+ * bytes that let AUTO pick its fastest family (the dense tensor-core one).
  */
 size_t cci_workspace_size(cci_algo algo, cci_dtype dtype, int64_t Cout, int64_t R);
 
@@ -183,7 +185,8 @@ size_t cci_workspace_size(cci_algo algo, cci_dtype dtype, int64_t Cout, int64_t 
  * aligned, `workspace_bytes` long; NULL / 0 allowed for families that need
  * none).  The call overwrites the workspace; calls that overlap on the GPU must
  * use different workspaces.  CCI_ALGO_AUTO uses the dense tensor-core family
- * for bf16 layers when the workspace is large enough, else the CUDA-core family.
+ * when the layer has one and the workspace is large enough, else the CUDA-core
+ * family.
  */
 cci_status cci_linear_ws(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
                          const void *values, const uint8_t *idx, int64_t Cout, int G, int K,

@@ -73,11 +73,17 @@ bool regtile_ptr_ok(const FwdParams &p)
 
 cci_status to_status(cudaError_t e) { return e == cudaSuccess ? CCI_OK : CCI_ERR_CUDA; }
 
-size_t dense_ws_bytes(int64_t Cout, int64_t R) { return static_cast<size_t>(Cout) * static_cast<size_t>(R) * 2; }
+// workspace of the dense tensor-core family: bf16 dense weights [Cout][R], or
+// for fp32 the hi and lo tf32 planes [2][Cout][R] of 4-byte elements
+size_t dense_ws_bytes(int dtype, int64_t Cout, int64_t R)
+{
+    return static_cast<size_t>(Cout) * static_cast<size_t>(R) * (dtype == CCI_F32 ? 8 : 2);
+}
 
 bool dense_tc_shape_ok(int dtype, int G, int K, int64_t Cin, int64_t R)
 {
-    return dense_tc_supported(dtype, G, K) && Cin % 8 == 0 && R % 8 == 0;
+    const int64_t v = dtype == CCI_F32 ? 4 : 8;  // elements per 16 bytes
+    return dense_tc_supported(dtype, G, K) && Cin % v == 0 && R % v == 0;
 }
 
 cci_status forward(FwdParams p, int dtype, int G, int K, cci_algo algo, void *ws, size_t ws_bytes,
@@ -85,17 +91,18 @@ cci_status forward(FwdParams p, int dtype, int G, int K, cci_algo algo, void *ws
 {
     if (p.N == 0) return CCI_OK;
     if (algo == CCI_ALGO_AUTO && dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) && ws &&
-        ws_bytes >= dense_ws_bytes(p.Cout, p.R) && aligned(ws, 16) && aligned(p.X, 16) && aligned(p.Y, 16))
+        ws_bytes >= dense_ws_bytes(dtype, p.Cout, p.R) && aligned(ws, 16) && aligned(p.X, 16) && aligned(p.Y, 16))
         algo = CCI_ALGO_DENSE_TC_WS;
     if (algo == CCI_ALGO_DENSE_TC || algo == CCI_ALGO_DENSE_TC_WS) {
         const bool use_ws = algo == CCI_ALGO_DENSE_TC_WS;
         if (!dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) || !aligned(p.X, 16) || !aligned(p.Y, 16))
             return CCI_ERR_UNSUPPORTED;
+        if (!use_ws && dtype != CCI_BF16) return CCI_ERR_UNSUPPORTED;  // shared-memory decompression: bf16 only
         if (use_ws) {
-            if (!ws || ws_bytes < dense_ws_bytes(p.Cout, p.R) || !aligned(ws, 16)) return CCI_ERR_WORKSPACE;
+            if (!ws || ws_bytes < dense_ws_bytes(dtype, p.Cout, p.R) || !aligned(ws, 16)) return CCI_ERR_WORKSPACE;
             p.wdense = ws;
         }
-        return to_status(launch_dense_tc(p, G, K, use_ws, stream));
+        return to_status(launch_dense_tc(p, dtype, G, K, use_ws, stream));
     }
     if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
         const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
@@ -275,7 +282,8 @@ cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
 size_t cci_workspace_size(cci_algo algo, cci_dtype dtype, int64_t Cout, int64_t R)
 {
     if (Cout < 1 || R < 1 || !mul_ok(Cout, R)) return 0;
-    if (algo == CCI_ALGO_DENSE_TC_WS || (algo == CCI_ALGO_AUTO && dtype == CCI_BF16)) return dense_ws_bytes(Cout, R);
+    if (!valid_dtype(dtype)) return 0;
+    if (algo == CCI_ALGO_DENSE_TC_WS || algo == CCI_ALGO_AUTO) return dense_ws_bytes(dtype, Cout, R);
     return 0;
 }
 
@@ -297,14 +305,22 @@ const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cou
                                          "dense_tc_ws_bf16_G16_K2", "dense_tc_ws_bf16_G16_K4", "dense_tc_ws_bf16_G16_K8",
                                          "dense_tc_ws_bf16_G32_K1", "dense_tc_ws_bf16_G32_K2", "dense_tc_ws_bf16_G32_K4",
                                          "dense_tc_ws_bf16_G32_K8", "dense_tc_ws_bf16_G32_K16"};
+        static const char *names_tf[] = {"dense_tc_ws_tf32x3_G4_K1", "dense_tc_ws_tf32x3_G4_K2",
+                                         "dense_tc_ws_tf32x3_G8_K1", "dense_tc_ws_tf32x3_G8_K2",
+                                         "dense_tc_ws_tf32x3_G8_K4", "dense_tc_ws_tf32x3_G16_K1",
+                                         "dense_tc_ws_tf32x3_G16_K2", "dense_tc_ws_tf32x3_G16_K4",
+                                         "dense_tc_ws_tf32x3_G16_K8", "dense_tc_ws_tf32x3_G32_K1",
+                                         "dense_tc_ws_tf32x3_G32_K2", "dense_tc_ws_tf32x3_G32_K4",
+                                         "dense_tc_ws_tf32x3_G32_K8", "dense_tc_ws_tf32x3_G32_K16"};
         if (!dense_tc_shape_ok(dtype, G, K, Cin, R)) return "";
         int i = 0;
         for (int g = 4; g <= 32; g *= 2)
             for (int k = 1; k <= g / 2; k *= 2, ++i)
-                if (g == G && k == K) return names_ws[i];
+                if (g == G && k == K) return dtype == CCI_F32 ? names_tf[i] : names_ws[i];
         return "";
     }
     if (algo == CCI_ALGO_DENSE_TC) {
+        if (dtype != CCI_BF16) return "";
         static const char *names[] = {"dense_tc_bf16_G4_K1", "dense_tc_bf16_G4_K2", "dense_tc_bf16_G8_K1",
                                       "dense_tc_bf16_G8_K2", "dense_tc_bf16_G8_K4", "dense_tc_bf16_G16_K1",
                                       "dense_tc_bf16_G16_K2", "dense_tc_bf16_G16_K4", "dense_tc_bf16_G16_K8",
@@ -375,8 +391,9 @@ extern "C" cci_status cci_linear_dense_tc_static(const void *X, cci_dtype dtype,
 {
     const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, Cin, G, K);
     if (st != CCI_OK) return st;
+    if (dtype != CCI_BF16) return CCI_ERR_UNSUPPORTED;  // the array holds bf16 dense weights
     if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
-    if (dense_ws_bytes(Cout, Cin) > kStaticWsBytes) return CCI_ERR_WORKSPACE;
+    if (dense_ws_bytes(dtype, Cout, Cin) > kStaticWsBytes) return CCI_ERR_WORKSPACE;
     if (N == 0) return CCI_OK;
     void *ws = nullptr;
     const cci_status a = static_ws_address(&ws);

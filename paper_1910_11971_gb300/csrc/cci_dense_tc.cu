@@ -407,6 +407,305 @@ cudaError_t launch(const FwdParams &p, cudaStream_t stream)
 
 }  // namespace tc
 
+// ===========================================================================
+// fp32 layers: three-pass tf32 product.  Every fp32 operand x is split as
+// x = hi + lo with hi = x with the low 13 mantissa bits cleared (exactly a
+// tf32 value) and lo = x - hi (exact in fp32); the product uses
+// hi*hi + hi*lo + lo*hi.  The dropped lo*lo term and the tf32 conversion of lo
+// are each below 2^-22 of |x||w|, whether the tensor core truncates or rounds.
+// Tile D[128 n][128 co], 32 fp32 (128 bytes) of r per stage, 3 stages; A planes
+// written by the producers from registers, B planes copied from the workspace
+// [2][Cout][R] (hi plane, then lo plane).
+// ===========================================================================
+namespace tf {
+
+constexpr int kM = 128, kN = 128, kKS = 32, kStages = 3, kLag = 1;
+constexpr int kThreads = 288;
+constexpr int kPlane = kM * kKS * 4;          // 16 KB: one 128 x 32 fp32 plane (A or B)
+constexpr int kStage = 4 * kPlane;            // A hi, A lo, B hi, B lo
+constexpr int kTmemCols = 256;                // two 128-column accumulators
+constexpr size_t kSmemBytes = 1024 + kStages * kStage + sizeof(tc::Smem) + 64;
+constexpr uint32_t kIdesc = (1u << 4)                 // D f32
+                            | (2u << 7) | (2u << 10)  // A, B tf32
+                            | (static_cast<uint32_t>(kN >> 3) << 17) | (static_cast<uint32_t>(kM >> 4) << 24);
+
+__device__ __forceinline__ void mma_tf32(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate)
+{
+    asm volatile(
+        "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
+        : "memory");
+}
+
+// byte offset of (row, element k) in a K-major plane of 128-byte rows (32 fp32)
+// with the 128-byte swizzle
+__device__ __forceinline__ uint32_t sw128f(int row, int k)
+{
+    return static_cast<uint32_t>(row * 128 + (((k >> 2) ^ (row & 7)) * 16) + (k & 3) * 4);
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
+{
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+
+__device__ __forceinline__ uint32_t hi_bits(uint32_t x) { return x & 0xffffe000u; }
+__device__ __forceinline__ uint32_t lo_bits(uint32_t x)
+{
+    return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
+}
+
+__global__ void __launch_bounds__(kThreads, 1) gemm_tf32x3_kernel(FwdParams p, int64_t n_ct, int64_t n_tiles)
+{
+    using tc::mbar_arrive;
+    using tc::mbar_init;
+    using tc::mbar_wait;
+    using tc::smem_u32;
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const uint32_t raw = smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    unsigned char *gbase = smem_raw + (base - raw);
+    tc::Smem *S = reinterpret_cast<tc::Smem *>(gbase + kStages * kStage);
+    volatile int *abort = &S->abort;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int nks = static_cast<int>((p.R + kKS - 1) / kKS);
+    const float *X = static_cast<const float *>(p.X);
+    const float *Wh = static_cast<const float *>(p.wdense);
+    const float *Wl = Wh + p.Cout * p.R;
+
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&S->full[s], 128);
+            mbar_init(&S->empty[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(&S->tmem_full[a], 1);
+            mbar_init(&S->tmem_empty[a], 128);
+        }
+        mbar_init(&S->drain, 1);
+        S->abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 8) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&S->tmem_base)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = S->tmem_base;
+
+    if (warp >= 4 && warp < 8) {
+        // ------------------------------------------------------------ producers
+        const int pt = tid - 128;
+        const int chunk = pt & 7;  // 16-byte chunk (4 fp32) of every A / B copy of this thread
+        const int rowb = pt >> 3;  // rows rowb + 16 i
+        int it = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            const int64_t ct = tile % n_ct;
+            const int64_t n0 = (tile / n_ct) * kM;
+            const int64_t co0 = ct * kN;
+            ColumnSite site[8];
+            bool colok[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int64_t n = n0 + rowb + 16 * i;
+                colok[i] = n < p.N;
+                site[i] = colok[i] ? column_site(p, n) : ColumnSite{0, 0, 0};
+            }
+            for (int ks = 0; ks < nks && ok; ++ks, ++it) {
+                const int s = it % kStages;
+                // the activation chunks of this stage, read before the buffer is free
+                const int64_t r = static_cast<int64_t>(ks) * kKS + chunk * 4;
+                const bool rok = r < p.R;
+                int kh = 0, kw = 0;
+                int64_t ci = r;
+                if (p.is_conv && rok) {
+                    const int tap = static_cast<int>(r / p.Cin);
+                    ci = r - static_cast<int64_t>(tap) * p.Cin;
+                    kh = tap / p.KW;
+                    kw = tap - kh * p.KW;
+                }
+                uint4 xa[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    xa[i] = make_uint4(0, 0, 0, 0);
+                    bool valid = colok[i] && rok;
+                    int64_t off = site[i].img + r;
+                    if (valid && p.is_conv) {
+                        const int h = site[i].hb + kh, w = site[i].wb + kw;
+                        valid = h >= 0 && h < p.H && w >= 0 && w < p.W;
+                        off = site[i].img + (static_cast<int64_t>(h) * p.W + w) * p.Cin + ci;
+                    }
+                    if (valid) xa[i] = __ldg(reinterpret_cast<const uint4 *>(X + off));
+                }
+                if (it >= kStages) ok = mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
+                if (!ok) break;
+                const uint32_t st = base + s * kStage;
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int row = rowb + 16 * i;
+                    const uint32_t o = sw128f(row, chunk * 4);
+                    st_shared_v4(st + o, hi_bits(xa[i].x), hi_bits(xa[i].y), hi_bits(xa[i].z), hi_bits(xa[i].w));
+                    st_shared_v4(st + kPlane + o, lo_bits(xa[i].x), lo_bits(xa[i].y), lo_bits(xa[i].z),
+                                 lo_bits(xa[i].w));
+                }
+                // B planes: 128 rows x 8 chunks each, from the workspace
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const int row = rowb + 16 * i;
+                    const bool valid = co0 + row < p.Cout && rok;
+                    const int64_t g = (co0 + row) * p.R + r;
+                    const uint32_t o = sw128f(row, chunk * 4);
+                    tc::cp_async16(st + 2 * kPlane + o, valid ? Wh + g : Wh, valid);
+                    tc::cp_async16(st + 3 * kPlane + o, valid ? Wl + g : Wl, valid);
+                }
+                asm volatile("cp.async.commit_group;" ::: "memory");
+                if (it >= kLag) {
+                    asm volatile("cp.async.wait_group %0;" ::"n"(kLag) : "memory");
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    mbar_arrive(&S->full[(it - kLag) % kStages]);
+                }
+            }
+        }
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        for (int q = (it >= kLag ? it - kLag : 0); q < it; ++q) mbar_arrive(&S->full[q % kStages]);
+    } else if (warp == 8) {
+        // ------------------------------------------------------------ MMA issuer
+        int it = 0, t = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+            const int acc = t & 1;
+            if (t >= 2) ok = mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
+            for (int ks = 0; ks < nks && ok; ++ks, ++it) {
+                const int s = it % kStages;
+                ok = mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
+                if (!ok) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                if (lane == 0) {
+                    const uint32_t st = base + s * kStage;
+#pragma unroll
+                    for (int k = 0; k < kKS / 8; ++k) {
+                        const uint64_t ah = tc::sw128_desc(st + k * 32);
+                        const uint64_t al = tc::sw128_desc(st + kPlane + k * 32);
+                        const uint64_t bh = tc::sw128_desc(st + 2 * kPlane + k * 32);
+                        const uint64_t bl = tc::sw128_desc(st + 3 * kPlane + k * 32);
+                        mma_tf32(d, al, bh, (ks > 0 || k > 0) ? 1u : 0u);
+                        mma_tf32(d, ah, bl, 1u);
+                        mma_tf32(d, ah, bh, 1u);
+                    }
+                    tc::mma_commit(&S->empty[s]);
+                }
+                __syncwarp();
+            }
+            if (ok && lane == 0) tc::mma_commit(&S->tmem_full[acc]);
+            __syncwarp();
+        }
+        if (lane == 0) tc::mma_commit(&S->drain);
+        __syncwarp();
+        int no_abort = 0;
+        mbar_wait(&S->drain, 0, &no_abort, p.status);
+    } else {
+        // ------------------------------------------------------------ epilogue (warps 0-3)
+        int t = 0;
+        bool ok = true;
+        const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+            const int acc = t & 1;
+            const int64_t ct = tile % n_ct;
+            const int64_t n0 = (tile / n_ct) * kM;
+            ok = mbar_wait(&S->tmem_full[acc], (t / 2) & 1, abort, p.status);
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const int64_t n = n0 + warp * 32 + lane;
+            const int64_t co0 = ct * kN;
+#pragma unroll 1
+            for (int c = 0; c < kN / 32; ++c) {
+                uint32_t v[32];
+                tc::tmem_ld32(tmem + lane_off + static_cast<uint32_t>(acc * kN + c * 32), v);
+                if (n < p.N) {
+                    float *y = p.Y + n * p.Cout + co0 + c * 32;
+                    if (co0 + c * 32 + 32 <= p.Cout) {
+#pragma unroll
+                        for (int q = 0; q < 8; ++q)
+                            __stcs(reinterpret_cast<float4 *>(y) + q,
+                                   make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
+                                               __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3])));
+                    } else {
+                        for (int q = 0; q < 32 && co0 + c * 32 + q < p.Cout; ++q) y[q] = __uint_as_float(v[q]);
+                    }
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            mbar_arrive(&S->tmem_empty[acc]);
+        }
+    }
+
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 8) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+    }
+}
+
+// one thread per (group gi, r): the hi and lo planes of the G dense weights of
+// column r (zero except the K kept ones); index sets strictly increasing
+template <int G, int K>
+__global__ void decompress_f32_split_kernel(const float *__restrict__ values, const uint8_t *__restrict__ idx,
+                                            int64_t Cout, int64_t R, float *__restrict__ wh, float *__restrict__ wl,
+                                            uint32_t *status)
+{
+    const int64_t total = (Cout / G) * R;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gi = t / R, r = t - gi * R;
+        uint32_t v[K];
+        int ix[K];
+        bool bad = false;
+#pragma unroll
+        for (int s = 0; s < K; ++s) {
+            v[s] = __float_as_uint(values[t * K + s]);
+            ix[s] = idx[t * K + s];
+            bad |= ix[s] >= G || (s > 0 && ix[s] <= ix[s - 1]);
+        }
+        if (bad) report(status, CCI_ERR_INDEX);
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+            uint32_t o = 0;
+#pragma unroll
+            for (int s = 0; s < K; ++s) o = (ix[s] == j) ? v[s] : o;
+            wh[(gi * G + j) * R + r] = __uint_as_float(hi_bits(o));
+            wl[(gi * G + j) * R + r] = __uint_as_float(lo_bits(o));
+        }
+    }
+}
+
+cudaError_t launch_gemm(const FwdParams &p, cudaStream_t stream)
+{
+    static const cudaError_t attr = cudaFuncSetAttribute(gemm_tf32x3_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                         static_cast<int>(kSmemBytes));
+    if (attr != cudaSuccess) return attr;
+    const int64_t n_ct = (p.Cout + kN - 1) / kN;
+    const int64_t n_tiles = n_ct * ((p.N + kM - 1) / kM);
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t grid = n_tiles < sms ? n_tiles : sms;
+    gemm_tf32x3_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, stream>>>(p, n_ct, n_tiles);
+    return cudaGetLastError();
+}
+
+}  // namespace tf
+
 // one thread per (group gi, r): the G weights W[gi*G + j][r] of the dense
 // matrix, zero except the K kept ones (bf16 copied bit for bit); index sets
 // must be strictly increasing (as cci_pack writes them)
@@ -439,8 +738,29 @@ __global__ void decompress_bf16_kernel(const uint16_t *__restrict__ values, cons
 }
 
 // (G, K) pairs with a dense tensor-core instantiation (G divides the 256-channel tile)
-cudaError_t launch_dense_tc(const FwdParams &p, int G, int K, bool ws, cudaStream_t stream)
+cudaError_t launch_dense_tc(const FwdParams &p, int dtype, int G, int K, bool ws, cudaStream_t stream)
 {
+    if (dtype == CCI_F32) {
+        if (!ws) return cudaErrorNotSupported;
+#define CCI_TF_CASE(g, k)                                                                            \
+    if (G == g && K == k) {                                                                          \
+        const int64_t total = (p.Cout / g) * p.R;                                                    \
+        const int64_t blocks = (total + 255) / 256;                                                  \
+        float *wh = static_cast<float *>(const_cast<void *>(p.wdense));                              \
+        tf::decompress_f32_split_kernel<g, k><<<static_cast<unsigned>(blocks < 65536 * 8 ? blocks : 65536 * 8), 256, \
+                                                0, stream>>>(static_cast<const float *>(p.values), p.idx, p.Cout, p.R, \
+                                                             wh, wh + p.Cout * p.R, p.status);             \
+        const cudaError_t e = cudaGetLastError();                                                    \
+        if (e != cudaSuccess) return e;                                                              \
+        return tf::launch_gemm(p, stream);                                                           \
+    }
+        CCI_TF_CASE(4, 1) CCI_TF_CASE(4, 2)
+        CCI_TF_CASE(8, 1) CCI_TF_CASE(8, 2) CCI_TF_CASE(8, 4)
+        CCI_TF_CASE(16, 1) CCI_TF_CASE(16, 2) CCI_TF_CASE(16, 4) CCI_TF_CASE(16, 8)
+        CCI_TF_CASE(32, 1) CCI_TF_CASE(32, 2) CCI_TF_CASE(32, 4) CCI_TF_CASE(32, 8) CCI_TF_CASE(32, 16)
+#undef CCI_TF_CASE
+        return cudaErrorNotSupported;
+    }
 #define CCI_TC_CASE(g, k)                                                                          \
     if (G == g && K == k) {                                                                        \
         if (!ws) return tc::launch<g, k, false>(p, stream);                                        \
@@ -463,7 +783,7 @@ cudaError_t launch_dense_tc(const FwdParams &p, int G, int K, bool ws, cudaStrea
 
 bool dense_tc_supported(int dtype, int G, int K)
 {
-    if (dtype != CCI_BF16) return false;
+    if (dtype != CCI_BF16 && dtype != CCI_F32) return false;
     const int gs[] = {4, 8, 16, 32};
     for (int g : gs)
         if (g == G) return K >= 1 && K <= G / 2 && (K & (K - 1)) == 0;

@@ -12,9 +12,10 @@ cudaError_t launch_fma_probe(float *out, int blocks, int threads, int iters, cud
 
 // dense tensor-core comparison kernel (tcgen05, bf16 only)
 bool dense_tc_supported(int dtype, int G, int K);
-// ws = true: decompress once into p.wdense (dense bf16 [Cout][R]) and copy B
-// tiles from it; ws = false: decompress each B tile in shared memory
-cudaError_t launch_dense_tc(const FwdParams &p, int G, int K, bool ws, cudaStream_t stream);
+// ws = true: decompress once into p.wdense and copy B tiles from it (bf16: dense
+// [Cout][R]; fp32: hi and lo tf32 planes [2][Cout][R], three-pass tf32 product);
+// ws = false (bf16 only): decompress each B tile in shared memory
+cudaError_t launch_dense_tc(const FwdParams &p, int dtype, int G, int K, bool ws, cudaStream_t stream);
 
 // One register-tiled instantiation: (dtype, G, K) -> tile shape and launcher.
 struct RegtileEntry {

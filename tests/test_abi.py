@@ -140,7 +140,10 @@ def test_workspace_rules(lib):
     ws = cci.ALGO_DENSE_TC_WS
     assert cci.workspace_size(ws, torch.bfloat16, 256, 64) == 256 * 64 * 2
     assert cci.workspace_size(cci.ALGO_EXPAND, torch.bfloat16, 256, 64) == 0
-    assert cci.workspace_size(cci.ALGO_AUTO, torch.float32, 256, 64) == 0
+    assert cci.workspace_size(cci.ALGO_AUTO, torch.float32, 256, 64) == 256 * 64 * 8
+    assert cci.workspace_size(ws, torch.float32, 256, 64) == 256 * 64 * 8
+    assert cci.kernel_name(torch.float32, 64, 64, 256, 8, 2, ws) == "dense_tc_ws_tf32x3_G8_K2"
+    assert cci.kernel_name(torch.float32, 64, 64, 256, 8, 2, cci.ALGO_DENSE_TC) == ""
     assert cci.workspace_size(cci.ALGO_AUTO, torch.bfloat16, 256, 64) == 256 * 64 * 2
     # the family needs a workspace: rejected before any launch (no device needed)
     assert linear(lib, dt=1, algo=ws) == 11

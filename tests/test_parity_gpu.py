@@ -435,3 +435,46 @@ def test_auto_with_workspace_uses_dense_tc_ws(dev):
     Ya = cci.linear(Xd, v, i, Cout, G, K, workspace=ws)
     Yw = cci.linear(Xd, v, i, Cout, G, K, algo=cci.ALGO_DENSE_TC_WS)
     assert torch.equal(Ya.view(torch.int32), Yw.view(torch.int32))
+
+
+# ---------------------------------------------------------------------------
+# fp32 on the tensor cores: three-pass tf32 product through the workspace family
+# ---------------------------------------------------------------------------
+F32_DENSE = [(128, 64, 128, 8, 2), (1, 16, 128, 8, 2), (200, 36, 200, 4, 1), (300, 132, 384, 16, 4),
+             (515, 64, 96, 32, 8), (129, 256, 1024, 8, 2), (77, 12, 64, 16, 8)]
+
+
+@pytest.mark.parametrize("case", F32_DENSE, ids=lambda c: "N{}_C{}x{}_G{}K{}".format(*c))
+def test_tf32x3_small(dev, case):
+    N, Cin, Cout, G, K = case
+    X, W = wl.random_small(N * 5 + Cin, "f32", N, Cin, Cout)
+    assert cci.kernel_name(F32, Cin, Cin, Cout, G, K, cci.ALGO_DENSE_TC_WS).startswith("dense_tc_ws_tf32x3")
+    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC_WS)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, str(case))
+
+
+def test_tf32x3_bottleneck_full(dev):
+    case = wl.BOTTLENECK_1X1
+    X, W = wl.linear_inputs(case)
+    Y = run_linear(dev, X, W, case.G, case.K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    rows = sample_rows(case.N, 2048, seed=3)
+    _, _, Wd, mask = oracle_reference(W, case.G, case.K)
+    Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name + " tf32x3")
+
+
+@pytest.mark.parametrize("case", [c for c in CONV_SMALL if c[-1] == "f32" and c[3] % 4 == 0 and c[9] in (4, 8, 16, 32)
+                                  and (c[10] & (c[10] - 1)) == 0 and c[10] <= c[9] // 2],
+                         ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
+def test_tf32x3_conv_small(dev, case):
+    B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
+    g = torch.Generator().manual_seed(B * 13 + Cin)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0)
+    W = torch.randn((Cout, KH * KW * Cin), generator=g)
+    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
