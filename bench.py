@@ -45,6 +45,23 @@ MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 N_SM, FMA_LANES, SM_MAX_GHZ = 152, 128, 2.070
 ALU_PEAK_TFLOPS = N_SM * FMA_LANES * 2 * SM_MAX_GHZ / 1e3
 L2_FLUSH_BYTES = 256 << 20
+HBM_ROOF_GBS = 8000.0  # the workload's stated memory roof (8 TB/s)
+
+
+def measured_peaks():
+    try:
+        with open(MEASURED_PEAKS) as f:
+            return json.load(f)
+    except (OSError, ValueError):
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+                "source": "fallback"}
+
+
+def tensor_peak(dtype_name: str) -> float:
+    """Dense tensor-core peak for the operand type: the measured bf16 burst figure,
+    times the nominal tf32/bf16 ratio (1.1 / 2.25 PFLOP/s) for tf32."""
+    bf16 = float(measured_peaks()["bf16_tflops"])
+    return bf16 if dtype_name == "bf16" else bf16 * 1.1 / 2.25
 
 
 def parse():
@@ -300,6 +317,13 @@ def run_ours(args, rank, world, local):
     values = torch.empty((case.Cout // case.G, case.R, case.K), dtype=Xd.dtype, device=dev)
     idx = torch.empty((case.Cout // case.G, case.R, case.K), dtype=torch.uint8, device=dev)
     Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
+    # the library's production path: AUTO with a workspace (the dense tensor-core
+    # family when the layer has one, else the CUDA-core family)
+    ws = cci.new_workspace(cci.ALGO_AUTO, Xd.dtype, case.Cout, case.R, dev)
+    kname = cci.kernel_name(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_DENSE_TC_WS)
+    on_tc = bool(kname) and ws is not None
+    if not on_tc:
+        kname = cci.kernel_name(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K)
     status = cci.new_status(dev)
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
 
@@ -308,7 +332,7 @@ def run_ours(args, rank, world, local):
 
     def step():
         cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
-        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status)
+        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status, workspace=ws)
 
     for _ in range(max(3, args.warmup)):
         step()
@@ -328,7 +352,7 @@ def run_ours(args, rank, world, local):
             a.record(stream)
             cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
             b.record(stream)
-            cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status)
+            cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status, workspace=ws)
             c.record(stream)
         torch.cuda.synchronize(dev)
         t_wall = time.perf_counter() - t_wall0
@@ -343,15 +367,35 @@ def run_ours(args, rank, world, local):
     nzf = case.nz_flops()
     value = world * nzf / (ms_step * 1e-3) / 1e12
     lin_avg = statistics.mean(lin_ms)
-    kname = cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K)
     achieved = nzf / (lin_avg * 1e-3) / 1e12
-    roofline = {"bound": "alu", "achieved": achieved, "peak": ALU_PEAK_TFLOPS, "unit": "TFLOP/s",
-                "frac": achieved / ALU_PEAK_TFLOPS, "traffic": measured_traffic(kname),
-                "kernel": kname,
-                "peak_source": "derived: 152 SMs x 128 FP32 FMA lanes x 2 flop x 2.070 GHz max clock",
-                "algorithmic_flops_per_launch": nzf,
-                "hbm_bytes_per_launch": case.N * case.Cin * X.element_size() + case.N * case.Cout * 4
-                + (case.Cout // case.G) * case.R * case.K * (X.element_size() + 1)}
+    alg_bytes = (case.N * case.Cin * X.element_size() + case.N * case.Cout * 4
+                 + (case.Cout // case.G) * case.R * case.K * (X.element_size() + 1))
+    if on_tc:
+        tdt = "bf16" if X.dtype == torch.bfloat16 else "tf32"
+        passes = 1 if tdt == "bf16" else 3
+        peak = tensor_peak(tdt)
+        executed = passes * case.dense_flops()
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                    "frac": achieved / peak, "traffic": measured_traffic(kname), "kernel": kname,
+                    "peak_source": f"measured bf16 burst {measured_peaks()['bf16_tflops']} TFLOP/s"
+                                   + (" x nominal tf32/bf16 ratio 1.1/2.25" if tdt == "tf32" else ""),
+                    "algorithmic_flops_per_launch": nzf,
+                    "tensor_flops_executed_per_launch": executed,
+                    "tensor_utilisation": executed / (lin_avg * 1e-3) / 1e12 / peak,
+                    "note": "linear time includes the one-pass weight decompression launch",
+                    "hbm_bytes_per_launch": alg_bytes}
+    else:
+        roofline = {"bound": "alu", "achieved": achieved, "peak": ALU_PEAK_TFLOPS, "unit": "TFLOP/s",
+                    "frac": achieved / ALU_PEAK_TFLOPS, "traffic": measured_traffic(kname),
+                    "kernel": kname,
+                    "peak_source": "derived: 152 SMs x 128 FP32 FMA lanes x 2 flop x 2.070 GHz max clock",
+                    "algorithmic_flops_per_launch": nzf, "hbm_bytes_per_launch": alg_bytes}
+    # the workload's own roofline: the slower of its nonzero flops at the CUDA-core
+    # FMA peak and its compressed bytes at 8 TB/s
+    floor_s = max(nzf / (ALU_PEAK_TFLOPS * 1e12), alg_bytes / (HBM_ROOF_GBS * 1e9))
+    metric_roofline = {"definition": "max(nonzero flops / CUDA-core FMA peak, compressed bytes / 8 TB/s)",
+                       "floor_us": floor_s * 1e6, "frac": floor_s / (lin_avg * 1e-3),
+                       "fma_peak_tflops": ALU_PEAK_TFLOPS}
 
     # ---- end to end through the public API: host X,W -> device, step, Y -> host ----
     Y_host = torch.empty((case.N, case.Cout), dtype=torch.float32).pin_memory()
@@ -360,7 +404,7 @@ def run_ours(args, rank, world, local):
         Xd.copy_(X_host, non_blocking=True)
         Wd.copy_(W_host, non_blocking=True)
         cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
-        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status)
+        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status, workspace=ws)
         Y_host.copy_(Y, non_blocking=True)
 
     for _ in range(2):
@@ -410,7 +454,8 @@ def run_ours(args, rank, world, local):
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": config_of(case), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": 2 * args.steps, "clocks": clk.summary(),
+            "gpu_launches": (3 if on_tc else 2) * args.steps, "clocks": clk.summary(),
+            "metric_roofline": metric_roofline,
             "breakdown_ms": {"pack": statistics.mean(pack_ms), "linear": lin_avg,
                              "wall_per_step_incl_flush": t_wall * 1e3 / args.steps},
             "dense_reference": dense, "cuda_core_families": families, **extras,
