@@ -72,6 +72,12 @@ struct ColumnSite {
 __device__ __forceinline__ ColumnSite column_site(const FwdParams &p, int64_t n)
 {
     ColumnSite s;
+    if (!p.is_conv) {  // a product: column n is row n of X, no receptive field
+        s.img = n * p.Cin;
+        s.hb = 0;
+        s.wb = 0;
+        return s;
+    }
     const int64_t pq = p.P * p.Q;
     const int64_t b = n / pq;
     const int64_t rem = n - b * pq;

@@ -20,7 +20,7 @@
 // Every mbarrier wait is bounded: on expiry the kernel records CCI_ERR_TIMEOUT,
 // raises a CTA abort flag so the other roles stop, drains its own copies and
 // MMAs, frees TMEM and exits.
-#include "cci_kernels.h"
+#include "cci_tc_common.cuh"
 
 namespace cci {
 namespace tc {
@@ -34,96 +34,8 @@ constexpr int kThreads = 288;
 constexpr int kATile = kM * kKS * 2;   // 16 KB
 constexpr int kBTile = kN * kKS * 2;   // 32 KB
 constexpr int kTmemCols = 512;         // two 256-column fp32 accumulators
-constexpr long long kWaitLimit = 1ll << 31;  // clock cycles (about 1 s) per wait
-
-struct Smem {
-    // stage buffers are placed at a 1024-byte aligned base (swizzle atoms)
-    uint64_t full[kStages];
-    uint64_t empty[kStages];
-    uint64_t tmem_full[2];
-    uint64_t tmem_empty[2];
-    uint64_t drain;
-    uint32_t tmem_base;
-    int abort;
-};
 
 constexpr size_t kSmemBytes = 1024 /*alignment slack*/ + kStages * (kATile + kBTile) + sizeof(Smem) + 64;
-
-__device__ __forceinline__ uint32_t smem_u32(const void *p)
-{
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint64_t *bar)
-{
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-
-// bounded wait for the phase with the given parity; false on timeout or abort
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort, uint32_t *status)
-{
-    const uint32_t a = smem_u32(bar);
-    const long long t0 = clock64();
-    while (true) {
-        uint32_t done;
-        asm volatile(
-            "{\n.reg .pred p;\n"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            "selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(done)
-            : "r"(a), "r"(parity)
-            : "memory");
-        if (done) return true;
-        if (*abort) return false;
-        if (clock64() - t0 > kWaitLimit) {
-            *abort = 1;
-            report(status, CCI_ERR_TIMEOUT);
-            return false;
-        }
-    }
-}
-
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, bool valid)
-{
-    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(valid ? 16 : 0)
-                 : "memory");
-}
-
-__device__ __forceinline__ void st_shared_v4_zero(uint32_t addr)
-{
-    asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(addr), "r"(0) : "memory");
-}
-
-__device__ __forceinline__ void st_shared_b16(uint32_t addr, uint16_t v)
-{
-    asm volatile("st.shared.b16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
-}
-
-// byte offset of (row, k) in a K-major tile of 128-byte rows with the 128-byte
-// swizzle: 16-byte chunk j of row i sits at chunk position j ^ (i % 8)
-__device__ __forceinline__ uint32_t sw128(int row, int k_elem)
-{
-    const int chunk = (k_elem >> 3) ^ (row & 7);
-    return static_cast<uint32_t>(row * 128 + chunk * 16 + (k_elem & 7) * 2);
-}
-
-// tcgen05 shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row
-// atoms of 1024 bytes (stride byte offset 1024), fixed field 0b001 at bit 46
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t addr)
-{
-    uint64_t d = 0;
-    d |= static_cast<uint64_t>((addr & 0x3ffff) >> 4);       // start address
-    d |= static_cast<uint64_t>(1) << 16;                       // leading byte offset (unused)
-    d |= static_cast<uint64_t>(1024 >> 4) << 32;               // stride byte offset
-    d |= static_cast<uint64_t>(1) << 46;                       // fixed 0b001
-    d |= static_cast<uint64_t>(2) << 61;                       // 128-byte swizzle
-    return d;
-}
 
 // instruction descriptor, kind::f16: D f32, A and B bf16, both K-major, M x N
 constexpr uint32_t kIdesc = (1u << 4)                 // D format f32
@@ -139,27 +51,7 @@ __device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64
         : "memory");
 }
 
-__device__ __forceinline__ void mma_commit(uint64_t *bar)
-{
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-                 : "memory");
-}
 
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32])
-{
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
-        "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
-          "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
-          "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
-          "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
-
-// WS = false: the producers decompress the CTA's packed groups into the B tile;
-// WS = true: B is copied (cp.async) from the dense workspace p.wdense [Cout][R]
 template <int G, int K, bool WS>
 __global__ void __launch_bounds__(kThreads, 1) dense_tc_kernel(FwdParams p, int64_t n_ct, int64_t n_tiles)
 {
@@ -456,207 +348,6 @@ __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
     return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
 }
 
-__global__ void __launch_bounds__(kThreads, 1) gemm_tf32x3_kernel(FwdParams p, int64_t n_ct, int64_t n_tiles)
-{
-    using tc::mbar_arrive;
-    using tc::mbar_init;
-    using tc::mbar_wait;
-    using tc::smem_u32;
-    extern __shared__ __align__(16) unsigned char smem_raw[];
-    const uint32_t raw = smem_u32(smem_raw);
-    const uint32_t base = (raw + 1023u) & ~1023u;
-    unsigned char *gbase = smem_raw + (base - raw);
-    tc::Smem *S = reinterpret_cast<tc::Smem *>(gbase + kStages * kStage);
-    volatile int *abort = &S->abort;
-    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int nks = static_cast<int>((p.R + kKS - 1) / kKS);
-    const float *X = static_cast<const float *>(p.X);
-    const float *Wh = static_cast<const float *>(p.wdense);
-    const float *Wl = Wh + p.Cout * p.R;
-
-    if (tid == 0) {
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(&S->full[s], 128);
-            mbar_init(&S->empty[s], 1);
-        }
-        for (int a = 0; a < 2; ++a) {
-            mbar_init(&S->tmem_full[a], 1);
-            mbar_init(&S->tmem_empty[a], 128);
-        }
-        mbar_init(&S->drain, 1);
-        S->abort = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    if (warp == 8) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&S->tmem_base)),
-                     "r"(kTmemCols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
-    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-    const uint32_t tmem = S->tmem_base;
-
-    if (warp >= 4 && warp < 8) {
-        // ------------------------------------------------------------ producers
-        const int pt = tid - 128;
-        const int chunk = pt & 7;  // 16-byte chunk (4 fp32) of every A / B copy of this thread
-        const int rowb = pt >> 3;  // rows rowb + 16 i
-        int it = 0;
-        bool ok = true;
-        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-            const int64_t ct = tile % n_ct;
-            const int64_t n0 = (tile / n_ct) * kM;
-            const int64_t co0 = ct * kN;
-            ColumnSite site[8];
-            bool colok[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                const int64_t n = n0 + rowb + 16 * i;
-                colok[i] = n < p.N;
-                site[i] = colok[i] ? column_site(p, n) : ColumnSite{0, 0, 0};
-            }
-            for (int ks = 0; ks < nks && ok; ++ks, ++it) {
-                const int s = it % kStages;
-                // the activation chunks of this stage, read before the buffer is free
-                const int64_t r = static_cast<int64_t>(ks) * kKS + chunk * 4;
-                const bool rok = r < p.R;
-                int kh = 0, kw = 0;
-                int64_t ci = r;
-                if (p.is_conv && rok) {
-                    const int tap = static_cast<int>(r / p.Cin);
-                    ci = r - static_cast<int64_t>(tap) * p.Cin;
-                    kh = tap / p.KW;
-                    kw = tap - kh * p.KW;
-                }
-                uint4 xa[8];
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    xa[i] = make_uint4(0, 0, 0, 0);
-                    bool valid = colok[i] && rok;
-                    int64_t off = site[i].img + r;
-                    if (valid && p.is_conv) {
-                        const int h = site[i].hb + kh, w = site[i].wb + kw;
-                        valid = h >= 0 && h < p.H && w >= 0 && w < p.W;
-                        off = site[i].img + (static_cast<int64_t>(h) * p.W + w) * p.Cin + ci;
-                    }
-                    if (valid) xa[i] = __ldg(reinterpret_cast<const uint4 *>(X + off));
-                }
-                if (it >= kStages) ok = mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
-                if (!ok) break;
-                const uint32_t st = base + s * kStage;
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int row = rowb + 16 * i;
-                    const uint32_t o = sw128f(row, chunk * 4);
-                    st_shared_v4(st + o, hi_bits(xa[i].x), hi_bits(xa[i].y), hi_bits(xa[i].z), hi_bits(xa[i].w));
-                    st_shared_v4(st + kPlane + o, lo_bits(xa[i].x), lo_bits(xa[i].y), lo_bits(xa[i].z),
-                                 lo_bits(xa[i].w));
-                }
-                // B planes: 128 rows x 8 chunks each, from the workspace
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int row = rowb + 16 * i;
-                    const bool valid = co0 + row < p.Cout && rok;
-                    const int64_t g = (co0 + row) * p.R + r;
-                    const uint32_t o = sw128f(row, chunk * 4);
-                    tc::cp_async16(st + 2 * kPlane + o, valid ? Wh + g : Wh, valid);
-                    tc::cp_async16(st + 3 * kPlane + o, valid ? Wl + g : Wl, valid);
-                }
-                asm volatile("cp.async.commit_group;" ::: "memory");
-                if (it >= kLag) {
-                    asm volatile("cp.async.wait_group %0;" ::"n"(kLag) : "memory");
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                    mbar_arrive(&S->full[(it - kLag) % kStages]);
-                }
-            }
-        }
-        asm volatile("cp.async.wait_group 0;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        for (int q = (it >= kLag ? it - kLag : 0); q < it; ++q) mbar_arrive(&S->full[q % kStages]);
-    } else if (warp == 8) {
-        // ------------------------------------------------------------ MMA issuer
-        int it = 0, t = 0;
-        bool ok = true;
-        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
-            const int acc = t & 1;
-            if (t >= 2) ok = mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
-            if (!ok) break;
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
-            for (int ks = 0; ks < nks && ok; ++ks, ++it) {
-                const int s = it % kStages;
-                ok = mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
-                if (!ok) break;
-                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                if (lane == 0) {
-                    const uint32_t st = base + s * kStage;
-#pragma unroll
-                    for (int k = 0; k < kKS / 8; ++k) {
-                        const uint64_t ah = tc::sw128_desc(st + k * 32);
-                        const uint64_t al = tc::sw128_desc(st + kPlane + k * 32);
-                        const uint64_t bh = tc::sw128_desc(st + 2 * kPlane + k * 32);
-                        const uint64_t bl = tc::sw128_desc(st + 3 * kPlane + k * 32);
-                        mma_tf32(d, al, bh, (ks > 0 || k > 0) ? 1u : 0u);
-                        mma_tf32(d, ah, bl, 1u);
-                        mma_tf32(d, ah, bh, 1u);
-                    }
-                    tc::mma_commit(&S->empty[s]);
-                }
-                __syncwarp();
-            }
-            if (ok && lane == 0) tc::mma_commit(&S->tmem_full[acc]);
-            __syncwarp();
-        }
-        if (lane == 0) tc::mma_commit(&S->drain);
-        __syncwarp();
-        int no_abort = 0;
-        mbar_wait(&S->drain, 0, &no_abort, p.status);
-    } else {
-        // ------------------------------------------------------------ epilogue (warps 0-3)
-        int t = 0;
-        bool ok = true;
-        const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
-        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
-            const int acc = t & 1;
-            const int64_t ct = tile % n_ct;
-            const int64_t n0 = (tile / n_ct) * kM;
-            ok = mbar_wait(&S->tmem_full[acc], (t / 2) & 1, abort, p.status);
-            if (!ok) break;
-            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-            const int64_t n = n0 + warp * 32 + lane;
-            const int64_t co0 = ct * kN;
-#pragma unroll 1
-            for (int c = 0; c < kN / 32; ++c) {
-                uint32_t v[32];
-                tc::tmem_ld32(tmem + lane_off + static_cast<uint32_t>(acc * kN + c * 32), v);
-                if (n < p.N) {
-                    float *y = p.Y + n * p.Cout + co0 + c * 32;
-                    if (co0 + c * 32 + 32 <= p.Cout) {
-#pragma unroll
-                        for (int q = 0; q < 8; ++q)
-                            __stcs(reinterpret_cast<float4 *>(y) + q,
-                                   make_float4(__uint_as_float(v[4 * q]), __uint_as_float(v[4 * q + 1]),
-                                               __uint_as_float(v[4 * q + 2]), __uint_as_float(v[4 * q + 3])));
-                    } else {
-                        for (int q = 0; q < 32 && co0 + c * 32 + q < p.Cout; ++q) y[q] = __uint_as_float(v[q]);
-                    }
-                }
-            }
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            mbar_arrive(&S->tmem_empty[acc]);
-        }
-    }
-
-    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    __syncthreads();
-    if (warp == 8) {
-        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
-    }
-}
-
 // one thread per (group gi, r): the hi and lo planes of the G dense weights of
 // column r (zero except the K kept ones); index sets strictly increasing
 template <int G, int K>
@@ -687,21 +378,6 @@ __global__ void decompress_f32_split_kernel(const float *__restrict__ values, co
             wl[(gi * G + j) * R + r] = __uint_as_float(lo_bits(o));
         }
     }
-}
-
-cudaError_t launch_gemm(const FwdParams &p, cudaStream_t stream)
-{
-    static const cudaError_t attr = cudaFuncSetAttribute(gemm_tf32x3_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                         static_cast<int>(kSmemBytes));
-    if (attr != cudaSuccess) return attr;
-    const int64_t n_ct = (p.Cout + kN - 1) / kN;
-    const int64_t n_tiles = n_ct * ((p.N + kM - 1) / kM);
-    int dev = 0, sms = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int64_t grid = n_tiles < sms ? n_tiles : sms;
-    gemm_tf32x3_kernel<<<static_cast<unsigned>(grid), kThreads, kSmemBytes, stream>>>(p, n_ct, n_tiles);
-    return cudaGetLastError();
 }
 
 }  // namespace tf
@@ -752,7 +428,7 @@ cudaError_t launch_dense_tc(const FwdParams &p, int dtype, int G, int K, bool ws
                                                              wh, wh + p.Cout * p.R, p.status);             \
         const cudaError_t e = cudaGetLastError();                                                    \
         if (e != cudaSuccess) return e;                                                              \
-        return tf::launch_gemm(p, stream);                                                           \
+        return launch_gemm_ws(p, CCI_F32, stream);                                                   \
     }
         CCI_TF_CASE(4, 1) CCI_TF_CASE(4, 2)
         CCI_TF_CASE(8, 1) CCI_TF_CASE(8, 2) CCI_TF_CASE(8, 4)
@@ -771,7 +447,7 @@ cudaError_t launch_dense_tc(const FwdParams &p, int dtype, int G, int K, bool ws
                                                  static_cast<uint16_t *>(const_cast<void *>(p.wdense)), p.status); \
         const cudaError_t e = cudaGetLastError();                                                  \
         if (e != cudaSuccess) return e;                                                            \
-        return tc::launch<g, k, true>(p, stream);                                                  \
+        return launch_gemm_ws(p, CCI_BF16, stream);                                                \
     }
     CCI_TC_CASE(4, 1) CCI_TC_CASE(4, 2)
     CCI_TC_CASE(8, 1) CCI_TC_CASE(8, 2) CCI_TC_CASE(8, 4)
