@@ -24,7 +24,7 @@
 namespace cci {
 namespace ws {
 
-enum Mode { kBf16Tma = 0, kBf16Gather = 1, kTf32x3 = 2 };
+enum Mode { kBf16Tma = 0, kBf16Gather = 1, kTf32x3 = 2, kTf32x3Tma = 3 };
 
 template <int MODE>
 struct Cfg;
@@ -39,7 +39,12 @@ struct Cfg<kBf16Gather> {
     static constexpr bool kATma = false, kTf32 = false;
 };
 template <>
-struct Cfg<kTf32x3> {
+struct Cfg<kTf32x3> {  // convolutions: activations gathered through registers
+    static constexpr int kM = 128, kN = 128, kKS = 32, kStages = 3, kAPlanes = 2, kBPlanes = 2;
+    static constexpr bool kATma = false, kTf32 = true;
+};
+template <>
+struct Cfg<kTf32x3Tma> {  // products: the raw activation tile by TMA, split in shared memory
     static constexpr int kM = 128, kN = 128, kKS = 32, kStages = 3, kAPlanes = 2, kBPlanes = 2;
     static constexpr bool kATma = false, kTf32 = true;
 };
@@ -115,6 +120,7 @@ __global__ void __launch_bounds__(288, 1)
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(&S->full[s], C::kATma ? 1 : 129);
             tc::mbar_init(&S->empty[s], 1);
+            tc::mbar_init(&S->aux[s], 1);
         }
         for (int a = 0; a < 2; ++a) {
             tc::mbar_init(&S->tmem_full[a], 1);
@@ -132,7 +138,7 @@ __global__ void __launch_bounds__(288, 1)
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
     if (tid == 128) {
-        if constexpr (C::kATma) tc::tma_prefetch_desc(&tmA);
+        if constexpr (C::kATma || MODE == kTf32x3Tma) tc::tma_prefetch_desc(&tmA);
         tc::tma_prefetch_desc(&tmB0);
         if constexpr (C::kBPlanes > 1) tc::tma_prefetch_desc(&tmB1);
     }
@@ -197,7 +203,7 @@ __global__ void __launch_bounds__(288, 1)
         };
         int64_t t1 = blockIdx.x, t2 = blockIdx.x;
         int k1 = 0, k2 = 0;
-        if constexpr (C::kTf32) {
+        if constexpr (MODE == kTf32x3) {
             load_x(xa, t1, k1);
             advance(t2, k2);
             load_x(xb, t2, k2);
@@ -219,12 +225,16 @@ __global__ void __launch_bounds__(288, 1)
             }
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
                 const int s = it % kStages;
-                if constexpr (C::kTf32) load_x(xc, t2, k2);  // two stages ahead
+                if constexpr (MODE == kTf32x3) load_x(xc, t2, k2);  // two stages ahead
                 if (it >= kStages) ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
                 if (!ok) break;
                 const uint32_t st = base + s * GE::kStage;
                 const uint32_t bst = st + C::kAPlanes * GE::kAPlane;
                 if (pt == 0) {
+                    if constexpr (MODE == kTf32x3Tma) {
+                        tc::mbar_arrive_expect_tx(&S->aux[s], GE::kAPlane);
+                        tc::tma_load_2d(st, &tmA, ks * kKS, static_cast<int>(n0), &S->aux[s]);
+                    }
                     tc::mbar_arrive_expect_tx(&S->full[s], GE::kTxBytes);
                     tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
                     if constexpr (C::kBPlanes > 1)
@@ -264,6 +274,23 @@ __global__ void __launch_bounds__(288, 1)
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                         tc::mbar_arrive(&S->full[(it - kLag) % kStages]);
                     }
+                } else if constexpr (MODE == kTf32x3Tma) {
+                    // the raw fp32 tile landed in the hi plane: split it in place
+                    ok = tc::mbar_wait(&S->aux[s], (it / kStages) & 1, abort, p.status);
+                    if (!ok) break;
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const uint32_t o = sw_chunk(rowb + 16 * i, chunk);
+                        uint4 v;
+                        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                                     : "r"(st + o)
+                                     : "memory");
+                        st_shared_v4(st + o, hi_bits(v.x), hi_bits(v.y), hi_bits(v.z), hi_bits(v.w));
+                        st_shared_v4(st + GE::kAPlane + o, lo_bits(v.x), lo_bits(v.y), lo_bits(v.z), lo_bits(v.w));
+                    }
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    tc::mbar_arrive(&S->full[s]);
                 } else if constexpr (C::kTf32) {
 #pragma unroll
                     for (int i = 0; i < 8; ++i) {
@@ -423,7 +450,8 @@ cudaError_t launch_mode(const FwdParams &p, cudaStream_t stream)
     CUtensorMap tmA{}, tmB0{}, tmB1{};
     const CUtensorMapDataType dt = C::kTf32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     const int elem = C::kTf32 ? 4 : 2;
-    if (C::kATma && !make_map(&tmA, p.X, dt, elem, p.Cin, p.N, C::kKS, C::kM)) return cudaErrorInvalidValue;
+    if ((C::kATma || MODE == kTf32x3Tma) && !make_map(&tmA, p.X, dt, elem, p.Cin, p.N, C::kKS, C::kM))
+        return cudaErrorInvalidValue;
     if (!make_map(&tmB0, p.wdense, dt, elem, p.R, p.Cout, C::kKS, C::kN)) return cudaErrorInvalidValue;
     if (C::kBPlanes > 1) {
         const char *lo = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
@@ -443,7 +471,8 @@ cudaError_t launch_mode(const FwdParams &p, cudaStream_t stream)
 
 cudaError_t launch_gemm_ws(const FwdParams &p, int dtype, cudaStream_t stream)
 {
-    if (dtype == CCI_F32) return ws::launch_mode<ws::kTf32x3>(p, stream);
+    if (dtype == CCI_F32) return p.is_conv ? ws::launch_mode<ws::kTf32x3>(p, stream)
+                                           : ws::launch_mode<ws::kTf32x3Tma>(p, stream);
     if (!p.is_conv) return ws::launch_mode<ws::kBf16Tma>(p, stream);
     return ws::launch_mode<ws::kBf16Gather>(p, stream);
 }

@@ -14,6 +14,7 @@ constexpr long long kWaitLimit = 1ll << 31;  // clock cycles (about 1 s) per bou
 struct Smem {
     uint64_t full[4];
     uint64_t empty[4];
+    uint64_t aux[4];  // per-stage barrier of a second copy (tf32x3: raw activation tile landed)
     uint64_t tmem_full[2];
     uint64_t tmem_empty[2];
     uint64_t drain;
