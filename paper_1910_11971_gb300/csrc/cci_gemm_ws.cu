@@ -13,9 +13,11 @@
 //   activations TMA over X[N][Cin] for bf16 products; otherwise the producer warps
 //          gather them (cp.async for bf16 convolutions; registers, two stages
 //          ahead, then the hi/lo split, for tf32x3).
-// Roles: warps 0-3 epilogue (TMEM lanes), warps 4-7 producers (producer thread 0
-// issues the TMA copies), warp 8 allocates TMEM and issues the MMAs.  Every
-// mbarrier wait is bounded (CCI_ERR_TIMEOUT, abort flag, drain, TMEM freed).
+// Roles: warps 0-3 epilogue (TMEM lanes), warps 4-7 producers of the activation
+// planes that are not copied by TMA, warp 8 allocates TMEM and issues the MMAs,
+// warp 9 issues the TMA copies as soon as a stage is free (so copy latency
+// overlaps the producers' work).  Every mbarrier wait is bounded
+// (CCI_ERR_TIMEOUT, abort flag, drain, TMEM freed).
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -99,8 +101,10 @@ __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
     return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
 }
 
+constexpr int kThreads = 320;
+
 template <int MODE>
-__global__ void __launch_bounds__(288, 1)
+__global__ void __launch_bounds__(kThreads, 1)
     gemm_ws_kernel(FwdParams p, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, int64_t n_ct, int64_t n_tiles)
 {
@@ -137,7 +141,7 @@ __global__ void __launch_bounds__(288, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
-    if (tid == 128) {
+    if (tid == 288) {
         if constexpr (C::kATma || MODE == kTf32x3Tma) tc::tma_prefetch_desc(&tmA);
         tc::tma_prefetch_desc(&tmB0);
         if constexpr (C::kBPlanes > 1) tc::tma_prefetch_desc(&tmB1);
@@ -147,7 +151,34 @@ __global__ void __launch_bounds__(288, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = S->tmem_base;
 
-    if (warp >= 4 && warp < 8) {
+    if (warp == 9) {
+        // ------------------------------------------------------------ TMA issuer
+        int it = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            const int64_t n0 = (tile / n_ct) * kM;
+            const int64_t co0 = (tile % n_ct) * kN;
+            for (int ks = 0; ks < nks && ok; ++ks, ++it) {
+                const int s = it % kStages;
+                if (it >= kStages) ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
+                if (!ok) break;
+                if (lane == 0) {
+                    const uint32_t st = base + s * GE::kStage;
+                    const uint32_t bst = st + C::kAPlanes * GE::kAPlane;
+                    if constexpr (MODE == kTf32x3Tma) {
+                        tc::mbar_arrive_expect_tx(&S->aux[s], GE::kAPlane);
+                        tc::tma_load_2d(st, &tmA, ks * kKS, static_cast<int>(n0), &S->aux[s]);
+                    }
+                    tc::mbar_arrive_expect_tx(&S->full[s], GE::kTxBytes);
+                    tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                    if constexpr (C::kBPlanes > 1)
+                        tc::tma_load_2d(bst + GE::kBPlane, &tmB1, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                    if constexpr (C::kATma) tc::tma_load_2d(st, &tmA, ks * kKS, static_cast<int>(n0), &S->full[s]);
+                }
+                __syncwarp();
+            }
+        }
+    } else if (warp >= 4 && warp < 8) {
         // ------------------------------------------------------------ producers
         const int pt = tid - 128;
         const int chunk = pt & 7;  // 16-byte chunk of every activation row this thread gathers
@@ -226,21 +257,13 @@ __global__ void __launch_bounds__(288, 1)
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
                 const int s = it % kStages;
                 if constexpr (MODE == kTf32x3) load_x(xc, t2, k2);  // two stages ahead
-                if (it >= kStages) ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
+                // gather / register modes write the stage themselves: wait until it is
+                // free; the split mode waits for its raw tile (copied after the stage
+                // was freed) instead
+                if (MODE != kTf32x3Tma && it >= kStages)
+                    ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
                 if (!ok) break;
                 const uint32_t st = base + s * GE::kStage;
-                const uint32_t bst = st + C::kAPlanes * GE::kAPlane;
-                if (pt == 0) {
-                    if constexpr (MODE == kTf32x3Tma) {
-                        tc::mbar_arrive_expect_tx(&S->aux[s], GE::kAPlane);
-                        tc::tma_load_2d(st, &tmA, ks * kKS, static_cast<int>(n0), &S->aux[s]);
-                    }
-                    tc::mbar_arrive_expect_tx(&S->full[s], GE::kTxBytes);
-                    tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
-                    if constexpr (C::kBPlanes > 1)
-                        tc::tma_load_2d(bst + GE::kBPlane, &tmB1, ks * kKS, static_cast<int>(co0), &S->full[s]);
-                    if constexpr (C::kATma) tc::tma_load_2d(st, &tmA, ks * kKS, static_cast<int>(n0), &S->full[s]);
-                }
                 if constexpr (MODE == kBf16Gather) {
                     const uint16_t *X = static_cast<const uint16_t *>(p.X);
                     const int64_t r = static_cast<int64_t>(ks) * kKS + chunk * 8;
@@ -463,7 +486,7 @@ cudaError_t launch_mode(const FwdParams &p, cudaStream_t stream)
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int64_t grid = n_tiles < sms ? n_tiles : sms;
-    kern<<<static_cast<unsigned>(grid), 288, GE::kSmem, stream>>>(p, tmA, tmB0, tmB1, n_ct, n_tiles);
+    kern<<<static_cast<unsigned>(grid), kThreads, GE::kSmem, stream>>>(p, tmA, tmB0, tmB1, n_ct, n_tiles);
     return cudaGetLastError();
 }
 
