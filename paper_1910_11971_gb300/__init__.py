@@ -176,11 +176,12 @@ def linear(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
     """Y[N][Cout] (fp32) = the CCI-sparse product of X[N][Cin] (Alg. 2).
 
     ``workspace``: device buffer for the families that need one (see
-    ``workspace_size``); with ``algo=ALGO_DENSE_TC_WS`` and none given, one is
-    allocated here (PyTorch memory, not by the library)."""
+    ``workspace_size``); with ``algo`` AUTO or ``ALGO_DENSE_TC_WS`` and none given,
+    one is allocated here from PyTorch memory (the library allocates nothing), so
+    AUTO can use the dense tensor-core family."""
     _cuda_contig(X, "X")
     N, Cin = X.shape
-    if workspace is None and algo == ALGO_DENSE_TC_WS:
+    if workspace is None and algo in (ALGO_AUTO, ALGO_DENSE_TC_WS):
         workspace = new_workspace(algo, X.dtype, Cout, Cin, X.device)
     Y = out if out is not None else torch.empty((N, Cout), dtype=torch.float32, device=X.device)
     wp, wb = _ws(workspace)
@@ -206,7 +207,7 @@ def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
     P, Q = conv_out_hw(H, W, KH, KW, stride, pad)
     Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=torch.float32,
                                                 device=X.device)
-    if workspace is None and algo == ALGO_DENSE_TC_WS:
+    if workspace is None and algo in (ALGO_AUTO, ALGO_DENSE_TC_WS):
         workspace = new_workspace(algo, X.dtype, Cout, KH * KW * Cin, X.device)
     wp, wb = _ws(workspace)
     code = lib().cci_conv2d_ws(X.data_ptr(), _dtype_code(X), B, H, W, Cin, values.data_ptr(),
