@@ -114,43 +114,100 @@ def max_over_ranks(x: float, world: int, device) -> float:
 # clocks during the timed region
 # ---------------------------------------------------------------------------
 class ClockSampler:
+    """SM clock and clock-event reasons during the timed region.
+
+    Reads NVML through ctypes (read-only queries: clocks and event reasons),
+    polling about every millisecond so that a timed region of a few ms still has
+    samples; falls back to `nvidia-smi -lms 200` when NVML cannot be loaded."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
-        self.gpu = gpu_index
+    def __init__(self, device: torch.device):
+        self.device = device
+        self.samples = []  # (sm_mhz, max_mhz, reasons bitmask)
+        self.smi_lines = []
         self.proc = None
-        self.lines = []
+        self.nvml = None
+        self.stop = threading.Event()
+        try:
+            import ctypes
+            lib = ctypes.CDLL("libnvidia-ml.so.1")
+            if lib.nvmlInit_v2() != 0:
+                raise OSError("nvmlInit failed")
+            h = ctypes.c_void_p()
+            uuid = "GPU-" + str(torch.cuda.get_device_properties(device).uuid)
+            if lib.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) != 0:
+                raise OSError("device handle")
+            self.nvml, self.handle, self.ct = lib, h, ctypes
+        except (OSError, AttributeError, RuntimeError):
+            self.nvml = None
+
+    def _poll_nvml(self):
+        ct, lib = self.ct, self.nvml
+        cur, mx, rs = ct.c_uint(), ct.c_uint(), ct.c_ulonglong()
+        get_reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self.stop.is_set():
+            if (lib.nvmlDeviceGetClockInfo(self.handle, 1, ct.byref(cur)) == 0
+                    and lib.nvmlDeviceGetMaxClockInfo(self.handle, 1, ct.byref(mx)) == 0):
+                r = rs.value if get_reasons(self.handle, ct.byref(rs)) == 0 else 0
+                self.samples.append((float(cur.value), float(mx.value), int(r)))
+            time.sleep(0.001)
+
+    def _read_smi(self):
+        for line in self.proc.stdout:
+            self.smi_lines.append(line.strip())
 
     def __enter__(self):
-        try:
-            self.proc = subprocess.Popen(
-                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
-                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.thread = threading.Thread(target=self._read, daemon=True)
+        if self.nvml is not None:
+            self.thread = threading.Thread(target=self._poll_nvml, daemon=True)
             self.thread.start()
-        except (OSError, FileNotFoundError):
-            self.proc = None
+            t0 = time.time()
+            while not self.samples and time.time() - t0 < 1.0:
+                time.sleep(0.001)
+            self.samples.clear()  # keep only the samples taken in the timed region
+        else:
+            try:
+                self.proc = subprocess.Popen(
+                    ["nvidia-smi", f"--id={self.device.index or 0}", f"--query-gpu={self.FIELDS}",
+                     "--format=csv,noheader,nounits", "-lms", "200"],
+                    stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                self.thread = threading.Thread(target=self._read_smi, daemon=True)
+                self.thread.start()
+            except (OSError, FileNotFoundError):
+                self.proc = None
         return self
 
-    def _read(self):
-        for line in self.proc.stdout:
-            self.lines.append(line.strip())
-
     def __exit__(self, *exc):
+        self.stop.set()
         if self.proc is not None:
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
+        elif self.nvml is not None:
+            self.thread.join(timeout=1.0)
 
     def summary(self):
+        if self.nvml is not None:
+            if not self.samples:
+                return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "source": "nvml"}
+            reasons = set()
+            for _, _, r in self.samples:
+                for bit, name in self.REASONS.items():
+                    if r & bit:
+                        reasons.add(name)
+            return {"sm_mhz": statistics.median(s[0] for s in self.samples),
+                    "sm_max_mhz": max(s[1] for s in self.samples), "reasons": sorted(reasons),
+                    "samples": len(self.samples), "source": "nvml"}
         sm, smax, reasons = [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for ln in self.lines:
+        for ln in self.smi_lines:
             parts = [p.strip() for p in ln.split(",")]
             if len(parts) < 9:
                 continue
@@ -163,9 +220,9 @@ class ClockSampler:
                 if val.lower() == "active":
                     reasons.add(name)
         if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "source": "nvidia-smi"}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "source": "nvidia-smi"}
 
 
 # ---------------------------------------------------------------------------
@@ -344,7 +401,7 @@ def run_ours(args, rank, world, local):
            torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     barrier(world)
     torch.cuda.synchronize(dev)
-    with ClockSampler(local) as clk:
+    with ClockSampler(dev) as clk:
         t_wall0 = time.perf_counter()
         for k in range(args.steps):
             flush()
