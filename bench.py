@@ -320,7 +320,7 @@ def kernel_source_hash() -> str:
 def measured_traffic(kernel: str):
     """DRAM bytes per launch from the committed ncu summary, if it was taken on
     the current kernel sources (else None)."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
     try:
         with open(path) as f:
             rec = json.load(f)
