@@ -556,8 +556,6 @@ def run_extras(cci, dev, stream, flush):
                                   "dense_tc_ms": ms_tc,
                                   "dense_tc_nz_tflops": case.nz_flops() / (ms_tc * 1e-3) / 1e12,
                                   "dense_tc_dense_equiv_tflops": case.dense_flops() / (ms_tc * 1e-3) / 1e12,
-                         "dense_tc_ws_ms": ms_ws, "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
-                         "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
                                   "dense_tc_ws_ms": ms_ws,
                                   "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
                                   "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
@@ -594,7 +592,81 @@ def run_extras(cci, dev, stream, flush):
                          "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
                          "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R, case.Cout,
                                                    case.G, case.K)}
+    out["resnet50_stack"] = run_resnet_stack(cci, dev, stream, flush)
     return out
+
+
+def layer_floor_us(c) -> float:
+    """The workload roofline of one layer: the slower of its nonzero flops at the
+    CUDA-core FMA peak and its compressed bytes (X, Y, values + idx) at 8 TB/s."""
+    es = 2 if c.dtype == "bf16" else 4
+    nbytes = c.B * c.H * c.W * c.Cin * es + c.N * c.Cout * 4 + (c.Cout // c.G) * c.R * c.K * (es + 1)
+    return max(c.nz_flops() / (ALU_PEAK_TFLOPS * 1e12), nbytes / (HBM_ROOF_GBS * 1e9)) * 1e6
+
+
+def run_resnet_stack(cci, dev, stream, flush, reps=5):
+    """The 52 convolutions of ResNet-50 after the stem, batch 128, bf16 inputs,
+    G = 8, K in {1, 2, 4}: every layer once, in network order, each on its own
+    synthetic input (the library's layers take bf16 activations and write fp32,
+    so layer outputs are not chained).  Both sequences are captured in CUDA
+    graphs (launch overhead out of the measurement) and replayed after an L2
+    flush; the dense line is cuDNN on the masked dense bf16 weights (bf16 output)."""
+    res = []
+    for K in (1, 2, 4):
+        layers = wl.resnet50_layers(K=K)
+        ours_calls, dense_calls = [], []
+        keep = []
+        for c in layers:
+            X, W = wl.conv_inputs(c, device=str(dev))
+            v, i = cci.pack(W, c.G, c.K)
+            Y = torch.empty((c.B, c.P, c.Q, c.Cout), dtype=torch.float32, device=dev)
+            ws = cci.new_workspace(cci.ALGO_AUTO, X.dtype, c.Cout, c.R, dev)
+            Wm = torch.zeros((c.Cout, c.R), dtype=W.dtype, device=dev)
+            Wm.view(c.Cout // c.G, c.G, c.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
+            w4 = Wm.view(c.Cout, c.KH, c.KW, c.Cin).permute(0, 3, 1, 2).contiguous(
+                memory_format=torch.channels_last)
+            x4 = X.permute(0, 3, 1, 2)
+            del W, Wm
+            keep.append((X, v, i, Y, ws, w4, x4))
+            ours_calls.append(lambda c=c, X=X, v=v, i=i, Y=Y, ws=ws: cci.conv2d(
+                X, v, i, c.Cout, c.G, c.K, c.KH, c.KW, (c.stride, c.stride), (c.pad, c.pad), out=Y,
+                workspace=ws))
+            dense_calls.append(lambda c=c, x4=x4, w4=w4: torch.nn.functional.conv2d(
+                x4, w4, stride=c.stride, padding=c.pad))
+
+        def ours():
+            for f in ours_calls:
+                f()
+
+        def dense():
+            for f in dense_calls:
+                f()
+
+        ours()
+        dense()
+        torch.cuda.synchronize(dev)
+        g_ours, g_dense = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g_ours):
+            ours()
+        with torch.cuda.graph(g_dense):
+            dense()
+        g_ours.replay()
+        g_dense.replay()
+        torch.cuda.synchronize(dev)
+        ms = statistics.median(time_device(g_ours.replay, reps, flush, stream))
+        dms = statistics.median(time_device(g_dense.replay, reps, flush, stream))
+        nzf = sum(c.nz_flops() for c in layers)
+        dense_f = sum(c.dense_flops() for c in layers)
+        floor_ms = sum(layer_floor_us(c) for c in layers) * 1e-3
+        res.append({"G": 8, "K": K, "layers": len(layers), "batch": layers[0].B, "ms": ms,
+                    "nz_gflop": nzf / 1e9, "nz_tflops": nzf / (ms * 1e-3) / 1e12,
+                    "dense_equiv_tflops": dense_f / (ms * 1e-3) / 1e12,
+                    "roofline_floor_ms": floor_ms, "roofline_frac": floor_ms / ms,
+                    "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
+                    "captured": "CUDA graph of the 52 calls (ours) / 52 cuDNN convolutions (dense)"})
+        del keep, ours_calls, dense_calls, g_ours, g_dense
+        torch.cuda.empty_cache()
+    return res
 
 
 def main():

@@ -90,12 +90,15 @@ cci_status forward(FwdParams p, int dtype, int G, int K, cci_algo algo, void *ws
                    cudaStream_t stream)
 {
     if (p.N == 0) return CCI_OK;
-    if (algo == CCI_ALGO_AUTO && dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) && ws &&
+    // a 1x1 convolution with unit stride and no padding is the product of X[B*H*W][Cin]
+    if (p.is_conv && p.KH == 1 && p.KW == 1 && p.sh == 1 && p.sw == 1 && p.ph == 0 && p.pw == 0) p.is_conv = 0;
+    const bool tc_fits = p.R < (int64_t(1) << 31) && p.Cout < (int64_t(1) << 31);  // 32-bit copy coordinates
+    if (algo == CCI_ALGO_AUTO && tc_fits && dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) && ws &&
         ws_bytes >= dense_ws_bytes(dtype, p.Cout, p.R) && aligned(ws, 16) && aligned(p.X, 16) && aligned(p.Y, 16))
         algo = CCI_ALGO_DENSE_TC_WS;
     if (algo == CCI_ALGO_DENSE_TC || algo == CCI_ALGO_DENSE_TC_WS) {
         const bool use_ws = algo == CCI_ALGO_DENSE_TC_WS;
-        if (!dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) || !aligned(p.X, 16) || !aligned(p.Y, 16))
+        if (!tc_fits || !dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) || !aligned(p.X, 16) || !aligned(p.Y, 16))
             return CCI_ERR_UNSUPPORTED;
         if (!use_ws && dtype != CCI_BF16) return CCI_ERR_UNSUPPORTED;  // shared-memory decompression: bf16 only
         if (use_ws) {

@@ -1,5 +1,7 @@
 // cci_dense_tc.cu -- comparison kernel: decompress the packed weights to dense
-// bf16 tiles in shared memory and multiply them on the tensor cores (tcgen05).
+// bf16 tiles in shared memory and multiply them on the tensor cores (tcgen05);
+// and the one-pass decompression into the workspace of CCI_ALGO_DENSE_TC_WS
+// (namespace dc) that precedes the workspace GEMM.
 //
 // The product of Alg. 2 equals the dense product with the pruned weights zero
 // (Sec. 3.1); this kernel computes it densely, paying G/K times the useful
@@ -300,47 +302,20 @@ cudaError_t launch(const FwdParams &p, cudaStream_t stream)
 }  // namespace tc
 
 // ===========================================================================
-// fp32 layers: three-pass tf32 product.  Every fp32 operand x is split as
-// x = hi + lo with hi = x with the low 13 mantissa bits cleared (exactly a
-// tf32 value) and lo = x - hi (exact in fp32); the product uses
-// hi*hi + hi*lo + lo*hi.  The dropped lo*lo term and the tf32 conversion of lo
-// are each below 2^-22 of |x||w|, whether the tensor core truncates or rounds.
-// Tile D[128 n][128 co], 32 fp32 (128 bytes) of r per stage, 3 stages; A planes
-// written by the producers from registers, B planes copied from the workspace
-// [2][Cout][R] (hi plane, then lo plane).
+// One-pass decompression of the packed weights into the workspace of
+// CCI_ALGO_DENSE_TC_WS: the dense W[Cout][R] (bf16, bit for bit), or for fp32
+// layers its hi and lo tf32 planes [2][Cout][R] (hi = w with the low 13 mantissa
+// bits cleared, exactly a tf32 value; lo = w - hi, exact in fp32) for the
+// three-pass product hi*hi + hi*lo + lo*hi.
+// One block per (group gi, slab of kSlab columns r): each thread scatters the K
+// kept weights of one column into a zeroed [G][kSlab] tile in shared memory,
+// then the block writes the G rows of the slab with 16-byte stores.  Index sets
+// must be strictly increasing (as cci_pack writes them); anything else is
+// reported as CCI_ERR_INDEX.
 // ===========================================================================
-namespace tf {
+namespace dc {
 
-constexpr int kM = 128, kN = 128, kKS = 32, kStages = 3, kLag = 1;
-constexpr int kThreads = 288;
-constexpr int kPlane = kM * kKS * 4;          // 16 KB: one 128 x 32 fp32 plane (A or B)
-constexpr int kStage = 4 * kPlane;            // A hi, A lo, B hi, B lo
-constexpr int kTmemCols = 256;                // two 128-column accumulators
-constexpr size_t kSmemBytes = 1024 + kStages * kStage + sizeof(tc::Smem) + 64;
-constexpr uint32_t kIdesc = (1u << 4)                 // D f32
-                            | (2u << 7) | (2u << 10)  // A, B tf32
-                            | (static_cast<uint32_t>(kN >> 3) << 17) | (static_cast<uint32_t>(kM >> 4) << 24);
-
-__device__ __forceinline__ void mma_tf32(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t accumulate)
-{
-    asm volatile(
-        "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
-        "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(tmem_d),
-        "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(accumulate)
-        : "memory");
-}
-
-// byte offset of (row, element k) in a K-major plane of 128-byte rows (32 fp32)
-// with the 128-byte swizzle
-__device__ __forceinline__ uint32_t sw128f(int row, int k)
-{
-    return static_cast<uint32_t>(row * 128 + (((k >> 2) ^ (row & 7)) * 16) + (k & 3) * 4);
-}
-
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
-{
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
-}
+constexpr int kSlab = 256;  // columns r per block (= threads per block)
 
 __device__ __forceinline__ uint32_t hi_bits(uint32_t x) { return x & 0xffffe000u; }
 __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
@@ -348,106 +323,80 @@ __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
     return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
 }
 
-// one thread per (group gi, r): the hi and lo planes of the G dense weights of
-// column r (zero except the K kept ones); index sets strictly increasing
-template <int G, int K>
-__global__ void decompress_f32_split_kernel(const float *__restrict__ values, const uint8_t *__restrict__ idx,
-                                            int64_t Cout, int64_t R, float *__restrict__ wh, float *__restrict__ wl,
-                                            uint32_t *status)
+// T = uint16_t (bf16 bits) or uint32_t (fp32 bits); SPLIT: write hi to w0 and
+// lo to w1 (fp32 only), else the weights to w0.  R must be a multiple of the
+// elements per 16 bytes.
+template <typename T, int G, int K, bool SPLIT>
+__global__ void __launch_bounds__(kSlab) decompress_kernel(const T *__restrict__ values,
+                                                           const uint8_t *__restrict__ idx, int64_t R,
+                                                           int64_t slabs, T *__restrict__ w0, T *__restrict__ w1,
+                                                           uint32_t *status)
 {
-    const int64_t total = (Cout / G) * R;
-    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
-         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t gi = t / R, r = t - gi * R;
-        uint32_t v[K];
-        int ix[K];
+    constexpr int V = 16 / static_cast<int>(sizeof(T));  // elements per 16-byte store
+    __shared__ __align__(16) T tile[G][kSlab];
+    const int64_t gi = blockIdx.x / slabs;
+    const int64_t r0 = (blockIdx.x - gi * slabs) * kSlab;
+    for (int e = threadIdx.x; e < G * kSlab / V; e += kSlab)
+        reinterpret_cast<uint4 *>(&tile[0][0])[e] = make_uint4(0, 0, 0, 0);
+    __syncthreads();
+    const int64_t r = r0 + threadIdx.x;
+    if (r < R) {
+        const int64_t t = gi * R + r;
         bool bad = false;
+        int prev = -1;
 #pragma unroll
         for (int s = 0; s < K; ++s) {
-            v[s] = __float_as_uint(values[t * K + s]);
-            ix[s] = idx[t * K + s];
-            bad |= ix[s] >= G || (s > 0 && ix[s] <= ix[s - 1]);
+            const T v = values[t * K + s];
+            const int j = idx[t * K + s];
+            bad |= j >= G || j <= prev;
+            prev = j;
+            if (j < G) tile[j][threadIdx.x] = v;
         }
         if (bad) report(status, CCI_ERR_INDEX);
-#pragma unroll
-        for (int j = 0; j < G; ++j) {
-            uint32_t o = 0;
-#pragma unroll
-            for (int s = 0; s < K; ++s) o = (ix[s] == j) ? v[s] : o;
-            wh[(gi * G + j) * R + r] = __uint_as_float(hi_bits(o));
-            wl[(gi * G + j) * R + r] = __uint_as_float(lo_bits(o));
+    }
+    __syncthreads();
+    constexpr int kVecs = kSlab / V;  // 16-byte vectors per tile row
+    for (int e = threadIdx.x; e < G * kVecs; e += kSlab) {
+        const int j = e / kVecs, c = e - j * kVecs;
+        const int64_t rr = r0 + static_cast<int64_t>(c) * V;
+        if (rr >= R) continue;
+        const uint4 x = *reinterpret_cast<const uint4 *>(&tile[j][c * V]);
+        const int64_t off = (gi * G + j) * R + rr;
+        if constexpr (SPLIT) {
+            __stcg(reinterpret_cast<uint4 *>(w0 + off), make_uint4(hi_bits(x.x), hi_bits(x.y), hi_bits(x.z), hi_bits(x.w)));
+            __stcg(reinterpret_cast<uint4 *>(w1 + off), make_uint4(lo_bits(x.x), lo_bits(x.y), lo_bits(x.z), lo_bits(x.w)));
+        } else {
+            __stcg(reinterpret_cast<uint4 *>(w0 + off), x);
         }
     }
 }
 
-}  // namespace tf
-
-// one thread per (group gi, r): the G weights W[gi*G + j][r] of the dense
-// matrix, zero except the K kept ones (bf16 copied bit for bit); index sets
-// must be strictly increasing (as cci_pack writes them)
-template <int G, int K>
-__global__ void decompress_bf16_kernel(const uint16_t *__restrict__ values, const uint8_t *__restrict__ idx,
-                                       int64_t Cout, int64_t R, uint16_t *__restrict__ wd, uint32_t *status)
+template <typename T, int G, int K, bool SPLIT>
+cudaError_t launch(const FwdParams &p, cudaStream_t stream)
 {
-    const int64_t total = (Cout / G) * R;
-    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
-         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t gi = t / R, r = t - gi * R;
-        uint16_t v[K];
-        int ix[K];
-        bool bad = false;
-#pragma unroll
-        for (int s = 0; s < K; ++s) {
-            v[s] = values[t * K + s];
-            ix[s] = idx[t * K + s];
-            bad |= ix[s] >= G || (s > 0 && ix[s] <= ix[s - 1]);
-        }
-        if (bad) report(status, CCI_ERR_INDEX);
-#pragma unroll
-        for (int j = 0; j < G; ++j) {
-            uint16_t o = 0;
-#pragma unroll
-            for (int s = 0; s < K; ++s) o = (ix[s] == j) ? v[s] : o;
-            wd[(gi * G + j) * R + r] = o;
-        }
-    }
+    const int64_t slabs = (p.R + kSlab - 1) / kSlab;
+    const int64_t blocks = (p.Cout / G) * slabs;
+    if (blocks > 0x7fffffff) return cudaErrorInvalidValue;
+    T *w0 = static_cast<T *>(const_cast<void *>(p.wdense));
+    T *w1 = SPLIT ? w0 + p.Cout * p.R : nullptr;
+    decompress_kernel<T, G, K, SPLIT><<<static_cast<unsigned>(blocks), kSlab, 0, stream>>>(
+        static_cast<const T *>(p.values), p.idx, p.R, slabs, w0, w1, p.status);
+    return cudaGetLastError();
 }
+
+}  // namespace dc
 
 // (G, K) pairs with a dense tensor-core instantiation (G divides the 256-channel tile)
 cudaError_t launch_dense_tc(const FwdParams &p, int dtype, int G, int K, bool ws, cudaStream_t stream)
 {
-    if (dtype == CCI_F32) {
-        if (!ws) return cudaErrorNotSupported;
-#define CCI_TF_CASE(g, k)                                                                            \
-    if (G == g && K == k) {                                                                          \
-        const int64_t total = (p.Cout / g) * p.R;                                                    \
-        const int64_t blocks = (total + 255) / 256;                                                  \
-        float *wh = static_cast<float *>(const_cast<void *>(p.wdense));                              \
-        tf::decompress_f32_split_kernel<g, k><<<static_cast<unsigned>(blocks < 65536 * 8 ? blocks : 65536 * 8), 256, \
-                                                0, stream>>>(static_cast<const float *>(p.values), p.idx, p.Cout, p.R, \
-                                                             wh, wh + p.Cout * p.R, p.status);             \
-        const cudaError_t e = cudaGetLastError();                                                    \
-        if (e != cudaSuccess) return e;                                                              \
-        return launch_gemm_ws(p, CCI_F32, stream);                                                   \
-    }
-        CCI_TF_CASE(4, 1) CCI_TF_CASE(4, 2)
-        CCI_TF_CASE(8, 1) CCI_TF_CASE(8, 2) CCI_TF_CASE(8, 4)
-        CCI_TF_CASE(16, 1) CCI_TF_CASE(16, 2) CCI_TF_CASE(16, 4) CCI_TF_CASE(16, 8)
-        CCI_TF_CASE(32, 1) CCI_TF_CASE(32, 2) CCI_TF_CASE(32, 4) CCI_TF_CASE(32, 8) CCI_TF_CASE(32, 16)
-#undef CCI_TF_CASE
-        return cudaErrorNotSupported;
-    }
-#define CCI_TC_CASE(g, k)                                                                          \
-    if (G == g && K == k) {                                                                        \
-        if (!ws) return tc::launch<g, k, false>(p, stream);                                        \
-        const int64_t total = (p.Cout / g) * p.R;                                                  \
-        const int64_t blocks = (total + 255) / 256;                                                \
-        decompress_bf16_kernel<g, k><<<static_cast<unsigned>(blocks < 65536 * 8 ? blocks : 65536 * 8), 256, 0, \
-                                       stream>>>(static_cast<const uint16_t *>(p.values), p.idx, p.Cout, p.R, \
-                                                 static_cast<uint16_t *>(const_cast<void *>(p.wdense)), p.status); \
-        const cudaError_t e = cudaGetLastError();                                                  \
-        if (e != cudaSuccess) return e;                                                            \
-        return launch_gemm_ws(p, CCI_BF16, stream);                                                \
+    if (dtype == CCI_F32 && !ws) return cudaErrorNotSupported;
+#define CCI_TC_CASE(g, k)                                                                   \
+    if (G == g && K == k) {                                                                 \
+        if (!ws) return tc::launch<g, k, false>(p, stream);                                 \
+        const cudaError_t e = dtype == CCI_F32 ? dc::launch<uint32_t, g, k, true>(p, stream) \
+                                               : dc::launch<uint16_t, g, k, false>(p, stream); \
+        if (e != cudaSuccess) return e;                                                     \
+        return launch_gemm_ws(p, dtype, stream);                                            \
     }
     CCI_TC_CASE(4, 1) CCI_TC_CASE(4, 2)
     CCI_TC_CASE(8, 1) CCI_TC_CASE(8, 2) CCI_TC_CASE(8, 4)

@@ -1,0 +1,655 @@
+// cci_gemm_ws.cuh -- the dense tensor-core product of the workspace family
+// (CCI_ALGO_DENSE_TC_WS) after the one-pass decompression of the packed weights.
+//
+// D[n][co] = sum_r x[n][r] * Wd[co][r] on tcgen05 with fp32 accumulators in TMEM,
+// tile [128 n][BN co], BN in {64, 128, 256}, two BN-column accumulators:
+//   bf16:  A = activation tile [128 n][64 r], B = weight tile [BN co][64 r], one
+//          kind::f16 MMA per 16 r.
+//   tf32x3 (fp32 layers): every operand split as hi + lo (hi: the low 13 mantissa
+//          bits cleared, exactly a tf32 value; lo = x - hi exactly); per 8 r three
+//          kind::tf32 MMAs lo*hi + hi*lo + hi*hi; 32 r per stage, planes A hi,
+//          A lo, B hi, B lo.
+// Operands (all K-major, 128-byte swizzle, 1024-byte aligned stage buffers):
+//   weights      TMA from the workspace planes (tensor maps over [Cout][R]);
+//   activations  one of (the template's ASRC):
+//     kA2d      products: TMA over X[N][Cin];
+//     kA4d      stride-1 convolutions with Cin a multiple of the stage depth:
+//               TMA over X[B][H][W][Cin] with a box of QB x PB x BB output
+//               pixels (QB*PB*BB <= 128 rows), shifted by the tap (kh, kw); the
+//               zero padding is the copy's out-of-range fill;
+//     kAGather  other convolutions: the producer warps gather rows (cp.async for
+//               bf16; registers, two stages ahead, then the hi/lo split, for fp32).
+//   fp32 activations copied by TMA land raw in the hi plane and the producer warps
+//   split them in place.
+// Output: fp32 Y written by TMA stores from a swizzled staging buffer (two
+// alternating 16 KB buffers of [128 rows][32 columns]), 2-D over Y[N][Cout] or,
+// for kA4d, 4-D over Y[B][P][Q][Cout] with the tile's pixel box.
+// Roles: warps 0-3 epilogue (TMEM lanes), warps 4-7 producers of the activation
+// planes that are not copied by TMA, warp 8 allocates TMEM and issues the MMAs,
+// warp 9 issues the TMA copies as soon as a stage is free (so copy latency
+// overlaps the producers' work).  Every mbarrier wait is bounded
+// (CCI_ERR_TIMEOUT, abort flag, drain, TMEM freed).
+#pragma once
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "cci_tc_common.cuh"
+
+namespace cci {
+namespace ws {
+
+enum ASrc { kA2d = 0, kA4d = 1, kAGather = 2 };
+
+// output-pixel box of one M tile of a convolution whose activations are copied
+// by 4-D TMA: rows m = (bi*PB + pi)*QB + qi of the tile are the pixels
+// (b0 + bi, p0 + pi, q0 + qi); rows >= QB*PB*BB are unused
+struct ConvBox {
+    int QB, PB, BB;  // box extent along q, p and the batch
+    int nQ, nP;      // boxes along q and p (the batch index is the rest)
+    int rows;        // QB * PB * BB
+    int64_t B;       // batch size
+};
+
+template <bool TF32, int ASRC, int BN>
+struct Cfg {
+    static constexpr int kM = 128, kN = BN;
+    static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
+    static constexpr int kAPlanes = TF32 ? 2 : 1, kBPlanes = TF32 ? 2 : 1;
+    static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
+    static constexpr bool kARaw = TF32 && ASRC != kAGather;   // raw fp32 A by TMA, split by the producers
+    static constexpr int kAPlane = kM * 128;                    // bytes: 128-byte rows
+    static constexpr int kBPlane = kN * 128;
+    static constexpr int kStage = kAPlanes * kAPlane + kBPlanes * kBPlane;
+    static constexpr int kYBuf = kM * 128;  // one output staging buffer: [128 rows][32 fp32]
+    static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - 2 * kYBuf - 1024;
+    static constexpr int kStages = (kBudget / kStage) < tc::kMaxStages ? (kBudget / kStage) : tc::kMaxStages;
+    static constexpr int kTmemCols = 2 * kN;
+    static constexpr size_t kSmem =
+        1024 + static_cast<size_t>(kStages) * kStage + 2 * kYBuf + sizeof(tc::Smem) + 64;
+    static constexpr uint32_t kBBytes = kBPlanes * kBPlane;
+    static constexpr uint32_t kIdesc = (1u << 4)                                           // D f32
+                                       | (TF32 ? (2u << 7) | (2u << 10) : (1u << 7) | (1u << 10))  // tf32 / bf16
+                                       | (static_cast<uint32_t>(kN >> 3) << 17) |
+                                       (static_cast<uint32_t>(kM >> 4) << 24);
+    static_assert(kSmem <= kMaxSmemPerBlock, "stage buffers over the per-block limit");
+    static_assert(kStages >= 3, "too few pipeline stages");
+    static_assert(kTmemCols == 128 || kTmemCols == 256 || kTmemCols == 512, "TMEM allocation not a power of 2");
+};
+
+template <bool TF32>
+__device__ __forceinline__ void mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc)
+{
+    if constexpr (TF32) {
+        asm volatile(
+            "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+            "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+            "l"(a), "l"(b), "r"(idesc), "r"(acc)
+            : "memory");
+    } else {
+        asm volatile(
+            "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+            "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+            "l"(a), "l"(b), "r"(idesc), "r"(acc)
+            : "memory");
+    }
+}
+
+// byte offset of (row, 16-byte chunk) in a plane of 128-byte rows, 128-byte swizzle
+__device__ __forceinline__ uint32_t sw_chunk(int row, int chunk)
+{
+    return static_cast<uint32_t>(row * 128 + ((chunk ^ (row & 7)) * 16));
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
+{
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+__device__ __forceinline__ uint32_t hi_bits(uint32_t x) { return x & 0xffffe000u; }
+__device__ __forceinline__ uint32_t lo_bits(uint32_t x)
+{
+    return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
+}
+
+constexpr int kThreads = 320;
+
+// (box along q, box along p, batch box) of M tile mt
+struct BoxIdx {
+    int qb, pb;
+    int64_t bb;
+};
+__device__ __forceinline__ BoxIdx box_of(int64_t mt, const ConvBox &box)
+{
+    BoxIdx i;
+    i.qb = static_cast<int>(mt % box.nQ);
+    const int64_t t = mt / box.nQ;
+    i.pb = static_cast<int>(t % box.nP);
+    i.bb = t / box.nP;
+    return i;
+}
+
+template <bool TF32, int ASRC, int BN>
+__global__ void __launch_bounds__(kThreads, 1)
+    gemm_ws_kernel(FwdParams p, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+                   const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmY, ConvBox box,
+                   int64_t n_ct, int64_t n_tiles)
+{
+    using C = Cfg<TF32, ASRC, BN>;
+    constexpr int kM = C::kM, kN = C::kN, kKS = C::kKS, kStages = C::kStages;
+    constexpr int kLag = 2;  // bf16 gather: stages in flight before a producer's arrive
+    extern __shared__ __align__(16) unsigned char smem_raw[];
+    const uint32_t raw = tc::smem_u32(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    const uint32_t ybuf = base + kStages * C::kStage;  // two output staging buffers
+    tc::Smem *S = reinterpret_cast<tc::Smem *>(smem_raw + (base - raw) + kStages * C::kStage + 2 * C::kYBuf);
+    volatile int *abort = &S->abort;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int nks = static_cast<int>((p.R + kKS - 1) / kKS);
+
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            tc::mbar_init(&S->full[s], C::kATma ? 1 : 129);
+            tc::mbar_init(&S->empty[s], 1);
+            tc::mbar_init(&S->aux[s], 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            tc::mbar_init(&S->tmem_full[a], 1);
+            tc::mbar_init(&S->tmem_empty[a], 128);
+        }
+        tc::mbar_init(&S->drain, 1);
+        S->abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (ASRC == kA4d && box.rows < kM) {
+        // rows past the box are never copied: keep them zero for the MMAs
+        for (uint32_t o = static_cast<uint32_t>(tid) * 16; o < static_cast<uint32_t>(kStages * C::kStage);
+             o += kThreads * 16)
+            tc::st_shared_v4_zero(base + o);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 8) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         tc::smem_u32(&S->tmem_base)),
+                     "r"(C::kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    if (tid == 288) {
+        if constexpr (ASRC != kAGather) tc::tma_prefetch_desc(&tmA);
+        tc::tma_prefetch_desc(&tmB0);
+        if constexpr (C::kBPlanes > 1) tc::tma_prefetch_desc(&tmB1);
+        tc::tma_prefetch_desc(&tmY);
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = S->tmem_base;
+
+    if (warp == 9) {
+        // ------------------------------------------------------------ TMA issuer
+        const uint32_t a_bytes = ASRC == kA4d ? static_cast<uint32_t>(box.rows) * 128u : C::kAPlane;
+        const int cpt = static_cast<int>(p.Cin / kKS);  // stages per tap (kA4d)
+        int it = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            const int64_t mt = tile / n_ct;
+            const int64_t co0 = (tile % n_ct) * kN;
+            BoxIdx bi{0, 0, 0};
+            if constexpr (ASRC == kA4d) bi = box_of(mt, box);
+            for (int ks = 0; ks < nks && ok; ++ks, ++it) {
+                const int s = it % kStages;
+                if (it >= kStages) ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
+                if (!ok) break;
+                if (lane == 0) {
+                    const uint32_t st = base + s * C::kStage;
+                    const uint32_t bst = st + C::kAPlanes * C::kAPlane;
+                    // the activation copy completes on aux (raw fp32, split afterwards) or full
+                    uint64_t *abar = C::kARaw ? &S->aux[s] : &S->full[s];
+                    if constexpr (C::kARaw) tc::mbar_arrive_expect_tx(abar, a_bytes);
+                    tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes + (C::kATma ? a_bytes : 0u));
+                    tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                    if constexpr (C::kBPlanes > 1)
+                        tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                    if constexpr (ASRC == kA2d) {
+                        tc::tma_load_2d(st, &tmA, ks * kKS, static_cast<int>(mt * kM), abar);
+                    } else if constexpr (ASRC == kA4d) {
+                        const int tap = ks / cpt;
+                        const int ci0 = (ks - tap * cpt) * kKS;
+                        const int kh = tap / p.KW, kw = tap - (tap / p.KW) * p.KW;
+                        tc::tma_load_4d(st, &tmA, ci0, bi.qb * box.QB - p.pw + kw, bi.pb * box.PB - p.ph + kh,
+                                        static_cast<int>(bi.bb * box.BB), abar);
+                    }
+                }
+                __syncwarp();
+            }
+        }
+    } else if (warp >= 4 && warp < 8) {
+        // ------------------------------------------------------------ producers
+        const int pt = tid - 128;
+        const int chunk = pt & 7;  // 16-byte chunk of every activation row this thread handles
+        const int rowb = pt >> 3;  // rows rowb + 16 i
+        int it = 0;
+        bool ok = true;
+        constexpr bool kRegs = TF32 && ASRC == kAGather;  // fp32 gather through registers
+        // fp32 gather: activation chunks of the next two stages, in registers
+        uint4 xa[kRegs ? 8 : 1], xb[kRegs ? 8 : 1], xc[kRegs ? 8 : 1];
+        ColumnSite xsite[kRegs ? 8 : 1];  // column sites of the tile being prefetched
+        int64_t xsite_tile = -1;
+        auto load_x = [&](uint4 (&dst)[kRegs ? 8 : 1], int64_t tile, int ks) {
+            if constexpr (kRegs) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) dst[i] = make_uint4(0, 0, 0, 0);
+                if (tile >= n_tiles || ks >= nks) return;
+                const int64_t n0 = (tile / n_ct) * kM;
+                if (tile != xsite_tile) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int64_t n = n0 + rowb + 16 * i;
+                        xsite[i] = n < p.N ? column_site(p, n) : ColumnSite{-1, 0, 0};
+                    }
+                    xsite_tile = tile;
+                }
+                const int64_t r = static_cast<int64_t>(ks) * kKS + chunk * 4;
+                if (r >= p.R) return;
+                int kh = 0, kw = 0;
+                int64_t ci = r;
+                if (p.is_conv) {
+                    const int tap = static_cast<int>(r / p.Cin);
+                    ci = r - static_cast<int64_t>(tap) * p.Cin;
+                    kh = tap / p.KW;
+                    kw = tap - kh * p.KW;
+                }
+                const float *X = static_cast<const float *>(p.X);
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    if (xsite[i].img < 0) continue;  // column past N
+                    int64_t off = xsite[i].img + r;
+                    if (p.is_conv) {
+                        const int h = xsite[i].hb + kh, w = xsite[i].wb + kw;
+                        if (h < 0 || h >= p.H || w < 0 || w >= p.W) continue;
+                        off = xsite[i].img + (static_cast<int64_t>(h) * p.W + w) * p.Cin + ci;
+                    }
+                    dst[i] = __ldg(reinterpret_cast<const uint4 *>(X + off));
+                }
+            }
+        };
+        // (tile, ks) of the stage after (tile, ks)
+        auto advance = [&](int64_t &tile, int &ks) {
+            if (++ks == nks) {
+                ks = 0;
+                tile += gridDim.x;
+            }
+        };
+        int64_t t2 = blockIdx.x;
+        int k2 = 0;
+        if constexpr (kRegs) {
+            load_x(xa, t2, k2);
+            advance(t2, k2);
+            load_x(xb, t2, k2);
+            advance(t2, k2);
+        }
+        if constexpr (!C::kATma) {
+            for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+                const int64_t n0 = (tile / n_ct) * kM;
+                ColumnSite site[8];
+                bool colok[8];
+                if constexpr (!TF32) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int64_t n = n0 + rowb + 16 * i;
+                        colok[i] = n < p.N;
+                        site[i] = colok[i] ? column_site(p, n) : ColumnSite{0, 0, 0};
+                    }
+                }
+                for (int ks = 0; ks < nks && ok; ++ks, ++it) {
+                    const int s = it % kStages;
+                    if constexpr (kRegs) load_x(xc, t2, k2);  // two stages ahead
+                    // gather / register modes write the stage themselves: wait until it is
+                    // free; the split mode waits for its raw tile (copied after the stage
+                    // was freed) instead
+                    if (!C::kARaw && it >= kStages)
+                        ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
+                    if (!ok) break;
+                    const uint32_t st = base + s * C::kStage;
+                    if constexpr (!TF32) {
+                        const uint16_t *X = static_cast<const uint16_t *>(p.X);
+                        const int64_t r = static_cast<int64_t>(ks) * kKS + chunk * 8;
+                        const bool rok = r < p.R;
+                        int kh = 0, kw = 0;
+                        int64_t ci = r;
+                        if (p.is_conv && rok) {
+                            const int tap = static_cast<int>(r / p.Cin);
+                            ci = r - static_cast<int64_t>(tap) * p.Cin;
+                            kh = tap / p.KW;
+                            kw = tap - kh * p.KW;
+                        }
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            bool valid = colok[i] && rok;
+                            const uint16_t *src = X;
+                            if (valid) {
+                                if (!p.is_conv) {
+                                    src = X + site[i].img + r;
+                                } else {
+                                    const int h = site[i].hb + kh, w = site[i].wb + kw;
+                                    valid = h >= 0 && h < p.H && w >= 0 && w < p.W;
+                                    if (valid)
+                                        src = X + site[i].img + (static_cast<int64_t>(h) * p.W + w) * p.Cin + ci;
+                                }
+                            }
+                            tc::cp_async16(st + sw_chunk(rowb + 16 * i, chunk), src, valid);
+                        }
+                        asm volatile("cp.async.commit_group;" ::: "memory");
+                        if (it >= kLag) {
+                            asm volatile("cp.async.wait_group %0;" ::"n"(kLag) : "memory");
+                            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                            tc::mbar_arrive(&S->full[(it - kLag) % kStages]);
+                        }
+                    } else if constexpr (C::kARaw) {
+                        // the raw fp32 tile landed in the hi plane: split it in place
+                        ok = tc::mbar_wait(&S->aux[s], (it / kStages) & 1, abort, p.status);
+                        if (!ok) break;
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const uint32_t o = sw_chunk(rowb + 16 * i, chunk);
+                            uint4 v;
+                            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                                         : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                                         : "r"(st + o)
+                                         : "memory");
+                            st_shared_v4(st + o, hi_bits(v.x), hi_bits(v.y), hi_bits(v.z), hi_bits(v.w));
+                            st_shared_v4(st + C::kAPlane + o, lo_bits(v.x), lo_bits(v.y), lo_bits(v.z),
+                                         lo_bits(v.w));
+                        }
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        tc::mbar_arrive(&S->full[s]);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const uint32_t o = sw_chunk(rowb + 16 * i, chunk);
+                            st_shared_v4(st + o, hi_bits(xa[i].x), hi_bits(xa[i].y), hi_bits(xa[i].z),
+                                         hi_bits(xa[i].w));
+                            st_shared_v4(st + C::kAPlane + o, lo_bits(xa[i].x), lo_bits(xa[i].y), lo_bits(xa[i].z),
+                                         lo_bits(xa[i].w));
+                        }
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        tc::mbar_arrive(&S->full[s]);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            xa[i] = xb[i];
+                            xb[i] = xc[i];
+                        }
+                        advance(t2, k2);
+                    }
+                }
+            }
+            if constexpr (!TF32) {
+                asm volatile("cp.async.wait_group 0;" ::: "memory");
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                for (int q = (it >= kLag ? it - kLag : 0); q < it; ++q) tc::mbar_arrive(&S->full[q % kStages]);
+            }
+        }
+    } else if (warp == 8) {
+        // ------------------------------------------------------------ MMA issuer
+        int it = 0, t = 0;
+        bool ok = true;
+        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+            const int acc = t & 1;
+            if (t >= 2) ok = tc::mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
+            if (!ok) break;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
+            for (int ks = 0; ks < nks && ok; ++ks, ++it) {
+                const int s = it % kStages;
+                ok = tc::mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
+                if (!ok) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                if (lane == 0) {
+                    const uint32_t st = base + s * C::kStage;
+                    const uint32_t bst = st + C::kAPlanes * C::kAPlane;
+                    if constexpr (TF32) {
+#pragma unroll
+                        for (int k = 0; k < kKS / 8; ++k) {
+                            const uint64_t ah = tc::sw128_desc(st + k * 32);
+                            const uint64_t al = tc::sw128_desc(st + C::kAPlane + k * 32);
+                            const uint64_t bh = tc::sw128_desc(bst + k * 32);
+                            const uint64_t bl = tc::sw128_desc(bst + C::kBPlane + k * 32);
+                            mma<TF32>(d, al, bh, C::kIdesc, (ks > 0 || k > 0) ? 1u : 0u);
+                            mma<TF32>(d, ah, bl, C::kIdesc, 1u);
+                            mma<TF32>(d, ah, bh, C::kIdesc, 1u);
+                        }
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < kKS / 16; ++k)
+                            mma<TF32>(d, tc::sw128_desc(st + k * 32), tc::sw128_desc(bst + k * 32), C::kIdesc,
+                                      (ks > 0 || k > 0) ? 1u : 0u);
+                    }
+                    tc::mma_commit(&S->empty[s]);
+                }
+                __syncwarp();
+            }
+            if (ok && lane == 0) tc::mma_commit(&S->tmem_full[acc]);
+            __syncwarp();
+        }
+        if (lane == 0) tc::mma_commit(&S->drain);
+        __syncwarp();
+        int no_abort = 0;
+        tc::mbar_wait(&S->drain, 0, &no_abort, p.status);
+    } else {
+        // ------------------------------------------------------------ epilogue (warps 0-3)
+        // Per 32-column chunk: TMEM -> registers -> swizzled staging buffer (row m =
+        // thread) -> one TMA store of the tile's box (rows past N, the image or
+        // Cout are clipped by the copy).  Two buffers alternate; a buffer is
+        // rewritten once the store issued from it two chunks earlier has read it.
+        // Every decision that gates a named barrier is uniform over the 128
+        // threads (named_and), so the barriers always see all of them.
+        int t = 0;
+        bool ok = true;
+        const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
+        const int m = tid;  // accumulator row = TMEM lane
+        int chunk_no = 0;
+        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+            const int acc = t & 1;
+            const int64_t mt = tile / n_ct;
+            const int co0 = static_cast<int>((tile % n_ct) * kN);
+            BoxIdx bi{0, 0, 0};
+            if constexpr (ASRC == kA4d) bi = box_of(mt, box);
+            ok = tc::mbar_wait(&S->tmem_full[acc], (t / 2) & 1, abort, p.status);
+            ok = tc::named_and(1, 128, ok);
+            if (!ok) break;
+            __syncwarp();
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+#pragma unroll 1
+            for (int c = 0; c < kN / 32 && co0 + c * 32 < p.Cout; ++c, ++chunk_no) {
+                uint32_t v[32];
+                tc::tmem_ld32(tmem + lane_off + static_cast<uint32_t>(acc * kN + c * 32), v);
+                const uint32_t buf = ybuf + static_cast<uint32_t>(chunk_no & 1) * C::kYBuf;
+                if (tid == 0) tc::bulk_wait_read<1>();
+                tc::named_sync(1, 128);
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    st_shared_v4(buf + sw_chunk(m, q), v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                tc::named_sync(1, 128);
+                if (tid == 0) {
+                    if constexpr (ASRC == kA4d)
+                        tc::tma_store_4d(&tmY, buf, co0 + c * 32, bi.qb * box.QB, bi.pb * box.PB,
+                                         static_cast<int>(bi.bb * box.BB));
+                    else
+                        tc::tma_store_2d(&tmY, buf, co0 + c * 32, static_cast<int>(mt * kM));
+                    tc::bulk_commit();
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            tc::mbar_arrive(&S->tmem_empty[acc]);
+        }
+        if (tid == 0) tc::bulk_wait_all();
+    }
+
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 8) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::kTmemCols)
+                     : "memory");
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host: tensor maps, tile choice and launch
+// ---------------------------------------------------------------------------
+inline PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+        return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    }();
+    return fn;
+}
+
+// map over a row-major array of `rank` dims (dims[0] innermost, element count
+// each), box[] elements per dim, 128-byte swizzle (box[0] * elem must be 128)
+inline bool make_map(CUtensorMap *m, const void *ptr, CUtensorMapDataType dt, int elem, int rank,
+                     const int64_t *dims, const int *box)
+{
+    auto fn = encode_fn();
+    if (!fn || rank < 1 || rank > 5) return false;
+    cuuint64_t gd[5], gs[4];
+    cuuint32_t bx[5], es[5];
+    uint64_t stride = static_cast<uint64_t>(elem);
+    for (int i = 0; i < rank; ++i) {
+        gd[i] = static_cast<cuuint64_t>(dims[i]);
+        bx[i] = static_cast<cuuint32_t>(box[i]);
+        es[i] = 1;
+        if (i > 0) gs[i - 1] = static_cast<cuuint64_t>(stride);
+        stride *= static_cast<uint64_t>(dims[i]);
+    }
+    return fn(m, dt, static_cast<cuuint32_t>(rank), const_cast<void *>(ptr), gd, gs, bx, es,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+inline int sm_count()
+{
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return sms > 0 ? sms : 1;
+}
+
+// the output-pixel box with the fewest M tiles (ties: longer runs along q, then
+// p).  Only the smallest box of each tile count along q and p is tried.
+inline ConvBox choose_box(int64_t B, int64_t P, int64_t Q)
+{
+    ConvBox best{1, 1, 1, 1, 1, 1, B};
+    int64_t best_tiles = -1;
+    for (int64_t QB = 1; QB <= Q && QB <= 128; ++QB) {
+        const int64_t nq = (Q + QB - 1) / QB;
+        if ((Q + nq - 1) / nq != QB) continue;
+        for (int64_t PB = 1; PB <= P && QB * PB <= 128; ++PB) {
+            const int64_t np = (P + PB - 1) / PB;
+            if ((P + np - 1) / np != PB) continue;
+            const int64_t BB = (128 / (QB * PB)) < B ? 128 / (QB * PB) : B;
+            const int64_t tiles = nq * np * ((B + BB - 1) / BB);
+            if (best_tiles < 0 || tiles <= best_tiles) {
+                best_tiles = tiles;
+                best.QB = static_cast<int>(QB);
+                best.PB = static_cast<int>(PB);
+                best.BB = static_cast<int>(BB);
+            }
+        }
+    }
+    best.nQ = static_cast<int>((Q + best.QB - 1) / best.QB);
+    best.nP = static_cast<int>((P + best.PB - 1) / best.PB);
+    best.rows = best.QB * best.PB * best.BB;
+    best.B = B;
+    return best;
+}
+
+// the activation source of a layer for stage depth ks (elements per 128-byte row)
+inline int a_source(const FwdParams &p, int ks)
+{
+    const int64_t lim = int64_t(1) << 30;
+    if (!p.is_conv) return p.N < lim ? kA2d : kAGather;
+    const bool fits = p.H < lim && p.W < lim && p.N < lim && (p.N / (p.P * p.Q)) < lim;
+    return (p.sh == 1 && p.sw == 1 && p.Cin % ks == 0 && fits) ? kA4d : kAGather;
+}
+
+// N tile among {64, 128, 256} (up to max_bn): fewest rounds of tiles over the
+// SMs weighted by the tile's width plus a fixed per-tile cost; ties: the wider
+inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn)
+{
+    const int64_t sms = sm_count();
+    int best = 64;
+    int64_t best_cost = -1;
+    for (int bn = 64; bn <= max_bn; bn *= 2) {
+        const int64_t tiles = m_tiles * ((Cout + bn - 1) / bn);
+        const int64_t cost = ((tiles + sms - 1) / sms) * (bn + 32);
+        if (best_cost < 0 || cost <= best_cost) {
+            best_cost = cost;
+            best = bn;
+        }
+    }
+    return best;
+}
+
+template <bool TF32, int ASRC, int BN>
+cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, cudaStream_t stream)
+{
+    using C = Cfg<TF32, ASRC, BN>;
+    auto kern = gemm_ws_kernel<TF32, ASRC, BN>;
+    static const cudaError_t attr =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::kSmem));
+    if (attr != cudaSuccess) return attr;
+    CUtensorMap tmA{}, tmB0{}, tmB1{}, tmY{};
+    const CUtensorMapDataType dt = TF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const int elem = TF32 ? 4 : 2;
+    if constexpr (ASRC == kA2d) {
+        const int64_t dims[2] = {p.Cin, p.N};
+        const int bx[2] = {C::kKS, C::kM};
+        if (!make_map(&tmA, p.X, dt, elem, 2, dims, bx)) return cudaErrorInvalidValue;
+    } else if constexpr (ASRC == kA4d) {
+        const int64_t dims[4] = {p.Cin, p.W, p.H, box.B};
+        const int bx[4] = {C::kKS, box.QB, box.PB, box.BB};
+        if (!make_map(&tmA, p.X, dt, elem, 4, dims, bx)) return cudaErrorInvalidValue;
+    }
+    const int64_t wdims[2] = {p.R, p.Cout};
+    const int wbox[2] = {C::kKS, C::kN};
+    if (!make_map(&tmB0, p.wdense, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
+    if (C::kBPlanes > 1) {
+        const char *lo = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
+        if (!make_map(&tmB1, lo, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
+    }
+    if constexpr (ASRC == kA4d) {
+        const int64_t dims[4] = {p.Cout, p.Q, p.P, box.B};
+        const int bx[4] = {32, box.QB, box.PB, box.BB};
+        if (!make_map(&tmY, p.Y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, 4, dims, bx)) return cudaErrorInvalidValue;
+    } else {
+        const int64_t dims[2] = {p.Cout, p.N};
+        const int bx[2] = {32, C::kM};
+        if (!make_map(&tmY, p.Y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, 2, dims, bx)) return cudaErrorInvalidValue;
+    }
+    const int64_t n_ct = (p.Cout + C::kN - 1) / C::kN;
+    const int64_t m_tiles = ASRC == kA4d ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)
+                                         : (p.N + C::kM - 1) / C::kM;
+    const int64_t n_tiles = n_ct * m_tiles;
+    const int64_t sms = sm_count();
+    const int64_t grid = n_tiles < sms ? n_tiles : sms;
+    kern<<<static_cast<unsigned>(grid), kThreads, C::kSmem, stream>>>(p, tmA, tmB0, tmB1, tmY, box, n_ct, n_tiles);
+    return cudaGetLastError();
+}
+
+// m tiles of the layer for the chosen activation source
+inline int64_t m_tiles_of(const FwdParams &p, int asrc, const ConvBox &box)
+{
+    if (asrc == kA4d) return static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB);
+    return (p.N + 127) / 128;
+}
+
+}  // namespace ws
+}  // namespace cci

@@ -1,0 +1,31 @@
+// cci_gemm_ws_tf32.cu -- fp32 layers of the workspace family (three-pass tf32
+// products): the kernel configurations and the choice among them.
+#include "cci_gemm_ws.cuh"
+
+namespace cci {
+
+cudaError_t launch_gemm_ws_tf32(const FwdParams &p, cudaStream_t stream)
+{
+    using namespace ws;
+    const int asrc = a_source(p, 32);
+    ConvBox box{1, 1, 1, 1, 1, 1, 1};
+    if (asrc == kA4d) box = choose_box(p.N / (p.P * p.Q), p.P, p.Q);
+    const int bn = choose_bn(m_tiles_of(p, asrc, box), p.Cout, 128);
+#define CCI_WS_CASE(A, N) \
+    if (asrc == A && bn == N) return launch_cfg<true, A, N>(p, box, stream);
+    CCI_WS_CASE(kA2d, 64)
+    CCI_WS_CASE(kA2d, 128)
+    CCI_WS_CASE(kA4d, 64)
+    CCI_WS_CASE(kA4d, 128)
+    CCI_WS_CASE(kAGather, 64)
+    CCI_WS_CASE(kAGather, 128)
+#undef CCI_WS_CASE
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_gemm_ws(const FwdParams &p, int dtype, cudaStream_t stream)
+{
+    return dtype == CCI_F32 ? launch_gemm_ws_tf32(p, stream) : launch_gemm_ws_bf16(p, stream);
+}
+
+}  // namespace cci

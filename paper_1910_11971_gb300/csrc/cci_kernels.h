@@ -18,8 +18,10 @@ bool dense_tc_supported(int dtype, int G, int K);
 cudaError_t launch_dense_tc(const FwdParams &p, int dtype, int G, int K, bool ws, cudaStream_t stream);
 
 // dense product on the tensor cores from the decompressed workspace p.wdense
-// (cci_gemm_ws.cu): bf16 dense [Cout][R], or fp32 hi / lo tf32 planes [2][Cout][R]
+// (cci_gemm_ws_*.cu): bf16 dense [Cout][R], or fp32 hi / lo tf32 planes [2][Cout][R]
 cudaError_t launch_gemm_ws(const FwdParams &p, int dtype, cudaStream_t stream);
+cudaError_t launch_gemm_ws_bf16(const FwdParams &p, cudaStream_t stream);
+cudaError_t launch_gemm_ws_tf32(const FwdParams &p, cudaStream_t stream);
 
 // One register-tiled instantiation: (dtype, G, K) -> tile shape and launcher.
 struct RegtileEntry {

@@ -9,12 +9,14 @@ namespace tc {
 
 constexpr long long kWaitLimit = 1ll << 31;  // clock cycles (about 1 s) per bounded wait
 
+constexpr int kMaxStages = 8;
+
 // barriers and TMEM slot of a tensor-core kernel (after its 1024-byte aligned
-// stage buffers); up to 4 pipeline stages
+// stage buffers); up to kMaxStages pipeline stages
 struct Smem {
-    uint64_t full[4];
-    uint64_t empty[4];
-    uint64_t aux[4];  // per-stage barrier of a second copy (tf32x3: raw activation tile landed)
+    uint64_t full[kMaxStages];
+    uint64_t empty[kMaxStages];
+    uint64_t aux[kMaxStages];  // per-stage barrier of a second copy (tf32x3: raw activation tile landed)
     uint64_t tmem_full[2];
     uint64_t tmem_empty[2];
     uint64_t drain;
@@ -136,6 +138,68 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const void *tmap, int 
         "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
         ::"r"(dst), "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(smem_u32(bar))
         : "memory");
+}
+
+// 4-D tile load of the box at (c0 innermost, c1, c2, c3); c0 * element size must
+// be a multiple of 16 bytes; the other coordinates may lie outside the tensor
+// (those elements read as zero)
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const void *tmap, int c0, int c1, int c2, int c3,
+                                            uint64_t *bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, "
+        "%5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar))
+        : "memory");
+}
+
+// tile stores from shared memory (bulk-group completion); elements of the box
+// outside the tensor are not written.  Coordinates must not be negative.
+__device__ __forceinline__ void tma_store_2d(const void *tmap, uint32_t src, int c0, int c1)
+{
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(tmap)),
+                 "r"(src), "r"(c0), "r"(c1)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tma_store_4d(const void *tmap, uint32_t src, int c0, int c1, int c2, int c3)
+{
+    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.tile.bulk_group [%0, {%2, %3, %4, %5}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(tmap)),
+                 "r"(src), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+                 : "memory");
+}
+
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+
+// wait until at most N committed bulk groups still read their shared memory
+template <int N>
+__device__ __forceinline__ void bulk_wait_read()
+{
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+
+// wait until every committed bulk group has completed
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+
+// named barrier `id` over `n` threads (non-aligned form: the threads of a warp
+// need not arrive converged)
+__device__ __forceinline__ void named_sync(int id, int n)
+{
+    asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+// named barrier `id` over `n` threads that returns the AND of every thread's v
+__device__ __forceinline__ bool named_and(int id, int n, bool v)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n.reg .pred p, q;\nsetp.ne.u32 p, %1, 0;\nbarrier.red.and.pred q, %2, %3, p;\nselp.u32 %0, 1, 0, q;\n}\n"
+        : "=r"(r)
+        : "r"(static_cast<uint32_t>(v)), "r"(id), "r"(n)
+        : "memory");
+    return r != 0;
 }
 
 __device__ __forceinline__ void tma_prefetch_desc(const void *tmap)

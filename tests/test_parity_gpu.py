@@ -326,14 +326,14 @@ def test_conv3x3_full(dev):
     check_conv_case(dev, case, npts=2048)
 
 
-RESNET_PICK = [0, 1, 3, 4, 11, 13, 24, 25, 42, 44, 49, 51]
+RESNET_PICK = [0, 1, 3, 4, 11, 13, 15, 24, 25, 28, 42, 44, 47, 49, 51]
 
 
 @pytest.mark.parametrize("K", [1, 2, 4])
 @pytest.mark.parametrize("li", RESNET_PICK)
 def test_resnet50_layer(dev, li, K):
-    """Layers of the ResNet-50 stack (batch 128), G=8: first/last 1x1, 3x3 s1 and
-    s2, strided downsample 1x1, 14x14 and 7x7 stages."""
+    """Layers of the ResNet-50 stack (batch 128), G=8: first/last 1x1, 3x3 s1 at
+    every stage (56, 28, 14, 7) and s2, strided downsample 1x1."""
     case = wl.resnet50_layers(K=K)[li]
     check_conv_case(dev, case, npts=512, seed=li)
 
@@ -478,3 +478,49 @@ def test_tf32x3_conv_small(dev, case):
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
     assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
+
+
+# ---------------------------------------------------------------------------
+# convolutions whose activations are copied by 4-D TMA (unit stride, Cin a
+# multiple of 64 for bf16 / 32 for fp32): output-pixel boxes with ragged edges,
+# asymmetric padding, windows wholly inside the padding, every N tile width
+# ---------------------------------------------------------------------------
+# (B, H, W, Cin, Cout, KH, KW, stride, pad, G, K, dtype)
+CONV_TMA = [
+    (3, 9, 7, 64, 64, 3, 3, (1, 1), (1, 1), 8, 2, "bf16"),
+    (2, 13, 11, 128, 192, 3, 3, (1, 1), (1, 1), 16, 4, "bf16"),
+    (1, 6, 20, 64, 32, 5, 3, (1, 1), (2, 0), 4, 2, "bf16"),
+    (5, 7, 7, 64, 128, 3, 3, (1, 1), (0, 0), 8, 4, "bf16"),
+    (2, 4, 4, 64, 64, 3, 3, (1, 1), (3, 3), 8, 1, "bf16"),
+    (2, 5, 5, 64, 64, 1, 1, (1, 1), (1, 1), 8, 2, "bf16"),
+    (33, 3, 5, 192, 256, 3, 3, (1, 1), (1, 1), 32, 8, "bf16"),
+    (2, 9, 7, 32, 64, 3, 3, (1, 1), (1, 1), 8, 2, "f32"),
+    (3, 5, 6, 64, 96, 3, 3, (1, 1), (1, 1), 16, 4, "f32"),
+    (2, 4, 4, 32, 32, 3, 3, (1, 1), (3, 3), 4, 1, "f32"),
+]
+
+
+@pytest.mark.parametrize("case", CONV_TMA, ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
+def test_dense_tc_ws_conv_tma(dev, case):
+    B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
+    g = torch.Generator().manual_seed(B * 17 + Cin + Cout)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(_dt(dtype))
+    W = torch.randn((Cout, KH * KW * Cin), generator=g).to(_dt(dtype))
+    Y = run_conv(dev, X, W, (KH, KW, stride, pad, Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
+
+
+def test_dense_tc_ws_conv_tma_equals_gather_bitwise(dev):
+    """A convolution whose activations arrive by 4-D copy equals, bit for bit,
+    the product of its im2col matrix (2-D copy): same operands, same order."""
+    B, H, Wi, Cin, Cout, G, K = 2, 6, 5, 64, 128, 8, 2
+    X = torch.randn((B, H, Wi, Cin)).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin)).to(BF16)
+    Yc = run_conv(dev, X, W, (3, 3, (1, 1), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    xp = torch.nn.functional.pad(X.float(), (0, 0, 1, 1, 1, 1))
+    cols = torch.stack([xp[:, kh:kh + H, kw:kw + Wi, :] for kh in range(3) for kw in range(3)], dim=3)
+    Xcol = cols.reshape(B * H * Wi, 9 * Cin).to(BF16)
+    Yl = run_linear(dev, Xcol, W, G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.equal(Yc.reshape(-1, Cout).view(torch.int32), Yl.view(torch.int32))
