@@ -75,7 +75,9 @@ def parse():
     ap.add_argument("--profile", type=int, default=0,
                     help="only the warm-up and timed steps of the main path (for ncu)")
     ap.add_argument("--workload", default="bottleneck_1x1",
-                    help="bottleneck_1x1 (default) or sweep_4096_G<G>_K<K>: the product timed")
+                    help="bottleneck_1x1 (default) or sweep_4096_G<G>_K<K>: the product timed; with "
+                         "--profile 1 also a convolution: conv3x3_28 or resnet50_lNN_K<K> (layer NN of "
+                         "the ResNet-50 stack)")
     return ap.parse_args()
 
 
@@ -356,6 +358,42 @@ def workload_case(name: str) -> wl.LinearCase:
     raise SystemExit(f"unknown workload {name}")
 
 
+def conv_case(name: str):
+    """A convolution workload by name, or None."""
+    if name == wl.CONV3X3_28.name:
+        return wl.CONV3X3_28
+    if name.startswith("resnet50_l") and "_K" in name:
+        li, k = name[len("resnet50_l"):].split("_K")
+        return wl.resnet50_layers(K=int(k))[int(li)]
+    return None
+
+
+def profile_conv(cci, case, args, dev, stream):
+    """Warm-up and timed steps (pack + convolution) of one convolution layer, for
+    profiler captures; prints the mean step time."""
+    X, W = wl.conv_inputs(case, device=str(dev))
+    values = torch.empty((case.Cout // case.G, case.R, case.K), dtype=X.dtype, device=dev)
+    idx = torch.empty((case.Cout // case.G, case.R, case.K), dtype=torch.uint8, device=dev)
+    Y = torch.empty((case.B, case.P, case.Q, case.Cout), dtype=torch.float32, device=dev)
+    ws = cci.new_workspace(cci.ALGO_AUTO, X.dtype, case.Cout, case.R, dev)
+    status = cci.new_status(dev)
+    flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+
+    def step():
+        cci.pack(W, case.G, case.K, status=status, check=False, out=(values, idx))
+        cci.conv2d(X, values, idx, case.Cout, case.G, case.K, case.KH, case.KW, (case.stride,) * 2,
+                   (case.pad,) * 2, out=Y, status=status, workspace=ws)
+
+    for _ in range(max(3, args.warmup)):
+        step()
+    torch.cuda.synchronize(dev)
+    ms = time_device(step, args.steps, lambda: flush_buf.fill_(1.0), stream)
+    assert cci.read_status(status) == 0
+    print(json.dumps({"workload": case.name, "ms_per_step": statistics.mean(ms), "steps": args.steps,
+                      "note": "profiling helper: pack + convolution per step"}), flush=True)
+    return 0
+
+
 def run_ours(args, rank, world, local):
     import paper_1910_11971_gb300 as cci
     from paper_1910_11971_gb300 import build as cci_build
@@ -366,6 +404,11 @@ def run_ours(args, rank, world, local):
     stream = torch.cuda.current_stream(dev)
     torch.backends.cuda.matmul.allow_tf32 = False
     torch.backends.cudnn.allow_tf32 = False
+    cc = conv_case(args.workload)
+    if cc is not None:
+        if not args.profile:
+            raise SystemExit("convolution workloads are profiling helpers: pass --profile 1")
+        return profile_conv(cci, cc, args, dev, stream)
     case = workload_case(args.workload)
     X, W = wl.linear_inputs(case, device="cpu")
     X_host = X.pin_memory()
@@ -655,6 +698,15 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
         torch.cuda.synchronize(dev)
         ms = statistics.median(time_device(g_ours.replay, reps, flush, stream))
         dms = statistics.median(time_device(g_dense.replay, reps, flush, stream))
+        per_layer = []
+        if K == 2:  # each layer alone, for the breakdown
+            for c, fo, fd in zip(layers, ours_calls, dense_calls):
+                lm = statistics.median(time_device(fo, reps, flush, stream))
+                ld = statistics.median(time_device(fd, reps, flush, stream))
+                per_layer.append({"layer": c.name, "ms": round(lm, 5), "floor_ms": round(layer_floor_us(c) * 1e-3, 5),
+                                  "cudnn_ms": round(ld, 5),
+                                  "kernel": cci.kernel_name(torch.bfloat16, c.Cin, c.R, c.Cout, c.G, c.K,
+                                                            cci.ALGO_DENSE_TC_WS)})
         nzf = sum(c.nz_flops() for c in layers)
         dense_f = sum(c.dense_flops() for c in layers)
         floor_ms = sum(layer_floor_us(c) for c in layers) * 1e-3
@@ -664,6 +716,8 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
                     "roofline_floor_ms": floor_ms, "roofline_frac": floor_ms / ms,
                     "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
                     "captured": "CUDA graph of the 52 calls (ours) / 52 cuDNN convolutions (dense)"})
+        if per_layer:
+            res[-1]["per_layer"] = per_layer
         del keep, ours_calls, dense_calls, g_ours, g_dense
         torch.cuda.empty_cache()
     return res

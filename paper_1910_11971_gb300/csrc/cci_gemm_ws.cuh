@@ -26,8 +26,11 @@
 // for kA4d, 4-D over Y[B][P][Q][Cout] with the tile's pixel box.
 // Roles: warps 0-3 epilogue (TMEM lanes), warps 4-7 producers of the activation
 // planes that are not copied by TMA, warp 8 allocates TMEM and issues the MMAs,
-// warp 9 issues the TMA copies as soon as a stage is free (so copy latency
-// overlaps the producers' work).  Every mbarrier wait is bounded
+// warps 9.. issue the TMA copies as soon as a stage is free (so copy latency
+// overlaps the producers' work), stage by stage in turn: the copies one thread
+// issues are processed one box after another (measured on GB300: about 0.5 us
+// per box of 16-64 KB from one issuer; copy throughput grows with the number of
+// issuing warps), so up to four warps issue.  Every mbarrier wait is bounded
 // (CCI_ERR_TIMEOUT, abort flag, drain, TMEM freed).
 #pragma once
 
@@ -49,6 +52,13 @@ struct ConvBox {
     int nQ, nP;      // boxes along q and p (the batch index is the rest)
     int rows;        // QB * PB * BB
     int64_t B;       // batch size
+};
+
+// activation tensor maps: [0] for products (2-D over X[N][Cin]); for a
+// convolution with strides (sh, sw) <= 2, map [rh * sw + rw] covers the input
+// pixels (h, w) = (rh + sh * h', rw + sw * w'), a 4-D tensor over (ci, w', h', b)
+struct AMaps {
+    CUtensorMap m[4];
 };
 
 template <bool TF32, int ASRC, int BN>
@@ -75,6 +85,13 @@ struct Cfg {
     static_assert(kSmem <= kMaxSmemPerBlock, "stage buffers over the per-block limit");
     static_assert(kStages >= 3, "too few pipeline stages");
     static_assert(kTmemCols == 128 || kTmemCols == 256 || kTmemCols == 512, "TMEM allocation not a power of 2");
+    // warps issuing the TMA copies, stage `it` by warp 9 + it % kIssuers: one
+    // thread's copies are processed one box at a time, so several issuers keep
+    // more boxes moving.  kIssuers <= kStages keeps every empty-barrier wait
+    // within one phase of the barrier (no parity aliasing).
+    static constexpr int kIssuers = ASRC == kAGather ? 1 : (kStages < 4 ? kStages : 4);
+    static constexpr int kThreads = 32 * (9 + kIssuers);
+    static_assert(kIssuers >= 1 && kIssuers <= kStages, "issuers must not outnumber the stages");
 };
 
 template <bool TF32>
@@ -111,7 +128,6 @@ __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
     return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
 }
 
-constexpr int kThreads = 320;
 
 // (box along q, box along p, batch box) of M tile mt
 struct BoxIdx {
@@ -129,8 +145,8 @@ __device__ __forceinline__ BoxIdx box_of(int64_t mt, const ConvBox &box)
 }
 
 template <bool TF32, int ASRC, int BN>
-__global__ void __launch_bounds__(kThreads, 1)
-    gemm_ws_kernel(FwdParams p, const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB0,
+__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
+    gemm_ws_kernel(FwdParams p, const __grid_constant__ AMaps tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmY, ConvBox box,
                    int64_t n_ct, int64_t n_tiles)
 {
@@ -163,7 +179,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (ASRC == kA4d && box.rows < kM) {
         // rows past the box are never copied: keep them zero for the MMAs
         for (uint32_t o = static_cast<uint32_t>(tid) * 16; o < static_cast<uint32_t>(kStages * C::kStage);
-             o += kThreads * 16)
+             o += C::kThreads * 16)
             tc::st_shared_v4_zero(base + o);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
@@ -175,7 +191,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
     if (tid == 288) {
-        if constexpr (ASRC != kAGather) tc::tma_prefetch_desc(&tmA);
+        if constexpr (ASRC == kA2d) tc::tma_prefetch_desc(&tmA.m[0]);
+        if constexpr (ASRC == kA4d)
+            for (int i = 0; i < p.sh * p.sw; ++i) tc::tma_prefetch_desc(&tmA.m[i]);
         tc::tma_prefetch_desc(&tmB0);
         if constexpr (C::kBPlanes > 1) tc::tma_prefetch_desc(&tmB1);
         tc::tma_prefetch_desc(&tmY);
@@ -185,10 +203,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = S->tmem_base;
 
-    if (warp == 9) {
-        // ------------------------------------------------------------ TMA issuer
+    if (warp >= 9) {
+        // ------------------------------------------------------------ TMA issuers
         const uint32_t a_bytes = ASRC == kA4d ? static_cast<uint32_t>(box.rows) * 128u : C::kAPlane;
         const int cpt = static_cast<int>(p.Cin / kKS);  // stages per tap (kA4d)
+        const int issuer = warp - 9;
         int it = 0;
         bool ok = true;
         for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
@@ -197,6 +216,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d) bi = box_of(mt, box);
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
+                if (it % C::kIssuers != issuer) continue;
                 const int s = it % kStages;
                 if (it >= kStages) ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
                 if (!ok) break;
@@ -211,12 +231,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if constexpr (C::kBPlanes > 1)
                         tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * kKS, static_cast<int>(co0), &S->full[s]);
                     if constexpr (ASRC == kA2d) {
-                        tc::tma_load_2d(st, &tmA, ks * kKS, static_cast<int>(mt * kM), abar);
+                        tc::tma_load_2d(st, &tmA.m[0], ks * kKS, static_cast<int>(mt * kM), abar);
                     } else if constexpr (ASRC == kA4d) {
                         const int tap = ks / cpt;
                         const int ci0 = (ks - tap * cpt) * kKS;
                         const int kh = tap / p.KW, kw = tap - (tap / p.KW) * p.KW;
-                        tc::tma_load_4d(st, &tmA, ci0, bi.qb * box.QB - p.pw + kw, bi.pb * box.PB - p.ph + kh,
+                        // input row h = p_out * sh + ah lies on lattice rh at h' = p_out + dh
+                        const int ah = kh - p.ph, aw = kw - p.pw;
+                        const int rh = ((ah % p.sh) + p.sh) % p.sh, rw = ((aw % p.sw) + p.sw) % p.sw;
+                        const int dh = (ah - rh) / p.sh, dw = (aw - rw) / p.sw;
+                        tc::tma_load_4d(st, &tmA.m[rh * p.sw + rw], ci0, bi.qb * box.QB + dw, bi.pb * box.PB + dh,
                                         static_cast<int>(bi.bb * box.BB), abar);
                     }
                 }
@@ -512,26 +536,62 @@ inline PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-// map over a row-major array of `rank` dims (dims[0] innermost, element count
-// each), box[] elements per dim, 128-byte swizzle (box[0] * elem must be 128)
-inline bool make_map(CUtensorMap *m, const void *ptr, CUtensorMapDataType dt, int elem, int rank,
-                     const int64_t *dims, const int *box)
+// map over `rank` dims (dims[0] innermost, element counts) with byte strides
+// strides[i] of dims 1.., box[] elements per dim, 128-byte swizzle (box[0] * elem
+// must be 128); false if the driver rejects it
+inline bool make_map_strided(CUtensorMap *m, const void *ptr, CUtensorMapDataType dt, int rank,
+                             const int64_t *dims, const int64_t *strides, const int *box)
 {
     auto fn = encode_fn();
     if (!fn || rank < 1 || rank > 5) return false;
     cuuint64_t gd[5], gs[4];
     cuuint32_t bx[5], es[5];
-    uint64_t stride = static_cast<uint64_t>(elem);
     for (int i = 0; i < rank; ++i) {
+        if (dims[i] < 1) return false;
         gd[i] = static_cast<cuuint64_t>(dims[i]);
         bx[i] = static_cast<cuuint32_t>(box[i]);
         es[i] = 1;
-        if (i > 0) gs[i - 1] = static_cast<cuuint64_t>(stride);
-        stride *= static_cast<uint64_t>(dims[i]);
+        if (i > 0) gs[i - 1] = static_cast<cuuint64_t>(strides[i - 1]);
     }
     return fn(m, dt, static_cast<cuuint32_t>(rank), const_cast<void *>(ptr), gd, gs, bx, es,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// the same over a packed row-major array
+inline bool make_map(CUtensorMap *m, const void *ptr, CUtensorMapDataType dt, int elem, int rank,
+                     const int64_t *dims, const int *box)
+{
+    int64_t strides[4];
+    int64_t s = elem;
+    for (int i = 0; i + 1 < rank && i < 4; ++i) {
+        s *= dims[i];
+        strides[i] = s;
+    }
+    return make_map_strided(m, ptr, dt, rank, dims, strides, box);
+}
+
+// activation maps of the layer for source asrc (stage depth ks elements); false
+// if a map cannot be encoded
+inline bool build_a_maps(const FwdParams &p, const ConvBox &box, int asrc, bool tf32, int ks, AMaps *am)
+{
+    const CUtensorMapDataType dt = tf32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const int64_t e = tf32 ? 4 : 2;
+    if (asrc == kA2d) {
+        const int64_t dims[2] = {p.Cin, p.N};
+        const int bx[2] = {ks, 128};
+        return make_map(&am->m[0], p.X, dt, static_cast<int>(e), 2, dims, bx);
+    }
+    if (asrc != kA4d) return true;
+    for (int rh = 0; rh < p.sh; ++rh)
+        for (int rw = 0; rw < p.sw; ++rw) {
+            const char *base = static_cast<const char *>(p.X) + (rh * p.W + rw) * p.Cin * e;
+            const int64_t dims[4] = {p.Cin, (p.W - rw + p.sw - 1) / p.sw, (p.H - rh + p.sh - 1) / p.sh, box.B};
+            const int64_t strides[3] = {p.sw * p.Cin * e, p.sh * p.W * p.Cin * e, p.H * p.W * p.Cin * e};
+            const int bx[4] = {ks, box.QB, box.PB, box.BB};
+            if (!make_map_strided(&am->m[rh * p.sw + rw], base, dt, 4, dims, strides, bx)) return false;
+        }
+    return true;
 }
 
 inline int sm_count()
@@ -577,7 +637,8 @@ inline int a_source(const FwdParams &p, int ks)
     const int64_t lim = int64_t(1) << 30;
     if (!p.is_conv) return p.N < lim ? kA2d : kAGather;
     const bool fits = p.H < lim && p.W < lim && p.N < lim && (p.N / (p.P * p.Q)) < lim;
-    return (p.sh == 1 && p.sw == 1 && p.Cin % ks == 0 && fits) ? kA4d : kAGather;
+    const bool strides_ok = p.sh >= 1 && p.sh <= 2 && p.sw >= 1 && p.sw <= 2 && p.H >= p.sh && p.W >= p.sw;
+    return (strides_ok && p.Cin % ks == 0 && fits) ? kA4d : kAGather;
 }
 
 // N tile among {64, 128, 256} (up to max_bn): fewest rounds of tiles over the
@@ -599,25 +660,16 @@ inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn)
 }
 
 template <bool TF32, int ASRC, int BN>
-cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, cudaStream_t stream)
+cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA, cudaStream_t stream)
 {
     using C = Cfg<TF32, ASRC, BN>;
     auto kern = gemm_ws_kernel<TF32, ASRC, BN>;
     static const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::kSmem));
     if (attr != cudaSuccess) return attr;
-    CUtensorMap tmA{}, tmB0{}, tmB1{}, tmY{};
+    CUtensorMap tmB0{}, tmB1{}, tmY{};
     const CUtensorMapDataType dt = TF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     const int elem = TF32 ? 4 : 2;
-    if constexpr (ASRC == kA2d) {
-        const int64_t dims[2] = {p.Cin, p.N};
-        const int bx[2] = {C::kKS, C::kM};
-        if (!make_map(&tmA, p.X, dt, elem, 2, dims, bx)) return cudaErrorInvalidValue;
-    } else if constexpr (ASRC == kA4d) {
-        const int64_t dims[4] = {p.Cin, p.W, p.H, box.B};
-        const int bx[4] = {C::kKS, box.QB, box.PB, box.BB};
-        if (!make_map(&tmA, p.X, dt, elem, 4, dims, bx)) return cudaErrorInvalidValue;
-    }
     const int64_t wdims[2] = {p.R, p.Cout};
     const int wbox[2] = {C::kKS, C::kN};
     if (!make_map(&tmB0, p.wdense, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
@@ -640,8 +692,26 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, cudaStream_t stre
     const int64_t n_tiles = n_ct * m_tiles;
     const int64_t sms = sm_count();
     const int64_t grid = n_tiles < sms ? n_tiles : sms;
-    kern<<<static_cast<unsigned>(grid), kThreads, C::kSmem, stream>>>(p, tmA, tmB0, tmB1, tmY, box, n_ct, n_tiles);
+    kern<<<static_cast<unsigned>(grid), C::kThreads, C::kSmem, stream>>>(p, tmA, tmB0, tmB1, tmY, box, n_ct, n_tiles);
     return cudaGetLastError();
+}
+
+// activation source, pixel box and activation maps of a layer (stage depth ks):
+// the 4-D copy when the layer allows it and its maps encode, else the gather
+struct Plan {
+    int asrc;
+    ConvBox box;
+    AMaps am;
+};
+inline void plan_layer(const FwdParams &p, bool tf32, int ks, Plan *pl)
+{
+    pl->asrc = a_source(p, ks);
+    pl->box = ConvBox{1, 1, 1, 1, 1, 1, 1};
+    if (pl->asrc == kA4d) pl->box = choose_box(p.N / (p.P * p.Q), p.P, p.Q);
+    if (!build_a_maps(p, pl->box, pl->asrc, tf32, ks, &pl->am)) {
+        pl->asrc = kAGather;
+        pl->box = ConvBox{1, 1, 1, 1, 1, 1, 1};
+    }
 }
 
 // m tiles of the layer for the chosen activation source

@@ -7,12 +7,12 @@ namespace cci {
 cudaError_t launch_gemm_ws_tf32(const FwdParams &p, cudaStream_t stream)
 {
     using namespace ws;
-    const int asrc = a_source(p, 32);
-    ConvBox box{1, 1, 1, 1, 1, 1, 1};
-    if (asrc == kA4d) box = choose_box(p.N / (p.P * p.Q), p.P, p.Q);
-    const int bn = choose_bn(m_tiles_of(p, asrc, box), p.Cout, 128);
+    Plan pl;
+    plan_layer(p, true, 32, &pl);
+    const int asrc = pl.asrc;
+    const int bn = choose_bn(m_tiles_of(p, asrc, pl.box), p.Cout, 128);
 #define CCI_WS_CASE(A, N) \
-    if (asrc == A && bn == N) return launch_cfg<true, A, N>(p, box, stream);
+    if (asrc == A && bn == N) return launch_cfg<true, A, N>(p, pl.box, pl.am, stream);
     CCI_WS_CASE(kA2d, 64)
     CCI_WS_CASE(kA2d, 128)
     CCI_WS_CASE(kA4d, 64)

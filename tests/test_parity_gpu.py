@@ -481,7 +481,7 @@ def test_tf32x3_conv_small(dev, case):
 
 
 # ---------------------------------------------------------------------------
-# convolutions whose activations are copied by 4-D TMA (unit stride, Cin a
+# convolutions whose activations are copied by 4-D TMA (strides 1 or 2, Cin a
 # multiple of 64 for bf16 / 32 for fp32): output-pixel boxes with ragged edges,
 # asymmetric padding, windows wholly inside the padding, every N tile width
 # ---------------------------------------------------------------------------
@@ -497,6 +497,16 @@ CONV_TMA = [
     (2, 9, 7, 32, 64, 3, 3, (1, 1), (1, 1), 8, 2, "f32"),
     (3, 5, 6, 64, 96, 3, 3, (1, 1), (1, 1), 16, 4, "f32"),
     (2, 4, 4, 32, 32, 3, 3, (1, 1), (3, 3), 4, 1, "f32"),
+    # strides 2: one copy map per parity lattice of the input
+    (2, 9, 7, 64, 64, 3, 3, (2, 2), (1, 1), 8, 2, "bf16"),
+    (3, 8, 10, 64, 128, 1, 1, (2, 2), (0, 0), 8, 2, "bf16"),
+    (2, 7, 6, 128, 64, 3, 3, (2, 1), (1, 0), 16, 4, "bf16"),
+    (1, 5, 5, 64, 32, 5, 5, (2, 2), (2, 2), 4, 1, "bf16"),
+    (2, 2, 3, 64, 64, 3, 3, (2, 2), (1, 1), 8, 2, "bf16"),
+    (2, 9, 7, 32, 64, 3, 3, (2, 2), (1, 1), 8, 2, "f32"),
+    (2, 6, 6, 32, 32, 1, 1, (2, 2), (0, 0), 4, 2, "f32"),
+    # stride 3: the row gather
+    (1, 10, 10, 64, 64, 3, 3, (3, 3), (1, 1), 8, 2, "bf16"),
 ]
 
 
