@@ -19,8 +19,10 @@
 //               zero padding is the copy's out-of-range fill;
 //     kAGather  other convolutions: the producer warps gather rows (cp.async for
 //               bf16; registers, two stages ahead, then the hi/lo split, for fp32).
-//   fp32 activations copied by TMA land raw in the hi plane and the producer warps
-//   split them in place.
+//   fp32 activations copied by TMA land raw in shared memory; the producer warps
+//   split each row into hi and lo and store both in tensor memory (per stage 64
+//   columns after the accumulators), from where the MMAs read A: the three
+//   passes then read only B from shared memory.
 // Output: fp32 Y written by TMA stores from a swizzled staging buffer (two
 // alternating 16 KB buffers of [128 rows][32 columns]), 2-D over Y[N][Cout] or,
 // for kA4d, 4-D over Y[B][P][Q][Cout] with the tile's pixel box.
@@ -65,16 +67,20 @@ template <bool TF32, int ASRC, int BN>
 struct Cfg {
     static constexpr int kM = 128, kN = BN;
     static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
-    static constexpr int kAPlanes = TF32 ? 2 : 1, kBPlanes = TF32 ? 2 : 1;
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
-    static constexpr bool kARaw = TF32 && ASRC != kAGather;   // raw fp32 A by TMA, split by the producers
+    // raw fp32 A by TMA; the producers split it into hi / lo and write both to
+    // tensor memory, where the MMAs read A (no A planes in shared memory)
+    static constexpr bool kARaw = TF32 && ASRC != kAGather;
+    static constexpr int kAPlanes = (TF32 && !kARaw) ? 2 : 1, kBPlanes = TF32 ? 2 : 1;
     static constexpr int kAPlane = kM * 128;                    // bytes: 128-byte rows
     static constexpr int kBPlane = kN * 128;
     static constexpr int kStage = kAPlanes * kAPlane + kBPlanes * kBPlane;
     static constexpr int kYBuf = kM * 128;  // one output staging buffer: [128 rows][32 fp32]
     static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - 2 * kYBuf - 1024;
     static constexpr int kStages = (kBudget / kStage) < tc::kMaxStages ? (kBudget / kStage) : tc::kMaxStages;
-    static constexpr int kTmemCols = 2 * kN;
+    // accumulators: 2 x kN columns; kARaw adds per stage A hi and A lo (32 columns each)
+    static constexpr int kAColBase = 2 * kN;
+    static constexpr int kTmemCols = kARaw ? 512 : 2 * kN;
     static constexpr size_t kSmem =
         1024 + static_cast<size_t>(kStages) * kStage + 2 * kYBuf + sizeof(tc::Smem) + 64;
     static constexpr uint32_t kBBytes = kBPlanes * kBPlane;
@@ -85,6 +91,7 @@ struct Cfg {
     static_assert(kSmem <= kMaxSmemPerBlock, "stage buffers over the per-block limit");
     static_assert(kStages >= 3, "too few pipeline stages");
     static_assert(kTmemCols == 128 || kTmemCols == 256 || kTmemCols == 512, "TMEM allocation not a power of 2");
+    static_assert(!kARaw || kAColBase + kStages * 64 <= 512, "A stages do not fit in tensor memory");
     // warps issuing the TMA copies, stage `it` by warp 9 + it % kIssuers: one
     // thread's copies are processed one box at a time, so several issuers keep
     // more boxes moving.  kIssuers <= kStages keeps every empty-barrier wait
@@ -110,6 +117,16 @@ __device__ __forceinline__ void mma(uint32_t d, uint64_t a, uint64_t b, uint32_t
             "l"(a), "l"(b), "r"(idesc), "r"(acc)
             : "memory");
     }
+}
+
+// tf32 MMA with A read from tensor memory (lane = row m, one column per k)
+__device__ __forceinline__ void mma_tf32_ta(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
+{
+    asm volatile(
+        "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
 }
 
 // byte offset of (row, 16-byte chunk) in a plane of 128-byte rows, 128-byte swizzle
@@ -370,22 +387,35 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
                             tc::mbar_arrive(&S->full[(it - kLag) % kStages]);
                         }
                     } else if constexpr (C::kARaw) {
-                        // the raw fp32 tile landed in the hi plane: split it in place
+                        // the raw fp32 tile landed: row m = pt, split into hi and lo in
+                        // registers and written to this stage's A columns of tensor
+                        // memory (lane m; warp 4 + q owns lanes 32q..32q+31)
                         ok = tc::mbar_wait(&S->aux[s], (it / kStages) & 1, abort, p.status);
+                        ok = __all_sync(0xffffffffu, ok);
                         if (!ok) break;
+                        uint32_t hv[32], lv[32];
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            const uint32_t o = sw_chunk(rowb + 16 * i, chunk);
+                        for (int q = 0; q < 8; ++q) {
                             uint4 v;
                             asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
                                          : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                                         : "r"(st + o)
+                                         : "r"(st + sw_chunk(pt, q))
                                          : "memory");
-                            st_shared_v4(st + o, hi_bits(v.x), hi_bits(v.y), hi_bits(v.z), hi_bits(v.w));
-                            st_shared_v4(st + C::kAPlane + o, lo_bits(v.x), lo_bits(v.y), lo_bits(v.z),
-                                         lo_bits(v.w));
+                            hv[4 * q] = hi_bits(v.x);
+                            hv[4 * q + 1] = hi_bits(v.y);
+                            hv[4 * q + 2] = hi_bits(v.z);
+                            hv[4 * q + 3] = hi_bits(v.w);
+                            lv[4 * q] = lo_bits(v.x);
+                            lv[4 * q + 1] = lo_bits(v.y);
+                            lv[4 * q + 2] = lo_bits(v.z);
+                            lv[4 * q + 3] = lo_bits(v.w);
                         }
-                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        const uint32_t ta = tmem + (static_cast<uint32_t>((warp - 4) * 32) << 16) +
+                                            static_cast<uint32_t>(C::kAColBase + s * 64);
+                        tc::tmem_st32(ta, hv);
+                        tc::tmem_st32(ta + 32, lv);
+                        asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+                        asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                         tc::mbar_arrive(&S->full[s]);
                     } else {
 #pragma unroll
@@ -431,7 +461,18 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
                 if (lane == 0) {
                     const uint32_t st = base + s * C::kStage;
                     const uint32_t bst = st + C::kAPlanes * C::kAPlane;
-                    if constexpr (TF32) {
+                    if constexpr (C::kARaw) {
+#pragma unroll
+                        for (int k = 0; k < kKS / 8; ++k) {
+                            const uint32_t ah = tmem + static_cast<uint32_t>(C::kAColBase + s * 64 + k * 8);
+                            const uint32_t al = ah + 32;
+                            const uint64_t bh = tc::sw128_desc(bst + k * 32);
+                            const uint64_t bl = tc::sw128_desc(bst + C::kBPlane + k * 32);
+                            mma_tf32_ta(d, al, bh, C::kIdesc, (ks > 0 || k > 0) ? 1u : 0u);
+                            mma_tf32_ta(d, ah, bl, C::kIdesc, 1u);
+                            mma_tf32_ta(d, ah, bh, C::kIdesc, 1u);
+                        }
+                    } else if constexpr (TF32) {
 #pragma unroll
                         for (int k = 0; k < kKS / 8; ++k) {
                             const uint64_t ah = tc::sw128_desc(st + k * 32);
