@@ -334,6 +334,9 @@ __global__ void __launch_bounds__(kSlab) decompress_kernel(const T *__restrict__
 {
     constexpr int V = 16 / static_cast<int>(sizeof(T));  // elements per 16-byte store
     __shared__ __align__(16) T tile[G][kSlab];
+    // the workspace GEMM that follows may start its prologue now; it waits for
+    // this grid's completion before reading the workspace
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int64_t gi = blockIdx.x / slabs;
     const int64_t r0 = (blockIdx.x - gi * slabs) * kSlab;
     for (int e = threadIdx.x; e < G * kSlab / V; e += kSlab)

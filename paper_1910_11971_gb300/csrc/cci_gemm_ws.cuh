@@ -219,6 +219,10 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = S->tmem_base;
+    // launched as a programmatic dependent of the decompression: everything above
+    // overlaps its tail; the workspace (and anything else in memory) is read only
+    // after that grid has completed and its writes are visible
+    asm volatile("griddepcontrol.wait;" ::: "memory");
 
     if (warp >= 9) {
         // ------------------------------------------------------------ TMA issuers
@@ -733,8 +737,21 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
     const int64_t n_tiles = n_ct * m_tiles;
     const int64_t sms = sm_count();
     const int64_t grid = n_tiles < sms ? n_tiles : sms;
-    kern<<<static_cast<unsigned>(grid), C::kThreads, C::kSmem, stream>>>(p, tmA, tmB0, tmB1, tmY, box, n_ct, n_tiles);
-    return cudaGetLastError();
+    // programmatic dependent launch: may start once every block of the preceding
+    // kernel on the stream (the decompression) has signalled; it waits for that
+    // kernel's completion before reading memory
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(C::kThreads);
+    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.stream = stream;
+    cudaLaunchAttribute la[1];
+    la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    la[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = la;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p, tmA, tmB0, tmB1, tmY, box, n_ct, n_tiles);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 // activation source, pixel box and activation maps of a layer (stage depth ks):
