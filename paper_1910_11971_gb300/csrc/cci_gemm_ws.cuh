@@ -63,9 +63,14 @@ struct AMaps {
     CUtensorMap m[4];
 };
 
-template <bool TF32, int ASRC, int BN>
+// CG = 2: a cluster of two CTAs computes a 256 x BN tile with tcgen05.mma
+// cta_group::2 issued by the even CTA; each CTA holds its 128 rows of A and half
+// of the BN rows of B (bf16 with TMA activations only)
+template <bool TF32, int ASRC, int BN, int CG>
 struct Cfg {
     static constexpr int kM = 128, kN = BN;
+    static_assert(CG == 1 || (CG == 2 && !TF32 && ASRC != kAGather), "pair mode: bf16 with TMA activations");
+    static constexpr int kBRows = kN / CG;  // B rows held by one CTA
     static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
     // raw fp32 A by TMA; the producers split it into hi / lo and write both to
@@ -73,7 +78,7 @@ struct Cfg {
     static constexpr bool kARaw = TF32 && ASRC != kAGather;
     static constexpr int kAPlanes = (TF32 && !kARaw) ? 2 : 1, kBPlanes = TF32 ? 2 : 1;
     static constexpr int kAPlane = kM * 128;                    // bytes: 128-byte rows
-    static constexpr int kBPlane = kN * 128;
+    static constexpr int kBPlane = kBRows * 128;
     static constexpr int kStage = kAPlanes * kAPlane + kBPlanes * kBPlane;
     static constexpr int kYBuf = kM * 128;  // one output staging buffer: [128 rows][32 fp32]
     static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - 2 * kYBuf - 1024;
@@ -87,7 +92,7 @@ struct Cfg {
     static constexpr uint32_t kIdesc = (1u << 4)                                           // D f32
                                        | (TF32 ? (2u << 7) | (2u << 10) : (1u << 7) | (1u << 10))  // tf32 / bf16
                                        | (static_cast<uint32_t>(kN >> 3) << 17) |
-                                       (static_cast<uint32_t>(kM >> 4) << 24);
+                                       (static_cast<uint32_t>((kM * CG) >> 4) << 24);
     static_assert(kSmem <= kMaxSmemPerBlock, "stage buffers over the per-block limit");
     static_assert(kStages >= 3, "too few pipeline stages");
     static_assert(kTmemCols == 128 || kTmemCols == 256 || kTmemCols == 512, "TMEM allocation not a power of 2");
@@ -101,10 +106,16 @@ struct Cfg {
     static_assert(kIssuers >= 1 && kIssuers <= kStages, "issuers must not outnumber the stages");
 };
 
-template <bool TF32>
+template <bool TF32, int CG>
 __device__ __forceinline__ void mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc)
 {
-    if constexpr (TF32) {
+    if constexpr (CG == 2) {
+        asm volatile(
+            "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+            "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+            "l"(a), "l"(b), "r"(idesc), "r"(acc)
+            : "memory");
+    } else if constexpr (TF32) {
         asm volatile(
             "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
             "tcgen05.mma.cta_group::1.kind::tf32 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
@@ -126,6 +137,63 @@ __device__ __forceinline__ void mma_tf32_ta(uint32_t d, uint32_t a_tmem, uint64_
         "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
         "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
         "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
+// ---- cluster-pair helpers (CG = 2) ----
+__device__ __forceinline__ uint32_t cluster_rank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// shared::cluster address of the same shared variable in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t local, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_sync()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr)
+{
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// tcgen05.commit of the pair's MMAs, arriving on the barrier at this offset in both CTAs
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar)
+{
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            tc::smem_u32(bar)),
+        "h"(static_cast<uint16_t>(3))
+        : "memory");
+}
+
+// TMA loads of either CTA of the pair completing on the even CTA's barrier
+// (cluster address)
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void *tmap, int x, int y, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, "
+        "{%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d_pair(uint32_t dst, const void *tmap, int c0, int c1, int c2, int c3,
+                                                 uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, "
+        "{%2, %3, %4, %5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
         : "memory");
 }
 
@@ -161,13 +229,13 @@ __device__ __forceinline__ BoxIdx box_of(int64_t mt, const ConvBox &box)
     return i;
 }
 
-template <bool TF32, int ASRC, int BN>
-__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
+template <bool TF32, int ASRC, int BN, int CG>
+__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
     gemm_ws_kernel(FwdParams p, const __grid_constant__ AMaps tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmY, ConvBox box,
                    int64_t n_ct, int64_t n_tiles)
 {
-    using C = Cfg<TF32, ASRC, BN>;
+    using C = Cfg<TF32, ASRC, BN, CG>;
     constexpr int kM = C::kM, kN = C::kN, kKS = C::kKS, kStages = C::kStages;
     constexpr int kLag = 2;  // bf16 gather: stages in flight before a producer's arrive
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -178,6 +246,12 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
     volatile int *abort = &S->abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nks = static_cast<int>((p.R + kKS - 1) / kKS);
+    const uint32_t crank = CG == 2 ? cluster_rank() : 0u;  // 0: issues the pair's MMAs
+    // work units: tiles (CG = 1) or pair tiles of 2 x 128 rows (CG = 2), strided over
+    // the CTAs (CG = 1) or the CTA pairs (CG = 2)
+    const int64_t u0 = CG == 2 ? blockIdx.x / 2 : blockIdx.x;
+    const int64_t ustep = CG == 2 ? gridDim.x / 2 : gridDim.x;
+    auto mtile = [&](int64_t u) -> int64_t { return CG == 2 ? 2 * (u / n_ct) + crank : u / n_ct; };
 
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -187,7 +261,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             tc::mbar_init(&S->tmem_full[a], 1);
-            tc::mbar_init(&S->tmem_empty[a], 128);
+            tc::mbar_init(&S->tmem_empty[a], 128 * CG);
         }
         tc::mbar_init(&S->drain, 1);
         S->abort = 0;
@@ -201,11 +275,19 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
     }
     if (warp == 8) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         tc::smem_u32(&S->tmem_base)),
-                     "r"(C::kTmemCols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        if constexpr (CG == 2) {  // one warp of each CTA of the pair, collectively
+            asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             tc::smem_u32(&S->tmem_base)),
+                         "r"(C::kTmemCols)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+        } else {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             tc::smem_u32(&S->tmem_base)),
+                         "r"(C::kTmemCols)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        }
     }
     if (tid == 288) {
         if constexpr (ASRC == kA2d) tc::tma_prefetch_desc(&tmA.m[0]);
@@ -217,6 +299,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    // the pair's barriers are initialised before either CTA signals the other's
+    if constexpr (CG == 2) cluster_sync();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = S->tmem_base;
     // launched as a programmatic dependent of the decompression: everything above
@@ -231,9 +315,9 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
         const int issuer = warp - 9;
         int it = 0;
         bool ok = true;
-        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
-            const int64_t mt = tile / n_ct;
-            const int64_t co0 = (tile % n_ct) * kN;
+        for (int64_t u = u0; u < n_tiles && ok; u += ustep) {
+            const int64_t mt = mtile(u);
+            const int64_t co0 = (u % n_ct) * kN + crank * C::kBRows;  // this CTA's B rows
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d) bi = box_of(mt, box);
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
@@ -241,7 +325,27 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
                 const int s = it % kStages;
                 if (it >= kStages) ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
                 if (!ok) break;
-                if (lane == 0) {
+                if (lane == 0 && CG == 2) {
+                    // both CTAs' copies complete on the even CTA's full barrier, which
+                    // expects the bytes of the pair
+                    const uint32_t st = base + s * C::kStage;
+                    const uint32_t bst = st + C::kAPlane;
+                    const uint32_t fb = map_to_rank(tc::smem_u32(&S->full[s]), 0);
+                    if (crank == 0) tc::mbar_arrive_expect_tx(&S->full[s], 2 * (C::kBBytes + a_bytes));
+                    tma_load_2d_pair(bst, &tmB0, ks * kKS, static_cast<int>(co0), fb);
+                    if constexpr (ASRC == kA2d) {
+                        tma_load_2d_pair(st, &tmA.m[0], ks * kKS, static_cast<int>(mt * kM), fb);
+                    } else {
+                        const int tap = ks / cpt;
+                        const int ci0 = (ks - tap * cpt) * kKS;
+                        const int kh = tap / p.KW, kw = tap - (tap / p.KW) * p.KW;
+                        const int ah = kh - p.ph, aw = kw - p.pw;
+                        const int rh = ((ah % p.sh) + p.sh) % p.sh, rw = ((aw % p.sw) + p.sw) % p.sw;
+                        const int dh = (ah - rh) / p.sh, dw = (aw - rw) / p.sw;
+                        tma_load_4d_pair(st, &tmA.m[rh * p.sw + rw], ci0, bi.qb * box.QB + dw,
+                                         bi.pb * box.PB + dh, static_cast<int>(bi.bb * box.BB), fb);
+                    }
+                } else if (lane == 0) {
                     const uint32_t st = base + s * C::kStage;
                     const uint32_t bst = st + C::kAPlanes * C::kAPlane;
                     // the activation copy completes on aux (raw fp32, split afterwards) or full
@@ -449,9 +553,17 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
         }
     } else if (warp == 8) {
         // ------------------------------------------------------------ MMA issuer
+        // (CG = 2: the even CTA issues for the pair; the odd CTA only waits for
+        // the drain)
         int it = 0, t = 0;
-        bool ok = true;
-        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+        bool ok = CG == 1 || crank == 0;
+        auto commit = [&](uint64_t *bar) {
+            if constexpr (CG == 2)
+                mma_commit_pair(bar);
+            else
+                tc::mma_commit(bar);
+        };
+        for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
             const int acc = t & 1;
             if (t >= 2) ok = tc::mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
             if (!ok) break;
@@ -483,24 +595,24 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
                             const uint64_t al = tc::sw128_desc(st + C::kAPlane + k * 32);
                             const uint64_t bh = tc::sw128_desc(bst + k * 32);
                             const uint64_t bl = tc::sw128_desc(bst + C::kBPlane + k * 32);
-                            mma<TF32>(d, al, bh, C::kIdesc, (ks > 0 || k > 0) ? 1u : 0u);
-                            mma<TF32>(d, ah, bl, C::kIdesc, 1u);
-                            mma<TF32>(d, ah, bh, C::kIdesc, 1u);
+                            mma<TF32, CG>(d, al, bh, C::kIdesc, (ks > 0 || k > 0) ? 1u : 0u);
+                            mma<TF32, CG>(d, ah, bl, C::kIdesc, 1u);
+                            mma<TF32, CG>(d, ah, bh, C::kIdesc, 1u);
                         }
                     } else {
 #pragma unroll
                         for (int k = 0; k < kKS / 16; ++k)
-                            mma<TF32>(d, tc::sw128_desc(st + k * 32), tc::sw128_desc(bst + k * 32), C::kIdesc,
-                                      (ks > 0 || k > 0) ? 1u : 0u);
+                            mma<TF32, CG>(d, tc::sw128_desc(st + k * 32), tc::sw128_desc(bst + k * 32), C::kIdesc,
+                                          (ks > 0 || k > 0) ? 1u : 0u);
                     }
-                    tc::mma_commit(&S->empty[s]);
+                    commit(&S->empty[s]);
                 }
                 __syncwarp();
             }
-            if (ok && lane == 0) tc::mma_commit(&S->tmem_full[acc]);
+            if (ok && lane == 0) commit(&S->tmem_full[acc]);
             __syncwarp();
         }
-        if (lane == 0) tc::mma_commit(&S->drain);
+        if (lane == 0 && (CG == 1 || crank == 0)) commit(&S->drain);
         __syncwarp();
         int no_abort = 0;
         tc::mbar_wait(&S->drain, 0, &no_abort, p.status);
@@ -517,10 +629,12 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
         const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
         const int m = tid;  // accumulator row = TMEM lane
         int chunk_no = 0;
-        for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x, ++t) {
+        // CG = 2: the odd CTA releases an accumulator on the even CTA's barrier
+        const uint32_t tmem_empty_remote = CG == 2 ? map_to_rank(tc::smem_u32(&S->tmem_empty[0]), 0) : 0u;
+        for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
             const int acc = t & 1;
-            const int64_t mt = tile / n_ct;
-            const int co0 = static_cast<int>((tile % n_ct) * kN);
+            const int64_t mt = mtile(u);
+            const int co0 = static_cast<int>((u % n_ct) * kN);
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d) bi = box_of(mt, box);
             ok = tc::mbar_wait(&S->tmem_full[acc], (t / 2) & 1, abort, p.status);
@@ -550,17 +664,27 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN>::kThreads, 1)
                 }
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            tc::mbar_arrive(&S->tmem_empty[acc]);
+            if (CG == 2 && crank != 0)
+                mbar_arrive_remote(tmem_empty_remote + static_cast<uint32_t>(acc * sizeof(uint64_t)));
+            else
+                tc::mbar_arrive(&S->tmem_empty[acc]);
         }
         if (tid == 0) tc::bulk_wait_all();
     }
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    // CG = 2: neither CTA leaves (or frees tensor memory) while the other may still
+    // signal its barriers or the pair's MMAs may read its shared memory
+    if constexpr (CG == 2) cluster_sync();
     if (warp == 8) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::kTmemCols)
-                     : "memory");
+        if constexpr (CG == 2)
+            asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::kTmemCols)
+                         : "memory");
+        else
+            asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(C::kTmemCols)
+                         : "memory");
     }
 }
 
@@ -687,14 +811,15 @@ inline int a_source(const FwdParams &p, int ks)
 }
 
 // N tile among {64, 128, 256} (up to max_bn): fewest rounds of tiles over the
-// SMs weighted by the tile's width plus a fixed per-tile cost; ties: the wider
-inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn)
+// SMs (CG = 2: pair tiles over the SM pairs) weighted by the tile's width plus a
+// fixed per-tile cost; ties: the wider
+inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn, int cg = 1)
 {
-    const int64_t sms = sm_count();
+    const int64_t sms = sm_count() / cg;
     int best = 64;
     int64_t best_cost = -1;
     for (int bn = 64; bn <= max_bn; bn *= 2) {
-        const int64_t tiles = m_tiles * ((Cout + bn - 1) / bn);
+        const int64_t tiles = ((m_tiles + cg - 1) / cg) * ((Cout + bn - 1) / bn);
         const int64_t cost = ((tiles + sms - 1) / sms) * (bn + 32);
         if (best_cost < 0 || cost <= best_cost) {
             best_cost = cost;
@@ -704,11 +829,11 @@ inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn)
     return best;
 }
 
-template <bool TF32, int ASRC, int BN>
+template <bool TF32, int ASRC, int BN, int CG>
 cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA, cudaStream_t stream)
 {
-    using C = Cfg<TF32, ASRC, BN>;
-    auto kern = gemm_ws_kernel<TF32, ASRC, BN>;
+    using C = Cfg<TF32, ASRC, BN, CG>;
+    auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG>;
     static const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::kSmem));
     if (attr != cudaSuccess) return attr;
@@ -716,7 +841,7 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
     const CUtensorMapDataType dt = TF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     const int elem = TF32 ? 4 : 2;
     const int64_t wdims[2] = {p.R, p.Cout};
-    const int wbox[2] = {C::kKS, C::kN};
+    const int wbox[2] = {C::kKS, C::kBRows};
     if (!make_map(&tmB0, p.wdense, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
     if (C::kBPlanes > 1) {
         const char *lo = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
@@ -734,9 +859,10 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
     const int64_t n_ct = (p.Cout + C::kN - 1) / C::kN;
     const int64_t m_tiles = ASRC == kA4d ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)
                                          : (p.N + C::kM - 1) / C::kM;
-    const int64_t n_tiles = n_ct * m_tiles;
-    const int64_t sms = sm_count();
-    const int64_t grid = n_tiles < sms ? n_tiles : sms;
+    // CG = 2: units are pair tiles (two M tiles), one per CTA pair
+    const int64_t n_tiles = n_ct * (CG == 2 ? (m_tiles + 1) / 2 : m_tiles);
+    const int64_t slots = sm_count() / CG;
+    const int64_t grid = CG * (n_tiles < slots ? n_tiles : slots);
     // programmatic dependent launch: may start once every block of the preceding
     // kernel on the stream (the decompression) has signalled; it waits for that
     // kernel's completion before reading memory
@@ -745,11 +871,15 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
     cfg.blockDim = dim3(C::kThreads);
     cfg.dynamicSmemBytes = C::kSmem;
     cfg.stream = stream;
-    cudaLaunchAttribute la[1];
+    cudaLaunchAttribute la[2];
     la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     la[0].val.programmaticStreamSerializationAllowed = 1;
+    la[1].id = cudaLaunchAttributeClusterDimension;
+    la[1].val.clusterDim.x = CG;
+    la[1].val.clusterDim.y = 1;
+    la[1].val.clusterDim.z = 1;
     cfg.attrs = la;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = CG == 2 ? 2 : 1;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p, tmA, tmB0, tmB1, tmY, box, n_ct, n_tiles);
     return e != cudaSuccess ? e : cudaGetLastError();
 }

@@ -1,5 +1,6 @@
 // cci_gemm_ws_bf16.cu -- bf16 layers of the workspace family: the kernel
-// configurations (activation source x N tile) and the choice among them.
+// configurations (activation source x N tile x CTAs per tile) and the choice
+// among them.
 #include "cci_gemm_ws.cuh"
 
 namespace cci {
@@ -10,9 +11,19 @@ cudaError_t launch_gemm_ws_bf16(const FwdParams &p, cudaStream_t stream)
     Plan pl;
     plan_layer(p, false, 64, &pl);
     const int asrc = pl.asrc;
-    const int bn = choose_bn(m_tiles_of(p, asrc, pl.box), p.Cout, 256);
+    const int64_t m_tiles = m_tiles_of(p, asrc, pl.box);
+    const int64_t nks = (p.R + 63) / 64;
+    // CTA pairs (256-row tiles, B split over the pair) halve each SM's B traffic,
+    // which pays on long reductions with 256-wide N tiles; shorter or narrower
+    // layers run faster on single CTAs (measured on the ResNet-50 stack)
+    const bool pair = asrc != kAGather && nks >= 16 && choose_bn(m_tiles, p.Cout, 256, 2) == 256;
+    if (pair) {
+        if (asrc == kA2d) return launch_cfg<false, kA2d, 256, 2>(p, pl.box, pl.am, stream);
+        return launch_cfg<false, kA4d, 256, 2>(p, pl.box, pl.am, stream);
+    }
+    const int bn = choose_bn(m_tiles, p.Cout, 256, 1);
 #define CCI_WS_CASE(A, N) \
-    if (asrc == A && bn == N) return launch_cfg<false, A, N>(p, pl.box, pl.am, stream);
+    if (asrc == A && bn == N) return launch_cfg<false, A, N, 1>(p, pl.box, pl.am, stream);
     CCI_WS_CASE(kA2d, 64)
     CCI_WS_CASE(kA2d, 128)
     CCI_WS_CASE(kA2d, 256)

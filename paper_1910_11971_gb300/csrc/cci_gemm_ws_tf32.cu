@@ -12,7 +12,7 @@ cudaError_t launch_gemm_ws_tf32(const FwdParams &p, cudaStream_t stream)
     const int asrc = pl.asrc;
     const int bn = choose_bn(m_tiles_of(p, asrc, pl.box), p.Cout, 128);
 #define CCI_WS_CASE(A, N) \
-    if (asrc == A && bn == N) return launch_cfg<true, A, N>(p, pl.box, pl.am, stream);
+    if (asrc == A && bn == N) return launch_cfg<true, A, N, 1>(p, pl.box, pl.am, stream);
     CCI_WS_CASE(kA2d, 64)
     CCI_WS_CASE(kA2d, 128)
     CCI_WS_CASE(kA4d, 64)

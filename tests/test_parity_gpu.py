@@ -534,3 +534,40 @@ def test_dense_tc_ws_conv_tma_equals_gather_bitwise(dev):
     Xcol = cols.reshape(B * H * Wi, 9 * Cin).to(BF16)
     Yl = run_linear(dev, Xcol, W, G, K, cci.ALGO_DENSE_TC_WS)
     assert torch.equal(Yc.reshape(-1, Cout).view(torch.int32), Yl.view(torch.int32))
+
+
+# ---------------------------------------------------------------------------
+# CTA-pair tiles (tcgen05 cta_group::2): bf16 layers with at least 16 stages of
+# 64 reduction indices and 256-wide N tiles run as 256-row tiles split over two
+# SMs.  Sizes below make the tile-round model pick that form; checked on sampled
+# outputs (first and last rows, the odd last M tile whose pair partner has no
+# rows, random rows).
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("N,Cin,Cout,G,K", [(38912 + 77, 1024, 736, 8, 2), (39040, 1088, 512, 16, 4)])
+def test_pair_tiles_product(dev, N, Cin, Cout, G, K):
+    X, W = wl.random_small(N + Cin, "bf16", N, Cin, Cout)
+    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    rows = np.unique(np.concatenate([sample_rows(N, 768, seed=N), np.arange(N - 200, N)]))
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, f"pair product {N}x{Cin}->{Cout}")
+
+
+@pytest.mark.parametrize("B,H,Cin,Cout,stride", [(63, 14, 128, 256, 1), (64, 28, 128, 256, 2)])
+def test_pair_tiles_conv(dev, B, H, Cin, Cout, stride):
+    G, K = 8, 2
+    g = torch.Generator().manual_seed(B * 31 + H)
+    X = torch.randn((B, H, H, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (3, 3, (stride, stride), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    P = (H + 2 - 3) // stride + 1
+    per = P * P
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    for b in (0, B - 1):
+        pts = np.unique(np.concatenate([np.arange(min(per, 64)), np.arange(per - 32, per),
+                                        np.random.default_rng(b).choice(per, size=64)]))
+        Yo, S = oracle.conv2d(f64(X[b:b + 1]), Wd, mask, 3, 3, (stride, stride), (1, 1), pts=pts)
+        Yg = f64(Y[b].reshape(-1, Cout)[torch.from_numpy(pts).to(dev)])
+        assert_within_tol(Yg, Yo, S, f"pair conv B={B} H={H} s={stride} image {b}")
