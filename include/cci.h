@@ -198,6 +198,35 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
                          int G, int K, float *Y, uint32_t *dev_status, cci_algo algo,
                          void *workspace, size_t workspace_bytes, cci_stream_t stream);
 
+/*
+ * cci_linear_fused / cci_conv2d_fused -- the product / convolution of
+ * cci_linear_ws / cci_conv2d_ws with CCI_ALGO_DENSE_TC_WS, followed by the usual
+ * output stage of a CNN layer, applied in the kernel's epilogue to each fp32
+ * accumulator y[n][co] (the sum of Alg. 2, Sec. 3.2):
+ *   y += bias[co]          when bias != NULL (fp32, Cout entries, 16-byte aligned);
+ *   y = max(y, 0)          when relu != 0;
+ *   Y[n][co] = y           as fp32 (out_dtype CCI_F32) or rounded to the nearest
+ *                          bf16, ties to even (out_dtype CCI_BF16; needs Cout % 8 == 0).
+ * The paper defines only the product; bias, ReLU and the bf16 output are the
+ * surrounding network's, fused here so that a layer's output is written once at
+ * the width the next layer reads.  X and Y must be 16-byte aligned and the
+ * workspace as for CCI_ALGO_DENSE_TC_WS (else CCI_ERR_ALIGN / CCI_ERR_WORKSPACE);
+ * layers without that family return CCI_ERR_UNSUPPORTED.  Y is [N][Cout] or NHWC
+ * [B][P][Q][Cout] of out_dtype; everything else as for cci_linear_ws /
+ * cci_conv2d_ws.  NaN accumulators become 0 under the ReLU.
+ */
+cci_status cci_linear_fused(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
+                            const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
+                            const float *bias, int relu, cci_dtype out_dtype, void *Y,
+                            uint32_t *dev_status, void *workspace, size_t workspace_bytes,
+                            cci_stream_t stream);
+cci_status cci_conv2d_fused(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W,
+                            int64_t Cin, const void *values, const uint8_t *idx, int64_t Cout,
+                            int KH, int KW, int stride_h, int stride_w, int pad_h, int pad_w,
+                            int G, int K, const float *bias, int relu, cci_dtype out_dtype,
+                            void *Y, uint32_t *dev_status, void *workspace,
+                            size_t workspace_bytes, cci_stream_t stream);
+
 /* Largest dense-weight size (Cout*R*2 bytes) that cci_linear_dense_tc_static accepts. */
 #define CCI_STATIC_WORKSPACE_BYTES (16u * 1024u * 1024u)
 

@@ -168,6 +168,22 @@ class Oracle:
 _default = None
 
 
+def epilogue(Y, S, bias=None, relu: bool = False):
+    """The output stage of a CNN layer applied to the exact product (fp64): Y + bias
+    per output channel (last axis), then max(., 0); with the error scale of the
+    sum extended by |bias|.  (Not part of the paper's method; the network around
+    a layer.)"""
+    Y = np.array(Y, dtype=np.float64, copy=True)
+    S = np.array(S, dtype=np.float64, copy=True)
+    if bias is not None:
+        b = _f64(bias).reshape(-1)
+        Y += b
+        S += np.abs(b)
+    if relu:
+        Y = np.maximum(Y, 0.0)
+    return Y, S
+
+
 def get() -> Oracle:
     """The oracle built from ``cci_oracle.c`` (compiled on first use)."""
     global _default

@@ -46,6 +46,11 @@ SIGNATURES = {
                              ctypes.c_size_t, _P]),
     "cci_conv2d_ws": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32, _I32,
                              _I32, _I32, _I32, _I32, _P, _U32P, _I32, _P, ctypes.c_size_t, _P]),
+    "cci_linear_fused": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _I32, _I32, _P,
+                                _U32P, _P, ctypes.c_size_t, _P]),
+    "cci_conv2d_fused": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32,
+                                _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _P, _U32P, _P,
+                                ctypes.c_size_t, _P]),
     "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
     "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
                                           _P]),
@@ -215,6 +220,65 @@ def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
                                G, K, Y.data_ptr(), status.data_ptr() if status is not None else None,
                                algo, wp, wb, _stream(X.device))
     _check(code, "cci_conv2d")
+    return Y
+
+
+def _out_code(dtype: torch.dtype) -> int:
+    if dtype == torch.float32:
+        return F32
+    if dtype == torch.bfloat16:
+        return BF16
+    raise TypeError(f"unsupported output dtype {dtype}: float32 or bfloat16")
+
+
+def linear_fused(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int, *,
+                 bias: Optional[torch.Tensor] = None, relu: bool = False,
+                 out_dtype: torch.dtype = torch.float32, out: Optional[torch.Tensor] = None,
+                 status: Optional[torch.Tensor] = None,
+                 workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Y[N][Cout] = relu?(product + bias) in ``out_dtype`` (fp32 or bf16), on the
+    workspace tensor-core family (``cci_linear_fused``)."""
+    _cuda_contig(X, "X")
+    N, Cin = X.shape
+    if workspace is None:
+        workspace = new_workspace(ALGO_DENSE_TC_WS, X.dtype, Cout, Cin, X.device)
+    Y = out if out is not None else torch.empty((N, Cout), dtype=out_dtype, device=X.device)
+    if bias is not None:
+        _cuda_contig(bias, "bias")
+    wp, wb = _ws(workspace)
+    code = lib().cci_linear_fused(X.data_ptr(), _dtype_code(X), N, Cin, values.data_ptr(), idx.data_ptr(),
+                                  Cout, G, K, bias.data_ptr() if bias is not None else None, int(relu),
+                                  _out_code(Y.dtype), Y.data_ptr(),
+                                  status.data_ptr() if status is not None else None, wp, wb,
+                                  _stream(X.device))
+    _check(code, "cci_linear_fused")
+    return Y
+
+
+def conv2d_fused(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int,
+                 KH: int, KW: int, stride=(1, 1), pad=(0, 0), *, bias: Optional[torch.Tensor] = None,
+                 relu: bool = False, out_dtype: torch.dtype = torch.float32,
+                 out: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
+                 workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Y NHWC [B][P][Q][Cout] = relu?(convolution + bias) in ``out_dtype`` (fp32 or
+    bf16), on the workspace tensor-core family (``cci_conv2d_fused``)."""
+    _cuda_contig(X, "X")
+    B, H, W, Cin = X.shape
+    P, Q = conv_out_hw(H, W, KH, KW, stride, pad)
+    Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=out_dtype,
+                                                device=X.device)
+    if workspace is None:
+        workspace = new_workspace(ALGO_DENSE_TC_WS, X.dtype, Cout, KH * KW * Cin, X.device)
+    if bias is not None:
+        _cuda_contig(bias, "bias")
+    wp, wb = _ws(workspace)
+    code = lib().cci_conv2d_fused(X.data_ptr(), _dtype_code(X), B, H, W, Cin, values.data_ptr(),
+                                  idx.data_ptr(), Cout, KH, KW, stride[0], stride[1], pad[0], pad[1], G, K,
+                                  bias.data_ptr() if bias is not None else None, int(relu),
+                                  _out_code(Y.dtype), Y.data_ptr(),
+                                  status.data_ptr() if status is not None else None, wp, wb,
+                                  _stream(X.device))
+    _check(code, "cci_conv2d_fused")
     return Y
 
 

@@ -89,10 +89,19 @@ bool dense_tc_shape_ok(int dtype, int G, int K, int64_t Cin, int64_t R)
 cci_status forward(FwdParams p, int dtype, int G, int K, cci_algo algo, void *ws, size_t ws_bytes,
                    cudaStream_t stream)
 {
-    if (p.N == 0) return CCI_OK;
     // a 1x1 convolution with unit stride and no padding is the product of X[B*H*W][Cin]
     if (p.is_conv && p.KH == 1 && p.KW == 1 && p.sh == 1 && p.sw == 1 && p.ph == 0 && p.pw == 0) p.is_conv = 0;
     const bool tc_fits = p.R < (int64_t(1) << 31) && p.Cout < (int64_t(1) << 31);  // 32-bit copy coordinates
+    if (p.bias || p.relu || p.out_bf16) {
+        // the output epilogue exists on the workspace tensor-core family only
+        if (!tc_fits || !dense_tc_shape_ok(dtype, G, K, p.Cin, p.R)) return CCI_ERR_UNSUPPORTED;
+        if (p.out_bf16 && p.Cout % 8 != 0) return CCI_ERR_UNSUPPORTED;  // 16-byte output rows
+        if (p.bias && !aligned(p.bias, 16)) return CCI_ERR_ALIGN;
+        if (!aligned(p.X, 16) || !aligned(p.Y, 16)) return CCI_ERR_ALIGN;
+        if (!ws || ws_bytes < dense_ws_bytes(dtype, p.Cout, p.R) || !aligned(ws, 16)) return CCI_ERR_WORKSPACE;
+        algo = CCI_ALGO_DENSE_TC_WS;
+    }
+    if (p.N == 0) return CCI_OK;
     if (algo == CCI_ALGO_AUTO && tc_fits && dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) && ws &&
         ws_bytes >= dense_ws_bytes(dtype, p.Cout, p.R) && aligned(ws, 16) && aligned(p.X, 16) && aligned(p.Y, 16))
         algo = CCI_ALGO_DENSE_TC_WS;
@@ -191,18 +200,31 @@ cci_status cci_pack(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int
                                  reinterpret_cast<cudaStream_t>(stream)));
 }
 
-cci_status cci_linear_ws(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
-                         const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
-                         cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream)
+}  // extern "C"
+
+namespace {
+
+struct Epilogue {
+    const float *bias;
+    int relu;
+    int out_bf16;
+};
+
+cci_status linear_impl(const void *X, int dtype, int64_t N, int64_t Cin, const void *values, const uint8_t *idx,
+                       int64_t Cout, int G, int K, void *Y, uint32_t *dev_status, cci_algo algo, void *workspace,
+                       size_t workspace_bytes, cci_stream_t stream, Epilogue e)
 {
-    const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, Cin, G, K);
+    const cci_status st = check_common(X, dtype, values, idx, static_cast<float *>(Y), N, Cout, Cin, G, K);
     if (st != CCI_OK) return st;
     if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
     FwdParams p{};
     p.X = X;
     p.values = values;
     p.idx = idx;
-    p.Y = Y;
+    p.Y = static_cast<float *>(Y);
+    p.bias = e.bias;
+    p.relu = e.relu;
+    p.out_bf16 = e.out_bf16;
     p.status = dev_status;
     p.N = N;
     p.Cout = Cout;
@@ -213,6 +235,33 @@ cci_status cci_linear_ws(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
     p.ph = p.pw = 0;
     p.is_conv = 0;
     return forward(p, dtype, G, K, algo, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cci_status conv_impl(const void *X, int dtype, int64_t B, int64_t H, int64_t W, int64_t Cin, const void *values,
+                     const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h, int stride_w, int pad_h,
+                     int pad_w, int G, int K, void *Y, uint32_t *dev_status, cci_algo algo, void *workspace,
+                     size_t workspace_bytes, cci_stream_t stream, Epilogue e);
+
+}  // namespace
+
+extern "C" {
+
+cci_status cci_linear_ws(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+                         const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
+                         cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream)
+{
+    return linear_impl(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, algo, workspace, workspace_bytes,
+                       stream, Epilogue{nullptr, 0, 0});
+}
+
+cci_status cci_linear_fused(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+                            const uint8_t *idx, int64_t Cout, int G, int K, const float *bias, int relu,
+                            cci_dtype out_dtype, void *Y, uint32_t *dev_status, void *workspace,
+                            size_t workspace_bytes, cci_stream_t stream)
+{
+    if (!valid_dtype(out_dtype)) return CCI_ERR_DTYPE;
+    return linear_impl(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, CCI_ALGO_DENSE_TC_WS, workspace,
+                       workspace_bytes, stream, Epilogue{bias, relu != 0, out_dtype == CCI_BF16});
 }
 
 cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
@@ -234,6 +283,32 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
                          int stride_w, int pad_h, int pad_w, int G, int K, float *Y, uint32_t *dev_status,
                          cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream)
 {
+    return conv_impl(X, dtype, B, H, W, Cin, values, idx, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, G, K, Y,
+                     dev_status, algo, workspace, workspace_bytes, stream, Epilogue{nullptr, 0, 0});
+}
+
+cci_status cci_conv2d_fused(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
+                            const void *values, const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h,
+                            int stride_w, int pad_h, int pad_w, int G, int K, const float *bias, int relu,
+                            cci_dtype out_dtype, void *Y, uint32_t *dev_status, void *workspace,
+                            size_t workspace_bytes, cci_stream_t stream)
+{
+    if (!valid_dtype(out_dtype)) return CCI_ERR_DTYPE;
+    return conv_impl(X, dtype, B, H, W, Cin, values, idx, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, G, K, Y,
+                     dev_status, CCI_ALGO_DENSE_TC_WS, workspace, workspace_bytes, stream,
+                     Epilogue{bias, relu != 0, out_dtype == CCI_BF16});
+}
+
+}  // extern "C"
+
+namespace {
+
+cci_status conv_impl(const void *X, int dtype, int64_t B, int64_t H, int64_t W, int64_t Cin, const void *values,
+                     const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h, int stride_w, int pad_h,
+                     int pad_w, int G, int K, void *Y_, uint32_t *dev_status, cci_algo algo, void *workspace,
+                     size_t workspace_bytes, cci_stream_t stream, Epilogue e)
+{
+    float *Y = static_cast<float *>(Y_);
     if (B < 0 || H < 1 || W < 1 || Cin < 1 || KH < 1 || KW < 1 || stride_h < 1 || stride_w < 1 || pad_h < 0 ||
         pad_w < 0)
         return valid_dtype(dtype) ? CCI_ERR_SHAPE : CCI_ERR_DTYPE;
@@ -270,8 +345,15 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
     p.ph = pad_h;
     p.pw = pad_w;
     p.is_conv = 1;
+    p.bias = e.bias;
+    p.relu = e.relu;
+    p.out_bf16 = e.out_bf16;
     return forward(p, dtype, G, K, algo, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
+
+}  // namespace
+
+extern "C" {
 
 cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
                          const void *values, const uint8_t *idx, int64_t Cout, int KH, int KW, int stride_h,

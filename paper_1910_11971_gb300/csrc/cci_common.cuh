@@ -15,7 +15,7 @@ struct FwdParams {
     const void *X;
     const void *values;
     const uint8_t *idx;
-    float *Y;
+    float *Y;            // fp32 output, or bf16 when out_bf16
     uint32_t *status;
     int64_t N;      // columns = B*P*Q
     int64_t Cout;
@@ -26,6 +26,10 @@ struct FwdParams {
     int KH, KW, sh, sw, ph, pw;
     int is_conv;
     const void *wdense;  // dense decompressed weights [Cout][R] (workspace kernels only)
+    // output epilogue (workspace kernels only): y + bias[co], ReLU, bf16 output
+    const float *bias;   // nullptr: none
+    int relu;
+    int out_bf16;        // Y holds bf16 (round to nearest even) instead of fp32
 };
 
 __device__ __forceinline__ void report(uint32_t *status, cci_status code)

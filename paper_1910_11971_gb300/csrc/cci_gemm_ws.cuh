@@ -197,6 +197,43 @@ __device__ __forceinline__ void tma_load_4d_pair(uint32_t dst, const void *tmap,
         : "memory");
 }
 
+// Output epilogue of a CNN layer, on 32 consecutive fp32 accumulator values of
+// one row at output channels col0..col0+31: y + bias[co] (when p.bias), then
+// max(y, 0) (when p.relu).  Channels >= Cout get no bias (their columns are
+// clipped by the store).
+__device__ __forceinline__ void epilogue_math(uint32_t (&v)[32], const FwdParams &p, int col0)
+{
+    if (p.bias) {
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const int col = col0 + 4 * q;
+            // Cout is a multiple of 4 and the bias 16-byte aligned: a float4 that
+            // starts inside the row of biases lies wholly inside it
+            const float4 b = col < p.Cout ? __ldg(reinterpret_cast<const float4 *>(p.bias + col))
+                                          : make_float4(0.f, 0.f, 0.f, 0.f);
+            v[4 * q] = __float_as_uint(__uint_as_float(v[4 * q]) + b.x);
+            v[4 * q + 1] = __float_as_uint(__uint_as_float(v[4 * q + 1]) + b.y);
+            v[4 * q + 2] = __float_as_uint(__uint_as_float(v[4 * q + 2]) + b.z);
+            v[4 * q + 3] = __float_as_uint(__uint_as_float(v[4 * q + 3]) + b.w);
+        }
+    }
+    if (p.relu) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            const float x = __uint_as_float(v[j]);
+            v[j] = __float_as_uint(x > 0.f ? x : 0.f);
+        }
+    }
+}
+
+// two fp32 values (lo at the lower address) rounded to nearest even bf16
+__device__ __forceinline__ uint32_t bf16x2_rn(uint32_t lo, uint32_t hi)
+{
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(__uint_as_float(hi)), "f"(__uint_as_float(lo)));
+    return r;
+}
+
 // byte offset of (row, 16-byte chunk) in a plane of 128-byte rows, 128-byte swizzle
 __device__ __forceinline__ uint32_t sw_chunk(int row, int chunk)
 {
@@ -618,12 +655,13 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
         tc::mbar_wait(&S->drain, 0, &no_abort, p.status);
     } else {
         // ------------------------------------------------------------ epilogue (warps 0-3)
-        // Per 32-column chunk: TMEM -> registers -> swizzled staging buffer (row m =
-        // thread) -> one TMA store of the tile's box (rows past N, the image or
-        // Cout are clipped by the copy).  Two buffers alternate; a buffer is
-        // rewritten once the store issued from it two chunks earlier has read it.
-        // Every decision that gates a named barrier is uniform over the 128
-        // threads (named_and), so the barriers always see all of them.
+        // Per chunk of one 128-byte output row (32 fp32 or 64 bf16 columns): TMEM ->
+        // registers (+ bias, ReLU, bf16 rounding when asked) -> swizzled staging
+        // buffer (row m = thread) -> one TMA store of the tile's box (rows past N,
+        // the image or Cout are clipped by the copy).  Two buffers alternate; a
+        // buffer is rewritten once the store issued from it two chunks earlier has
+        // read it.  Every decision that gates a named barrier is uniform over the
+        // 128 threads (named_and), so the barriers always see all of them.
         int t = 0;
         bool ok = true;
         const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
@@ -642,10 +680,25 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
             if (!ok) break;
             __syncwarp();
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const int sc = p.out_bf16 ? 64 : 32;  // output columns per staged 128-byte row
 #pragma unroll 1
-            for (int c = 0; c < kN / 32 && co0 + c * 32 < p.Cout; ++c, ++chunk_no) {
+            for (int c0 = 0; c0 < kN && co0 + c0 < p.Cout; c0 += sc, ++chunk_no) {
                 uint32_t v[32];
-                tc::tmem_ld32(tmem + lane_off + static_cast<uint32_t>(acc * kN + c * 32), v);
+                const uint32_t tcol = tmem + lane_off + static_cast<uint32_t>(acc * kN + c0);
+                if (!p.out_bf16) {
+                    tc::tmem_ld32(tcol, v);
+                    epilogue_math(v, p, co0 + c0);
+                } else {
+                    uint32_t w[32];
+                    tc::tmem_ld32(tcol, w);
+                    epilogue_math(w, p, co0 + c0);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) v[j] = bf16x2_rn(w[2 * j], w[2 * j + 1]);
+                    tc::tmem_ld32(tcol + 32, w);
+                    epilogue_math(w, p, co0 + c0 + 32);
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) v[16 + j] = bf16x2_rn(w[2 * j], w[2 * j + 1]);
+                }
                 const uint32_t buf = ybuf + static_cast<uint32_t>(chunk_no & 1) * C::kYBuf;
                 if (tid == 0) tc::bulk_wait_read<1>();
                 tc::named_sync(1, 128);
@@ -656,10 +709,10 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
                 tc::named_sync(1, 128);
                 if (tid == 0) {
                     if constexpr (ASRC == kA4d)
-                        tc::tma_store_4d(&tmY, buf, co0 + c * 32, bi.qb * box.QB, bi.pb * box.PB,
+                        tc::tma_store_4d(&tmY, buf, co0 + c0, bi.qb * box.QB, bi.pb * box.PB,
                                          static_cast<int>(bi.bb * box.BB));
                     else
-                        tc::tma_store_2d(&tmY, buf, co0 + c * 32, static_cast<int>(mt * kM));
+                        tc::tma_store_2d(&tmY, buf, co0 + c0, static_cast<int>(mt * kM));
                     tc::bulk_commit();
                 }
             }
@@ -847,14 +900,17 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
         const char *lo = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
         if (!make_map(&tmB1, lo, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
     }
+    // output rows of 128 bytes: 32 fp32 or 64 bf16 channels
+    const CUtensorMapDataType ydt = p.out_bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    const int yel = p.out_bf16 ? 2 : 4, ysc = p.out_bf16 ? 64 : 32;
     if constexpr (ASRC == kA4d) {
         const int64_t dims[4] = {p.Cout, p.Q, p.P, box.B};
-        const int bx[4] = {32, box.QB, box.PB, box.BB};
-        if (!make_map(&tmY, p.Y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, 4, dims, bx)) return cudaErrorInvalidValue;
+        const int bx[4] = {ysc, box.QB, box.PB, box.BB};
+        if (!make_map(&tmY, p.Y, ydt, yel, 4, dims, bx)) return cudaErrorInvalidValue;
     } else {
         const int64_t dims[2] = {p.Cout, p.N};
-        const int bx[2] = {32, C::kM};
-        if (!make_map(&tmY, p.Y, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, 2, dims, bx)) return cudaErrorInvalidValue;
+        const int bx[2] = {ysc, C::kM};
+        if (!make_map(&tmY, p.Y, ydt, yel, 2, dims, bx)) return cudaErrorInvalidValue;
     }
     const int64_t n_ct = (p.Cout + C::kN - 1) / C::kN;
     const int64_t m_tiles = ASRC == kA4d ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)

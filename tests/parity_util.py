@@ -61,3 +61,18 @@ def sample_rows(N: int, k: int, seed: int = 0) -> np.ndarray:
     edge = min(64, k // 4)
     mid = rng.choice(np.arange(edge, N - edge), size=k - 2 * edge, replace=False)
     return np.unique(np.concatenate([np.arange(edge), np.sort(mid), np.arange(N - edge, N)]))
+
+
+def assert_fused_within_tol(y_gpu: np.ndarray, y_ref: np.ndarray, S: np.ndarray, out_bf16: bool, what: str = ""):
+    """Outputs of the fused epilogue against oracle.epilogue(): the product's bound
+    1e-5 * S (S including |bias|; ReLU is 1-Lipschitz) plus, for bf16 outputs, the
+    final rounding (half a bf16 unit in the last place <= 2^-8 * |y|)."""
+    assert y_gpu.shape == y_ref.shape, (y_gpu.shape, y_ref.shape)
+    assert np.isfinite(y_gpu).all(), f"{what}: non-finite outputs"
+    lim = TOL * (1 + 2.0 ** -8) * S + (2.0 ** -8 * np.abs(y_ref) if out_bf16 else 0.0)
+    err = np.abs(y_gpu - y_ref)
+    bad = err > lim
+    if bad.any():
+        i = np.argwhere(bad)[0]
+        raise AssertionError(f"{what}: {bad.sum()} of {bad.size} outputs out of tolerance; first at "
+                             f"{i.tolist()}: gpu={y_gpu[tuple(i)]!r} ref={y_ref[tuple(i)]!r} S={S[tuple(i)]!r}")

@@ -164,3 +164,29 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(cci, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="not built"):
         cci.lib()
+
+
+def fused(lib, X=FAKE, dt=1, N=16, Cin=64, V=FAKE, I=FAKE, Cout=64, G=8, K=2, bias=None, relu=1, od=1,
+          Y=FAKE, ws=FAKE, wsb=1 << 20):
+    return lib.cci_linear_fused(X, dt, N, Cin, V, I, Cout, G, K, bias, relu, od, Y, None, ws, wsb, None)
+
+
+def test_fused_rejects(lib):
+    """The fused epilogue (bias, ReLU, bf16 output) exists on the workspace
+    tensor-core family only; every argument error is returned before a launch."""
+    assert fused(lib, od=5) == DTYPE
+    assert fused(lib, dt=5) == DTYPE
+    assert fused(lib, V=None) == NULL
+    assert fused(lib, Cout=60) == GROUP                   # Cout % G
+    assert fused(lib, G=64, Cout=64) == UNSUP             # G without a dense tensor-core kernel
+    assert fused(lib, G=4, K=2, Cout=68) == UNSUP         # bf16 rows need Cout % 8 == 0
+    assert fused(lib, bias=FAKE + 4) == ALIGN             # bias must be 16-byte aligned
+    assert fused(lib, Y=FAKE + 8) == ALIGN
+    assert fused(lib, X=FAKE + 8) == ALIGN
+    assert fused(lib, ws=None, wsb=0) == 11               # CCI_ERR_WORKSPACE
+    assert fused(lib, wsb=64 * 64 * 2 - 2) == 11
+    assert fused(lib, ws=FAKE + 8) == 11
+    assert lib.cci_conv2d_fused(FAKE, 1, 1, 4, 4, 64, FAKE, FAKE, 64, 3, 3, 1, 1, 1, 1, 8, 2, None, 1, 1,
+                                FAKE, None, None, 0, None) == 11
+    assert lib.cci_conv2d_fused(FAKE, 1, 1, 4, 4, 64, FAKE, FAKE, 64, 3, 3, 1, 1, 1, 1, 8, 2, None, 1, 7,
+                                FAKE, None, FAKE, 1 << 20, None) == DTYPE

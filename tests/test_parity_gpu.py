@@ -186,6 +186,18 @@ def test_linear_sweep_full(dev, G, K):
     assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name)
 
 
+def test_linear_sweep_every_output_G8_K2(dev):
+    """4096 -> 4096, N = 8192, bf16, G = 8, K = 2 through the production path:
+    every one of the 33.5 M outputs against the oracle (about 69 GFLOP of fp64
+    work on the host)."""
+    case = wl.sweep_case(8, 2)
+    X, W = wl.linear_inputs(case, device="cpu")
+    Y = run_linear(dev, X, W, 8, 2)
+    _, _, Wd, mask = oracle_reference(W, 8, 2)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, case.name + " (all outputs)")
+
+
 @pytest.mark.parametrize("algo", [cci.ALGO_GENERIC] + REGTILE_ALGOS)
 def test_linear_bad_index_reported(dev, algo):
     G, K, Cout, Cin, N = 8, 2, 16, 32, 40
@@ -571,3 +583,93 @@ def test_pair_tiles_conv(dev, B, H, Cin, Cout, stride):
         Yo, S = oracle.conv2d(f64(X[b:b + 1]), Wd, mask, 3, 3, (stride, stride), (1, 1), pts=pts)
         Yg = f64(Y[b].reshape(-1, Cout)[torch.from_numpy(pts).to(dev)])
         assert_within_tol(Yg, Yo, S, f"pair conv B={B} H={H} s={stride} image {b}")
+
+
+# ---------------------------------------------------------------------------
+# fused output epilogue: + bias, ReLU, fp32 or bf16 (round to nearest even)
+# output, on every activation source and tile form of the workspace family
+# ---------------------------------------------------------------------------
+from parity_util import assert_fused_within_tol  # noqa: E402
+
+# (N, Cin, Cout, G, K, in dtype, bias, relu, out dtype)
+FUSED_PRODUCTS = [
+    (300, 64, 256, 8, 2, "bf16", True, True, "bf16"),
+    (300, 64, 256, 8, 2, "bf16", True, False, "f32"),
+    (1000, 128, 136, 8, 2, "bf16", False, True, "bf16"),
+    (517, 96, 128, 16, 4, "f32", True, True, "bf16"),
+    (129, 256, 1024, 8, 2, "f32", True, False, "f32"),
+]
+
+
+def _bias(Cout, seed):
+    return (torch.randn(Cout, generator=torch.Generator().manual_seed(seed)) * 0.5).float()
+
+
+@pytest.mark.parametrize("case", FUSED_PRODUCTS, ids=lambda c: "N{}_C{}x{}_G{}K{}_{}_b{}_r{}_{}".format(*c))
+def test_fused_product(dev, case):
+    N, Cin, Cout, G, K, dt, use_bias, relu, od = case
+    X, W = wl.random_small(N + Cout, dt, N, Cin, Cout)
+    b = _bias(Cout, N) if use_bias else None
+    v, i = cci.pack(W.to(dev), G, K)
+    Y = cci.linear_fused(X.to(dev), v, i, Cout, G, K, bias=b.to(dev) if b is not None else None, relu=relu,
+                         out_dtype=_dt(od))
+    assert Y.dtype == _dt(od)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    Yr, Sr = oracle.epilogue(Yo, S, f64(b) if b is not None else None, relu)
+    assert_fused_within_tol(f64(Y), Yr, Sr, od == "bf16", str(case))
+    if relu:
+        assert (f64(Y) >= 0).all()
+
+
+# (B, H, W, Cin, Cout, KH, KW, stride, pad, G, K, in dtype): 4-D copy, stride-2
+# lattices, row gather (stride 3), fp32 input
+FUSED_CONVS = [
+    (3, 9, 7, 64, 64, 3, 3, (1, 1), (1, 1), 8, 2, "bf16"),
+    (2, 9, 7, 64, 128, 3, 3, (2, 2), (1, 1), 8, 2, "bf16"),
+    (1, 10, 10, 64, 64, 3, 3, (3, 3), (1, 1), 8, 2, "bf16"),
+    (2, 9, 7, 32, 64, 3, 3, (1, 1), (1, 1), 8, 2, "f32"),
+]
+
+
+@pytest.mark.parametrize("od", ["bf16", "f32"])
+@pytest.mark.parametrize("case", FUSED_CONVS, ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
+def test_fused_conv(dev, case, od):
+    B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dt = case
+    g = torch.Generator().manual_seed(B * 41 + Cin + Cout)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(_dt(dt))
+    W = torch.randn((Cout, KH * KW * Cin), generator=g).to(_dt(dt))
+    b = _bias(Cout, B + Cout)
+    v, i = cci.pack(W.to(dev), G, K)
+    Y = cci.conv2d_fused(X.to(dev), v, i, Cout, G, K, KH, KW, stride, pad, bias=b.to(dev), relu=True,
+                         out_dtype=_dt(od))
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, stride, pad)
+    Yr, Sr = oracle.epilogue(Yo, S, f64(b), True)
+    assert_fused_within_tol(f64(Y).reshape(-1, Cout), Yr, Sr, od == "bf16", str(case))
+
+
+def test_fused_pair_tiles(dev):
+    """CTA-pair tiles (long reduction, 256-wide N tile) with bias, ReLU and bf16
+    output; sampled rows."""
+    N, Cin, Cout, G, K = 38912 + 77, 1024, 736, 8, 2
+    X, W = wl.random_small(N + 1, "bf16", N, Cin, Cout)
+    b = _bias(Cout, 3)
+    v, i = cci.pack(W.to(dev), G, K)
+    Y = cci.linear_fused(X.to(dev), v, i, Cout, G, K, bias=b.to(dev), relu=True, out_dtype=BF16)
+    rows = np.unique(np.concatenate([sample_rows(N, 512, seed=9), np.arange(N - 160, N)]))
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
+    Yr, Sr = oracle.epilogue(Yo, S, f64(b), True)
+    assert_fused_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yr, Sr, True, "fused pair")
+
+
+def test_fused_identity_equals_plain_product(dev):
+    """No bias, no ReLU, fp32 output: bit for bit the plain workspace product."""
+    N, Cin, Cout, G, K = 700, 128, 256, 8, 2
+    X, W = wl.random_small(5, "bf16", N, Cin, Cout)
+    Xd = X.to(dev)
+    v, i = cci.pack(W.to(dev), G, K)
+    Yf = cci.linear_fused(Xd, v, i, Cout, G, K)
+    Yp = cci.linear(Xd, v, i, Cout, G, K, algo=cci.ALGO_DENSE_TC_WS)
+    assert torch.equal(Yf.view(torch.int32), Yp.view(torch.int32))
