@@ -147,6 +147,20 @@ def resnet50_layers(batch: int = 128, G: int = 8, K: int = 2) -> List[ConvCase]:
     return layers
 
 
+def resnet50_roles() -> List[str]:
+    """Role of each of the 52 layers of resnet50_layers() in its bottleneck block:
+    'a' (1x1 reduce, reads the block input), 'b' (3x3, reads a's output), 'c' (1x1
+    expand, reads b's output; its output is the next block's input when the
+    residual add is left out) and 'proj' (strided 1x1 shortcut, reads the block
+    input)."""
+    roles: List[str] = []
+    for blocks in (3, 4, 6, 3):
+        for b in range(blocks):
+            roles += ["a", "b", "c"] + (["proj"] if b == 0 else [])
+    assert len(roles) == 52
+    return roles
+
+
 # ---------------------------------------------------------------------------
 # seeded draws
 # ---------------------------------------------------------------------------
