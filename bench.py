@@ -636,7 +636,94 @@ def run_extras(cci, dev, stream, flush):
                          "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R, case.Cout,
                                                    case.G, case.K)}
     out["resnet50_stack"] = run_resnet_stack(cci, dev, stream, flush)
+    out["mobilenetv2_pointwise"] = run_pointwise_stack(cci, dev, stream, flush)
+    out["allocation_error"] = run_allocation_error(cci, dev, stream, flush)
     return out
+
+
+def run_pointwise_stack(cci, dev, stream, flush, reps=5):
+    """The 34 pointwise convolutions of MobileNetV2 (batch 128, bf16, G = 8, K = 2:
+    the paper's 75 % case), each on its own synthetic input, captured in CUDA
+    graphs: fp32 outputs (the library's product), bf16 outputs with bias through
+    the fused epilogue, and cuDNN on the masked dense weights (bf16 output)."""
+    layers = wl.mobilenetv2_pointwise_layers()
+    plain, fused, dense, keep = [], [], [], []
+    for c in layers:
+        X, W = wl.conv_inputs(c, device=str(dev))
+        v, i = cci.pack(W, c.G, c.K)
+        Y = torch.empty((c.B, c.P, c.Q, c.Cout), dtype=torch.float32, device=dev)
+        Yb = torch.empty((c.B, c.P, c.Q, c.Cout), dtype=torch.bfloat16, device=dev)
+        bias = torch.zeros(c.Cout, dtype=torch.float32, device=dev)
+        ws = cci.new_workspace(cci.ALGO_AUTO, X.dtype, c.Cout, c.R, dev)
+        Wm = torch.zeros((c.Cout, c.R), dtype=W.dtype, device=dev)
+        Wm.view(c.Cout // c.G, c.G, c.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
+        w4 = Wm.view(c.Cout, 1, 1, c.Cin).permute(0, 3, 1, 2).contiguous(memory_format=torch.channels_last)
+        x4 = X.permute(0, 3, 1, 2)
+        del W, Wm
+        keep.append((X, v, i, Y, Yb, bias, ws, w4, x4))
+        plain.append(lambda c=c, X=X, v=v, i=i, Y=Y, ws=ws: cci.conv2d(
+            X, v, i, c.Cout, c.G, c.K, 1, 1, (1, 1), (0, 0), out=Y, workspace=ws))
+        fused.append(lambda c=c, X=X, v=v, i=i, Yb=Yb, ws=ws, bias=bias: cci.conv2d_fused(
+            X, v, i, c.Cout, c.G, c.K, 1, 1, (1, 1), (0, 0), bias=bias, out=Yb, workspace=ws))
+        dense.append(lambda x4=x4, w4=w4: torch.nn.functional.conv2d(x4, w4))
+    res = {"layers": len(layers), "batch": layers[0].B, "G": 8, "K": 2}
+    for name, calls in (("ms", plain), ("fused_bf16_out_ms", fused), ("dense_cudnn_bf16_ms", dense)):
+        for f in calls:
+            f()
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for f in calls:
+                f()
+        g.replay()
+        torch.cuda.synchronize(dev)
+        res[name] = statistics.median(time_device(g.replay, reps, flush, stream))
+        del g
+    nzf = sum(c.nz_flops() for c in layers)
+    floor_ms = sum(layer_floor_us(c) for c in layers) * 1e-3
+    res.update({"nz_gflop": nzf / 1e9, "nz_tflops": nzf / (res["ms"] * 1e-3) / 1e12,
+                "dense_equiv_tflops": sum(c.dense_flops() for c in layers) / (res["ms"] * 1e-3) / 1e12,
+                "roofline_floor_ms": floor_ms, "roofline_frac": floor_ms / res["ms"],
+                "speedup_over_dense": res["dense_cudnn_bf16_ms"] / res["ms"],
+                "fused_speedup_over_dense": res["dense_cudnn_bf16_ms"] / res["fused_bf16_out_ms"]})
+    del keep, plain, fused, dense
+    torch.cuda.empty_cache()
+    return res
+
+
+def run_allocation_error(cci, dev, stream, flush, reps=5):
+    """Eq. 1 measured: cci_pack_stats on 4096 x 8192 fp32 weight matrices whose
+    zeros are independent with probability Ps (seeded), K = G (1 - Ps), next to the
+    closed form (tests/golden/eq1_pd.txt); plus the counting kernel's rate
+    (weights read once)."""
+    eq1 = {}
+    with open(os.path.join(ROOT, "tests", "golden", "eq1_pd.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                ps, g, _, pd = line.split()
+                num, den = ps.split("/")
+                eq1[(int(num) / int(den), int(g))] = float(pd)
+    Cout, R = 4096, 8192
+    rows = []
+    for Ps in (0.5, 0.75, 0.875, 0.9375):
+        g = torch.Generator(device=str(dev)).manual_seed(int(Ps * 10000))
+        W = torch.randn((Cout, R), generator=g, device=dev)
+        W[torch.rand((Cout, R), generator=g, device=dev) < Ps] = 0
+        for G in (2, 4, 8, 16, 32, 64, 128, 256):
+            K = G * (1 - Ps)
+            if K < 1 or abs(K - round(K)) > 1e-9:
+                continue
+            K = int(round(K))
+            counts = cci.pack_stats(W, G, K)
+            nz, dropped = counts.cpu().tolist()
+            rows.append({"Ps": Ps, "G": G, "K": K, "measured_Pd": dropped / nz, "eq1_Pd": eq1.get((Ps, G))})
+        del W
+    W = torch.randn((Cout, R), device=dev)
+    counts = torch.zeros(2, dtype=torch.int64, device=dev)
+    ms = statistics.median(time_device(lambda: cci.pack_stats(W, 8, 2, counts=counts), reps, flush, stream))
+    return {"points": rows, "stats_kernel_ms_4096x8192_f32": ms,
+            "stats_kernel_gbs": Cout * R * 4 / (ms * 1e-3) / 1e9,
+            "what": "dropped nonzero weights / nonzero weights when packing iid-sparse matrices (Eq. 1)"}
 
 
 def layer_floor_us(c) -> float:

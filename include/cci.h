@@ -199,6 +199,20 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
                          void *workspace, size_t workspace_bytes, cci_stream_t stream);
 
 /*
+ * cci_pack_stats -- the allocation error of packing W (Sec. 4, Eq. 1, measured):
+ * adds to counts[0] the number of nonzero weights of W[Cout][R] and to counts[1]
+ * the number of them that cci_pack with (G, K) cannot keep (per group of G
+ * output channels at one input index, the nonzeros beyond K).  counts[1] /
+ * counts[0] estimates Eq. 1's P_d when the zeros of W are independent with
+ * probability Ps and K = G*(1 - Ps).  A weight is nonzero when its magnitude
+ * bits are (-0 counts as zero).  W: device, row-major, dtype bf16 or fp32;
+ * counts: device, two 8-byte-aligned unsigned 64-bit counters the caller zeroes
+ * and reads after a stream sync.  Argument errors as for cci_pack.
+ */
+cci_status cci_pack_stats(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K,
+                          unsigned long long *counts, cci_stream_t stream);
+
+/*
  * cci_linear_fused / cci_conv2d_fused -- the product / convolution of
  * cci_linear_ws / cci_conv2d_ws with CCI_ALGO_DENSE_TC_WS, followed by the usual
  * output stage of a CNN layer, applied in the kernel's epilogue to each fp32

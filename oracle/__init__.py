@@ -24,6 +24,9 @@ import ctypes
 import os
 import subprocess
 
+import math
+from fractions import Fraction
+
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -166,6 +169,48 @@ class Oracle:
 
 
 _default = None
+
+
+def allocation_error(G: int, Ps: float) -> float:
+    """Eq. 1 (Sec. 4): probability that a nonzero weight finds no encoding slot
+    when each of the G weights of a group is nonzero independently with
+    probability 1 - Ps and the group has s = G * (1 - Ps) slots:
+    sum over i > s of (i - s) * Binomial(i; G, 1 - Ps), divided by s."""
+    s = G * (1.0 - Ps)
+    si = int(round(s))
+    if si < 1 or abs(s - si) > 1e-9:
+        raise ValueError("s = G * (1 - Ps) must be a positive integer")
+    p = 1.0 - Ps
+    total = 0.0
+    for i in range(si + 1, G + 1):
+        total += (i - si) * math.comb(G, i) * p ** i * (1.0 - p) ** (G - i)
+    return total / si
+
+
+def allocation_error_exact(G: int, Ps) -> Fraction:
+    """Eq. 1 in exact rational arithmetic (Ps a Fraction or a string such as '3/4')."""
+    Ps = Fraction(Ps)
+    p = 1 - Ps
+    s = G * p
+    if s.denominator != 1 or s < 1:
+        raise ValueError("s = G * (1 - Ps) must be a positive integer")
+    si = int(s)
+    total = Fraction(0)
+    for i in range(si + 1, G + 1):
+        total += (i - si) * math.comb(G, i) * p ** i * (1 - p) ** (G - i)
+    return total / si
+
+
+def pack_stats(W, G: int, K: int):
+    """(nonzero weights of W[Cout][R], nonzero weights that packing with group size G
+    and K slots cannot keep): per group (G consecutive output channels at one r,
+    Sec. 3.1) the nonzeros beyond K, summed.  Plain counting."""
+    W = np.asarray(W)
+    Cout, R = W.shape
+    if Cout % G:
+        raise ValueError("Cout % G != 0")
+    nz = (W.reshape(Cout // G, G, R) != 0).sum(axis=1)
+    return int(nz.sum()), int(np.maximum(nz - K, 0).sum())
 
 
 def epilogue(Y, S, bias=None, relu: bool = False):

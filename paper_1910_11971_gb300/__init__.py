@@ -51,6 +51,7 @@ SIGNATURES = {
     "cci_conv2d_fused": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _P, _I64, _I32, _I32, _I32,
                                 _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _P, _U32P, _P,
                                 ctypes.c_size_t, _P]),
+    "cci_pack_stats": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, _P, _P]),
     "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
     "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
                                           _P]),
@@ -221,6 +222,19 @@ def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
                                algo, wp, wb, _stream(X.device))
     _check(code, "cci_conv2d")
     return Y
+
+
+def pack_stats(W: torch.Tensor, G: int, K: int, counts: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Adds (nonzero weights of W, nonzero weights packing with (G, K) drops) into
+    ``counts`` (int64 device tensor of 2, zeroed here when not given) and returns it
+    (``cci_pack_stats``; read it after a sync)."""
+    _cuda_contig(W, "W")
+    Cout, R = W.shape
+    if counts is None:
+        counts = torch.zeros(2, dtype=torch.int64, device=W.device)
+    _check(lib().cci_pack_stats(W.data_ptr(), _dtype_code(W), Cout, R, G, K, counts.data_ptr(),
+                                _stream(W.device)), "cci_pack_stats")
+    return counts
 
 
 def _out_code(dtype: torch.dtype) -> int:

@@ -246,6 +246,18 @@ cci_status conv_impl(const void *X, int dtype, int64_t B, int64_t H, int64_t W, 
 
 extern "C" {
 
+cci_status cci_pack_stats(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K,
+                          unsigned long long *counts, cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!W || !counts) return CCI_ERR_NULL;
+    if (Cout < 1 || R < 1 || !mul_ok(Cout, R)) return CCI_ERR_SHAPE;
+    const cci_status g = check_group(Cout, G, K);
+    if (g != CCI_OK) return g;
+    if (!aligned(W, elem_size(dtype)) || !aligned(counts, 8)) return CCI_ERR_ALIGN;
+    return to_status(launch_pack_stats(W, dtype, Cout, R, G, K, counts, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 cci_status cci_linear_ws(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
                          const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
                          cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream)

@@ -63,6 +63,71 @@ cudaError_t launch_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G
 }
 
 // ---------------------------------------------------------------------------
+// allocation statistics of packing (Sec. 4, Eq. 1 measured on a weight matrix):
+// per (group, r) the nonzero weights among the G and those beyond the K slots;
+// one thread per (group, r), warp sums, one 64-bit atomic per warp and counter.
+// A weight is nonzero when its magnitude bits are (so -0 is zero).
+// ---------------------------------------------------------------------------
+template <typename TB>
+__global__ void pack_stats_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, int G, int K,
+                                  unsigned long long *counts)
+{
+    constexpr uint32_t kMag = sizeof(TB) == 4 ? 0x7fffffffu : 0x7fffu;
+    const int64_t total = (Cout / G) * R;
+    uint32_t nz_sum = 0, drop_sum = 0;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gi = t / R, r = t - gi * R;
+        const TB *w = W + gi * G * R + r;
+        int nz = 0;
+        for (int j = 0; j < G; ++j) nz += (static_cast<uint32_t>(w[j * R]) & kMag) != 0;
+        nz_sum += static_cast<uint32_t>(nz);
+        drop_sum += static_cast<uint32_t>(nz > K ? nz - K : 0);
+    }
+    // block sum (warp shuffles, then the first warp over the warp sums), one
+    // atomic per block and counter
+    __shared__ unsigned long long part[2][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    nz_sum = __reduce_add_sync(0xffffffffu, nz_sum);
+    drop_sum = __reduce_add_sync(0xffffffffu, drop_sum);
+    if (lane == 0) {
+        part[0][warp] = nz_sum;
+        part[1][warp] = drop_sum;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = blockDim.x >> 5;
+        unsigned long long a = lane < nw ? part[0][lane] : 0ull, b = lane < nw ? part[1][lane] : 0ull;
+        for (int o = 16; o > 0; o >>= 1) {
+            a += __shfl_down_sync(0xffffffffu, a, o);
+            b += __shfl_down_sync(0xffffffffu, b, o);
+        }
+        if (lane == 0) {
+            atomicAdd(counts, a);
+            atomicAdd(counts + 1, b);
+        }
+    }
+}
+
+cudaError_t launch_pack_stats(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K,
+                              unsigned long long *counts, cudaStream_t stream)
+{
+    const int64_t total = (Cout / G) * R;
+    const int threads = 256;
+    const int64_t blocks = (total + threads - 1) / threads;
+    // at most 8 blocks per SM with grid-stride loops: few atomics; a thread's
+    // sums stay far below 2^32 for any matrix that fits in memory
+    const int grid = static_cast<int>(blocks < 152 * 8 ? blocks : 152 * 8);
+    if (dtype == CCI_F32)
+        pack_stats_kernel<uint32_t><<<grid, threads, 0, stream>>>(static_cast<const uint32_t *>(W), Cout, R, G, K,
+                                                                  counts);
+    else
+        pack_stats_kernel<uint16_t><<<grid, threads, 0, stream>>>(static_cast<const uint16_t *>(W), Cout, R, G, K,
+                                                                  counts);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // generic product: any G <= 256, any K, any alignment.  A CTA of 128 threads
 // owns one group and 128 columns; thread = column; the G accumulators of the
 // column live in shared memory acc[G][128] (the thread's own column only).

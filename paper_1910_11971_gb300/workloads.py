@@ -147,6 +147,35 @@ def resnet50_layers(batch: int = 128, G: int = 8, K: int = 2) -> List[ConvCase]:
     return layers
 
 
+def mobilenetv2_pointwise_layers(batch: int = 128, G: int = 8, K: int = 2) -> List[ConvCase]:
+    """The 34 pointwise (1x1) convolutions of MobileNetV2 (width 1.0, 224x224
+    input, torchvision layout): per inverted-residual block the expansion (when
+    the expansion factor is 6) at the block's input resolution and the projection
+    at its output resolution, then the final 1x1 320 -> 1280; the paper makes
+    these layers CCI-sparse (Sec. 4, Sec. 5; G = 8, K = 2 is its 75 % case)."""
+    layers: List[ConvCase] = []
+
+    def add(h, cin, cout):
+        i = len(layers)
+        layers.append(ConvCase(f"mobilenetv2_pw{i:02d}_{cin}to{cout}_h{h}", B=batch, H=h, W=h, Cin=cin,
+                               Cout=cout, KH=1, KW=1, stride=1, pad=0, G=G, K=K, dtype="bf16", seed=100 + i))
+
+    h, cin = 112, 32
+    for t, c, n, s in ((1, 16, 1, 1), (6, 24, 2, 2), (6, 32, 3, 2), (6, 64, 4, 2), (6, 96, 3, 1),
+                       (6, 160, 3, 2), (6, 320, 1, 1)):
+        for b in range(n):
+            stride = s if b == 0 else 1
+            hidden = cin * t
+            if t != 1:
+                add(h, cin, hidden)
+            h = (h + 2 - 3) // stride + 1  # the 3x3 depthwise convolution (not CCI)
+            add(h, hidden, c)
+            cin = c
+    add(h, cin, 1280)
+    assert len(layers) == 34
+    return layers
+
+
 def resnet50_roles() -> List[str]:
     """Role of each of the 52 layers of resnet50_layers() in its bottleneck block:
     'a' (1x1 reduce, reads the block input), 'b' (3x3, reads a's output), 'c' (1x1

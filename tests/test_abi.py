@@ -190,3 +190,15 @@ def test_fused_rejects(lib):
                                 FAKE, None, None, 0, None) == 11
     assert lib.cci_conv2d_fused(FAKE, 1, 1, 4, 4, 64, FAKE, FAKE, 64, 3, 3, 1, 1, 1, 1, 8, 2, None, 1, 7,
                                 FAKE, None, FAKE, 1 << 20, None) == DTYPE
+
+
+def test_pack_stats_rejects(lib):
+    s = lib.cci_pack_stats
+    assert s(FAKE, 5, 16, 8, 8, 2, FAKE, None) == DTYPE
+    assert s(None, 1, 16, 8, 8, 2, FAKE, None) == NULL
+    assert s(FAKE, 1, 16, 8, 8, 2, None, None) == NULL
+    assert s(FAKE, 1, 0, 8, 8, 2, FAKE, None) == SHAPE
+    assert s(FAKE, 1, 12, 8, 8, 2, FAKE, None) == GROUP
+    assert s(FAKE, 1, 16, 8, 8, 9, FAKE, None) == GROUP
+    assert s(FAKE + 1, 1, 16, 8, 8, 2, FAKE, None) == ALIGN
+    assert s(FAKE, 1, 16, 8, 8, 2, FAKE + 4, None) == ALIGN

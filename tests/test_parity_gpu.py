@@ -673,3 +673,41 @@ def test_fused_identity_equals_plain_product(dev):
     Yf = cci.linear_fused(Xd, v, i, Cout, G, K)
     Yp = cci.linear(Xd, v, i, Cout, G, K, algo=cci.ALGO_DENSE_TC_WS)
     assert torch.equal(Yf.view(torch.int32), Yp.view(torch.int32))
+
+
+# ---------------------------------------------------------------------------
+# allocation statistics of packing (Eq. 1 measured): exact counts against the
+# oracle, and the counted ratio against the closed form on independent zeros
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("Cout,R,G,K,Ps", [(64, 33, 8, 2, 0.75), (48, 1000, 16, 4, 0.5), (1024, 4096, 8, 2, 0.75),
+                                           (4, 7, 4, 1, 0.3), (512, 96, 32, 8, 0.9)])
+def test_pack_stats_exact(dev, dtype, Cout, R, G, K, Ps):
+    rng = np.random.default_rng(Cout + R + G)
+    W = rng.standard_normal((Cout, R)).astype(np.float32)
+    W[rng.random((Cout, R)) < Ps] = 0
+    W[-1, : min(R, 6)] = -0.0
+    Wt = torch.from_numpy(W).to(_dt(dtype))
+    counts = cci.pack_stats(Wt.to(dev), G, K)
+    got = counts.cpu().tolist()
+    assert got == list(oracle.pack_stats(f64(Wt), G, K))
+    cci.pack_stats(Wt.to(dev), G, K, counts=counts)  # accumulates
+    assert counts.cpu().tolist() == [2 * got[0], 2 * got[1]]
+
+
+@pytest.mark.parametrize("G,Ps", [(4, 0.5), (8, 0.75), (16, 0.875), (64, 0.75), (256, 0.9375)])
+def test_pack_stats_estimates_eq1(dev, G, Ps):
+    """Independent zeros with probability Ps, K = G(1 - Ps): the GPU-counted
+    dropped fraction is within 5 standard errors of Eq. 1."""
+    K = int(round(G * (1 - Ps)))
+    g = torch.Generator(device="cuda").manual_seed(G)
+    Cout, R = 4096, 8192
+    W = torch.randn((Cout, R), generator=g, device=dev)
+    W[torch.rand((Cout, R), generator=g, device=dev) < Ps] = 0
+    nz, dropped = cci.pack_stats(W, G, K).cpu().tolist()
+    groups = (Cout // G) * R
+    est = dropped / nz
+    pd = oracle.allocation_error(G, Ps)
+    # per group the overflow is at most G - K; its variance is bounded by E[over] * (G - K)
+    se = np.sqrt(pd * K * (G - K) / groups) / K
+    assert abs(est - pd) < 5 * se + 1e-9, (est, pd, se)
