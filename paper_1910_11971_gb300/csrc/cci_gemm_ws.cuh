@@ -66,7 +66,10 @@ struct AMaps {
 // CG = 2: a cluster of two CTAs computes a 256 x BN tile with tcgen05.mma
 // cta_group::2 issued by the even CTA; each CTA holds its 128 rows of A and half
 // of the BN rows of B (bf16 with TMA activations only)
-template <bool TF32, int ASRC, int BN, int CG>
+// EPI = 2: a second epilogue group (warps 4-7, idle when bf16 activations are
+// copied by TMA) and two staging buffers per group, for layers whose tiles have
+// few stages (the output write dominates); EPI = 1: one group, more stages
+template <bool TF32, int ASRC, int BN, int CG, int EPI>
 struct Cfg {
     static constexpr int kM = 128, kN = BN;
     static_assert(CG == 1 || (CG == 2 && !TF32 && ASRC != kAGather), "pair mode: bf16 with TMA activations");
@@ -81,13 +84,18 @@ struct Cfg {
     static constexpr int kBPlane = kBRows * 128;
     static constexpr int kStage = kAPlanes * kAPlane + kBPlanes * kBPlane;
     static constexpr int kYBuf = kM * 128;  // one output staging buffer: [128 rows][32 fp32]
-    static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - 2 * kYBuf - 1024;
+    // epilogue groups: warps 0-3, and warps 4-7 too when they have no producer work
+    // (TMA-copied bf16 activations); two staging buffers per group
+    static constexpr int kEG = (kATma && EPI == 2) ? 2 : 1;
+    static constexpr int kYBufs = 2 * kEG;
+    static_assert(EPI == 1 || EPI == 2, "epilogue groups");
+    static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - kYBufs * kYBuf - 1024;
     static constexpr int kStages = (kBudget / kStage) < tc::kMaxStages ? (kBudget / kStage) : tc::kMaxStages;
     // accumulators: 2 x kN columns; kARaw adds per stage A hi and A lo (32 columns each)
     static constexpr int kAColBase = 2 * kN;
     static constexpr int kTmemCols = kARaw ? 512 : 2 * kN;
     static constexpr size_t kSmem =
-        1024 + static_cast<size_t>(kStages) * kStage + 2 * kYBuf + sizeof(tc::Smem) + 64;
+        1024 + static_cast<size_t>(kStages) * kStage + kYBufs * kYBuf + sizeof(tc::Smem) + 64;
     static constexpr uint32_t kBBytes = kBPlanes * kBPlane;
     static constexpr uint32_t kIdesc = (1u << 4)                                           // D f32
                                        | (TF32 ? (2u << 7) | (2u << 10) : (1u << 7) | (1u << 10))  // tf32 / bf16
@@ -266,20 +274,20 @@ __device__ __forceinline__ BoxIdx box_of(int64_t mt, const ConvBox &box)
     return i;
 }
 
-template <bool TF32, int ASRC, int BN, int CG>
-__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
+template <bool TF32, int ASRC, int BN, int CG, int EPI>
+__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
     gemm_ws_kernel(FwdParams p, const __grid_constant__ AMaps tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmY, ConvBox box,
                    int64_t n_ct, int64_t n_tiles)
 {
-    using C = Cfg<TF32, ASRC, BN, CG>;
+    using C = Cfg<TF32, ASRC, BN, CG, EPI>;
     constexpr int kM = C::kM, kN = C::kN, kKS = C::kKS, kStages = C::kStages;
     constexpr int kLag = 2;  // bf16 gather: stages in flight before a producer's arrive
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const uint32_t raw = tc::smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
-    const uint32_t ybuf = base + kStages * C::kStage;  // two output staging buffers
-    tc::Smem *S = reinterpret_cast<tc::Smem *>(smem_raw + (base - raw) + kStages * C::kStage + 2 * C::kYBuf);
+    const uint32_t ybuf = base + kStages * C::kStage;  // output staging buffers, two per epilogue group
+    tc::Smem *S = reinterpret_cast<tc::Smem *>(smem_raw + (base - raw) + kStages * C::kStage + C::kYBufs * C::kYBuf);
     volatile int *abort = &S->abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nks = static_cast<int>((p.R + kKS - 1) / kKS);
@@ -409,7 +417,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
                 __syncwarp();
             }
         }
-    } else if (warp >= 4 && warp < 8) {
+    } else if (warp >= 4 && warp < 8 && C::kEG == 1) {
         // ------------------------------------------------------------ producers
         const int pt = tid - 128;
         const int chunk = pt & 7;  // 16-byte chunk of every activation row this thread handles
@@ -654,35 +662,35 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
         int no_abort = 0;
         tc::mbar_wait(&S->drain, 0, &no_abort, p.status);
     } else {
-        // ------------------------------------------------------------ epilogue (warps 0-3)
-        // Per chunk of one 128-byte output row (32 fp32 or 64 bf16 columns): TMEM ->
-        // registers (+ bias, ReLU, bf16 rounding when asked) -> swizzled staging
-        // buffer (row m = thread) -> one TMA store of the tile's box (rows past N,
-        // the image or Cout are clipped by the copy).  Two buffers alternate; a
-        // buffer is rewritten once the store issued from it two chunks earlier has
-        // read it.  Every decision that gates a named barrier is uniform over the
-        // 128 threads (named_and), so the barriers always see all of them.
-        int t = 0;
+        // ------------------------------------------------------------ epilogue (warps 0-3;
+        // with EPI = 2 also warps 4-7 as a second group: group g takes the tiles
+        // whose accumulator is g)
+        constexpr int kEG = C::kEG;
+        const int eg = warp >> 2;              // this thread's group
+        const int etid = tid - 128 * eg;       // thread within the group; 0 issues its stores
+        const int ebar = 1 + eg;               // the group's named barrier
+        int t = eg;
         bool ok = true;
-        const uint32_t lane_off = static_cast<uint32_t>(warp * 32) << 16;
-        const int m = tid;  // accumulator row = TMEM lane
+        const uint32_t lane_off = static_cast<uint32_t>((warp & 3) * 32) << 16;
+        const int m = etid;  // accumulator row = TMEM lane
         int chunk_no = 0;
         // CG = 2: the odd CTA releases an accumulator on the even CTA's barrier
         const uint32_t tmem_empty_remote = CG == 2 ? map_to_rank(tc::smem_u32(&S->tmem_empty[0]), 0) : 0u;
-        for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
+        for (int64_t u = u0 + eg * ustep; u < n_tiles && ok; u += kEG * ustep, t += kEG) {
             const int acc = t & 1;
             const int64_t mt = mtile(u);
             const int co0 = static_cast<int>((u % n_ct) * kN);
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d) bi = box_of(mt, box);
             ok = tc::mbar_wait(&S->tmem_full[acc], (t / 2) & 1, abort, p.status);
-            ok = tc::named_and(1, 128, ok);
+            ok = tc::named_and(ebar, 128, ok);
             if (!ok) break;
             __syncwarp();
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const int sc = p.out_bf16 ? 64 : 32;  // output columns per staged 128-byte row
+            const int cend = (p.Cout - co0) < kN ? static_cast<int>(p.Cout - co0) : kN;
 #pragma unroll 1
-            for (int c0 = 0; c0 < kN && co0 + c0 < p.Cout; c0 += sc, ++chunk_no) {
+            for (int c0 = 0; c0 < cend; c0 += sc, ++chunk_no) {
                 uint32_t v[32];
                 const uint32_t tcol = tmem + lane_off + static_cast<uint32_t>(acc * kN + c0);
                 if (!p.out_bf16) {
@@ -699,15 +707,25 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
 #pragma unroll
                     for (int j = 0; j < 16; ++j) v[16 + j] = bf16x2_rn(w[2 * j], w[2 * j + 1]);
                 }
-                const uint32_t buf = ybuf + static_cast<uint32_t>(chunk_no & 1) * C::kYBuf;
-                if (tid == 0) tc::bulk_wait_read<1>();
-                tc::named_sync(1, 128);
+                if (c0 + sc >= cend) {
+                    // the tile's accumulator is all in registers: release it to the MMAs
+                    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+                    if (CG == 2 && crank != 0)
+                        mbar_arrive_remote(tmem_empty_remote + static_cast<uint32_t>(acc * sizeof(uint64_t)));
+                    else
+                        tc::mbar_arrive(&S->tmem_empty[acc]);
+                }
+                // the group's two buffers alternate; a buffer is rewritten once the
+                // store issued from it two chunks earlier has read it
+                const uint32_t buf = ybuf + static_cast<uint32_t>(2 * eg + (chunk_no & 1)) * C::kYBuf;
+                if (etid == 0) tc::bulk_wait_read<1>();
+                tc::named_sync(ebar, 128);
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
                     st_shared_v4(buf + sw_chunk(m, q), v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                tc::named_sync(1, 128);
-                if (tid == 0) {
+                tc::named_sync(ebar, 128);
+                if (etid == 0) {
                     if constexpr (ASRC == kA4d)
                         tc::tma_store_4d(&tmY, buf, co0 + c0, bi.qb * box.QB, bi.pb * box.PB,
                                          static_cast<int>(bi.bb * box.BB));
@@ -716,13 +734,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG>::kThreads, 1)
                     tc::bulk_commit();
                 }
             }
-            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-            if (CG == 2 && crank != 0)
-                mbar_arrive_remote(tmem_empty_remote + static_cast<uint32_t>(acc * sizeof(uint64_t)));
-            else
-                tc::mbar_arrive(&S->tmem_empty[acc]);
         }
-        if (tid == 0) tc::bulk_wait_all();
+        if (etid == 0) tc::bulk_wait_all();
     }
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -882,11 +895,11 @@ inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn, int cg = 1)
     return best;
 }
 
-template <bool TF32, int ASRC, int BN, int CG>
+template <bool TF32, int ASRC, int BN, int CG, int EPI = 1>
 cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA, cudaStream_t stream)
 {
-    using C = Cfg<TF32, ASRC, BN, CG>;
-    auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG>;
+    using C = Cfg<TF32, ASRC, BN, CG, EPI>;
+    auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG, EPI>;
     static const cudaError_t attr =
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::kSmem));
     if (attr != cudaSuccess) return attr;

@@ -22,6 +22,20 @@ cudaError_t launch_gemm_ws_bf16(const FwdParams &p, cudaStream_t stream)
         return launch_cfg<false, kA4d, 256, 2>(p, pl.box, pl.am, stream);
     }
     const int bn = choose_bn(m_tiles, p.Cout, 256, 1);
+    // tiles of at most 4 stages: the output write dominates, two epilogue groups
+    // with two staging buffers each; longer ones keep the shared memory for stages
+    const bool short_k = nks <= 4 && asrc != kAGather;
+    if (short_k) {
+#define CCI_WS_SHORT(A, N) \
+    if (asrc == A && bn == N) return launch_cfg<false, A, N, 1, 2>(p, pl.box, pl.am, stream);
+        CCI_WS_SHORT(kA2d, 64)
+        CCI_WS_SHORT(kA2d, 128)
+        CCI_WS_SHORT(kA2d, 256)
+        CCI_WS_SHORT(kA4d, 64)
+        CCI_WS_SHORT(kA4d, 128)
+        CCI_WS_SHORT(kA4d, 256)
+#undef CCI_WS_SHORT
+    }
 #define CCI_WS_CASE(A, N) \
     if (asrc == A && bn == N) return launch_cfg<false, A, N, 1>(p, pl.box, pl.am, stream);
     CCI_WS_CASE(kA2d, 64)
