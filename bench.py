@@ -638,7 +638,32 @@ def run_extras(cci, dev, stream, flush):
     out["resnet50_stack"] = run_resnet_stack(cci, dev, stream, flush)
     out["mobilenetv2_pointwise"] = run_pointwise_stack(cci, dev, stream, flush)
     out["allocation_error"] = run_allocation_error(cci, dev, stream, flush)
+    out["td_mask"] = run_td_mask(cci, dev, stream, flush)
     return out
+
+
+def run_td_mask(cci, dev, stream, flush, reps=10):
+    """One targeted-dropout step (Sec. 5.1) on a 4096 x 8192 weight matrix, G = 8,
+    K = 2, rate 0.75, per dtype: bytes moved (W, uniforms, W_out, mask) against
+    the measured HBM copy bandwidth."""
+    res = []
+    Cout, R = 4096, 8192
+    for dt in (torch.float32, torch.bfloat16):
+        g = torch.Generator(device=str(dev)).manual_seed(11)
+        W = torch.randn((Cout, R), generator=g, device=dev).to(dt)
+        u = torch.rand((Cout, R), generator=g, device=dev)
+        Wo = torch.empty_like(W)
+        m = torch.empty((Cout, R), dtype=torch.uint8, device=dev)
+        fn = lambda: cci.td_mask(W, 8, 2, 0.75, u, out=Wo, mask=m)  # noqa: E731
+        fn()
+        ms = statistics.median(time_device(fn, reps, flush, stream))
+        nbytes = Cout * R * (2 * W.element_size() + 4 + 1)
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        res.append({"dtype": str(dt).replace("torch.", ""), "ms": ms, "gbs": gbs,
+                    "hbm_frac": gbs / float(measured_peaks()["hbm_gbs"]),
+                    "dropped_frac_of_candidates": float((m == 0).sum().item()) / (Cout * R * 6 / 8)})
+        del W, u, Wo, m
+    return res
 
 
 def run_pointwise_stack(cci, dev, stream, flush, reps=5):

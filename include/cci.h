@@ -199,6 +199,25 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
                          void *workspace, size_t workspace_bytes, cci_stream_t stream);
 
 /*
+ * cci_td_mask -- one step of the improved targeted dropout used to train CCI
+ * layers (Sec. 5.1).  Per group of G output channels at one input index r the K
+ * weights of largest |w| (those cci_pack keeps: same ranking, ties to the lower
+ * index) are protected; each other weight is a pruning candidate and is dropped
+ * for this training pass when its uniform draw is below `rate`:
+ *   W_out[co][r] = 0 if (co is a candidate and uniforms[co][r] < rate) else W[co][r]
+ *   mask[co][r]  = 1 if W_out keeps the weight, else 0      (mask may be NULL)
+ * The paper starts the candidate drop rate at 0.5 and raises it toward 1 during
+ * training (rate is the caller's schedule).  The random numbers are an input:
+ * uniforms[Cout][R] fp32 in [0, 1), device.  W, W_out: device [Cout][R] of dtype
+ * (W_out may not alias W); mask: device uint8 [Cout][R].  rate outside [0, 1]
+ * or NaN: CCI_ERR_VALUE; NaN weights are reported in dev_status as for cci_pack;
+ * other argument errors as for cci_pack.
+ */
+cci_status cci_td_mask(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K, float rate,
+                       const float *uniforms, void *W_out, uint8_t *mask, uint32_t *dev_status,
+                       cci_stream_t stream);
+
+/*
  * cci_pack_stats -- the allocation error of packing W (Sec. 4, Eq. 1, measured):
  * adds to counts[0] the number of nonzero weights of W[Cout][R] and to counts[1]
  * the number of them that cci_pack with (G, K) cannot keep (per group of G

@@ -201,6 +201,21 @@ def allocation_error_exact(G: int, Ps) -> Fraction:
     return total / si
 
 
+def td_mask(W, G: int, K: int, rate: float, u):
+    """Targeted dropout for CCI training (Sec. 5.1): the weights that packing keeps
+    are protected; each other weight (a pruning candidate) is dropped when its
+    uniform draw is below the rate (both compared as fp32).  Returns (W_out, mask)."""
+    W = _f64(W)
+    Cout, R = W.shape
+    _, idx = pack(W, G, K)
+    keep = np.zeros((Cout, R), dtype=bool)
+    for gi in range(Cout // G):
+        for s in range(K):
+            keep[gi * G + idx[gi, :, s].astype(np.int64), np.arange(R)] = True
+    drop = ~keep & (np.asarray(u, dtype=np.float32) < np.float32(rate))
+    return np.where(drop, 0.0, W), (~drop).astype(np.uint8)
+
+
 def pack_stats(W, G: int, K: int):
     """(nonzero weights of W[Cout][R], nonzero weights that packing with group size G
     and K slots cannot keep): per group (G consecutive output channels at one r,

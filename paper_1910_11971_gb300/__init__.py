@@ -52,6 +52,7 @@ SIGNATURES = {
                                 _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _P, _U32P, _P,
                                 ctypes.c_size_t, _P]),
     "cci_pack_stats": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, _P, _P]),
+    "cci_td_mask": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, ctypes.c_float, _P, _P, _P, _U32P, _P]),
     "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
     "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
                                           _P]),
@@ -222,6 +223,31 @@ def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
                                algo, wp, wb, _stream(X.device))
     _check(code, "cci_conv2d")
     return Y
+
+
+def td_mask(W: torch.Tensor, G: int, K: int, rate: float, uniforms: torch.Tensor, *,
+            out: Optional[torch.Tensor] = None, mask: Optional[torch.Tensor] = None,
+            status: Optional[torch.Tensor] = None):
+    """(W_out, mask) of one targeted-dropout step (``cci_td_mask``): candidates (the
+    weights packing would drop) zeroed where ``uniforms < rate``."""
+    _cuda_contig(W, "W")
+    _cuda_contig(uniforms, "uniforms")
+    Cout, R = W.shape
+    Wo = out if out is not None else torch.empty_like(W)
+    m = mask if mask is not None else torch.empty((Cout, R), dtype=torch.uint8, device=W.device)
+    _check(lib().cci_td_mask(W.data_ptr(), _dtype_code(W), Cout, R, G, K, float(rate), uniforms.data_ptr(),
+                             Wo.data_ptr(), m.data_ptr(), status.data_ptr() if status is not None else None,
+                             _stream(W.device)), "cci_td_mask")
+    return Wo, m
+
+
+def td_drop_rate(step: int, ramp_steps: int, start: float = 0.5, end: float = 1.0) -> float:
+    """The candidate drop rate of Sec. 5.1: from ``start`` (50 %) toward ``end``
+    (100 %); the paper fixes the end points only, the ramp here is linear over
+    ``ramp_steps`` steps and then constant."""
+    if ramp_steps <= 0:
+        return end
+    return start + (end - start) * min(max(step, 0) / ramp_steps, 1.0)
 
 
 def pack_stats(W: torch.Tensor, G: int, K: int, counts: Optional[torch.Tensor] = None) -> torch.Tensor:

@@ -246,6 +246,21 @@ cci_status conv_impl(const void *X, int dtype, int64_t B, int64_t H, int64_t W, 
 
 extern "C" {
 
+cci_status cci_td_mask(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K, float rate,
+                       const float *uniforms, void *W_out, uint8_t *mask, uint32_t *dev_status, cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!W || !uniforms || !W_out) return CCI_ERR_NULL;
+    if (Cout < 1 || R < 1 || !mul_ok(Cout, R)) return CCI_ERR_SHAPE;
+    const cci_status g = check_group(Cout, G, K);
+    if (g != CCI_OK) return g;
+    if (!(rate >= 0.0f && rate <= 1.0f)) return CCI_ERR_VALUE;  // also NaN
+    const size_t es = elem_size(dtype);
+    if (!aligned(W, es) || !aligned(W_out, es) || !aligned(uniforms, 4)) return CCI_ERR_ALIGN;
+    return to_status(launch_td_mask(W, dtype, Cout, R, G, K, rate, uniforms, W_out, mask, dev_status,
+                                    reinterpret_cast<cudaStream_t>(stream)));
+}
+
 cci_status cci_pack_stats(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K,
                           unsigned long long *counts, cci_stream_t stream)
 {

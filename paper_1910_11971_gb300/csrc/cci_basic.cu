@@ -1,4 +1,5 @@
-// cci_basic.cu -- the pack kernel, the generic product kernel and the FMA probe.
+// cci_basic.cu -- the pack kernel, the targeted-dropout mask, the allocation
+// statistics of packing, the generic product kernel and the FMA probe.
 #include "cci_kernels.h"
 
 namespace cci {
@@ -59,6 +60,62 @@ cudaError_t launch_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G
     else
         pack_kernel<uint16_t><<<grid, threads, 0, stream>>>(static_cast<const uint16_t *>(W), Cout, R, G, K,
                                                             static_cast<uint16_t *>(values), idx, status);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// targeted dropout for CCI training (Sec. 5.1): per (group, r) the K weights of
+// largest |w| (the ones pack keeps, same ranking and tie rule) are protected;
+// every other weight is a pruning candidate and is zeroed for this pass when
+// its uniform draw u < rate.  One thread per (group, r).
+// ---------------------------------------------------------------------------
+template <typename TB>
+__global__ void td_mask_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, int G, int K, float rate,
+                               const float *__restrict__ u, TB *__restrict__ Wout, uint8_t *__restrict__ mask,
+                               uint32_t *status)
+{
+    constexpr uint32_t kAbs = sizeof(TB) == 4 ? 0x7fffffffu : 0x7fffu;
+    constexpr uint32_t kInf = sizeof(TB) == 4 ? 0x7f800000u : 0x7f80u;
+    const int64_t total = (Cout / G) * R;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gi = t / R;
+        const int64_t r = t - gi * R;
+        const TB *col = W + gi * G * R + r;
+        bool nan = false;
+        for (int j = 0; j < G; ++j) {
+            const TB wj = col[static_cast<int64_t>(j) * R];
+            const uint32_t a = static_cast<uint32_t>(wj) & kAbs;
+            nan |= a > kInf;
+            int rank = 0;  // number of entries ranked ahead of j
+            for (int j2 = 0; j2 < G && rank < K; ++j2) {
+                const uint32_t b = static_cast<uint32_t>(col[static_cast<int64_t>(j2) * R]) & kAbs;
+                rank += (b > a) || (b == a && j2 < j);
+            }
+            const int64_t off = (gi * G + j) * R + r;
+            const bool keep = rank < K || !(u[off] < rate);
+            Wout[off] = keep ? wj : static_cast<TB>(0);
+            if (mask) mask[off] = keep ? 1 : 0;
+        }
+        if (nan) report(status, CCI_ERR_VALUE);
+    }
+}
+
+cudaError_t launch_td_mask(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K, float rate,
+                           const float *u, void *Wout, uint8_t *mask, uint32_t *status, cudaStream_t stream)
+{
+    const int64_t total = (Cout / G) * R;
+    const int threads = 256;
+    const int64_t blocks = (total + threads - 1) / threads;
+    const int grid = static_cast<int>(blocks < 65536 * 16 ? blocks : 65536 * 16);
+    if (dtype == CCI_F32)
+        td_mask_kernel<uint32_t><<<grid, threads, 0, stream>>>(static_cast<const uint32_t *>(W), Cout, R, G, K,
+                                                               rate, u, static_cast<uint32_t *>(Wout), mask,
+                                                               status);
+    else
+        td_mask_kernel<uint16_t><<<grid, threads, 0, stream>>>(static_cast<const uint16_t *>(W), Cout, R, G, K,
+                                                               rate, u, static_cast<uint16_t *>(Wout), mask,
+                                                               status);
     return cudaGetLastError();
 }
 

@@ -202,3 +202,17 @@ def test_pack_stats_rejects(lib):
     assert s(FAKE, 1, 16, 8, 8, 9, FAKE, None) == GROUP
     assert s(FAKE + 1, 1, 16, 8, 8, 2, FAKE, None) == ALIGN
     assert s(FAKE, 1, 16, 8, 8, 2, FAKE + 4, None) == ALIGN
+
+
+def test_td_mask_rejects(lib):
+    t = lib.cci_td_mask
+    assert t(FAKE, 5, 16, 8, 8, 2, 0.5, FAKE, FAKE, None, None, None) == DTYPE
+    assert t(None, 0, 16, 8, 8, 2, 0.5, FAKE, FAKE, None, None, None) == NULL
+    assert t(FAKE, 0, 16, 8, 8, 2, 0.5, None, FAKE, None, None, None) == NULL
+    assert t(FAKE, 0, 16, 8, 8, 2, 0.5, FAKE, None, None, None, None) == NULL
+    assert t(FAKE, 0, 16, 0, 8, 2, 0.5, FAKE, FAKE, None, None, None) == SHAPE
+    assert t(FAKE, 0, 12, 8, 8, 2, 0.5, FAKE, FAKE, None, None, None) == GROUP
+    assert t(FAKE, 0, 16, 8, 8, 2, 1.5, FAKE, FAKE, None, None, None) == VALUE
+    assert t(FAKE, 0, 16, 8, 8, 2, -0.1, FAKE, FAKE, None, None, None) == VALUE
+    assert t(FAKE, 0, 16, 8, 8, 2, float("nan"), FAKE, FAKE, None, None, None) == VALUE
+    assert t(FAKE + 2, 0, 16, 8, 8, 2, 0.5, FAKE, FAKE, None, None, None) == ALIGN
