@@ -639,7 +639,50 @@ def run_extras(cci, dev, stream, flush):
     out["mobilenetv2_pointwise"] = run_pointwise_stack(cci, dev, stream, flush)
     out["allocation_error"] = run_allocation_error(cci, dev, stream, flush)
     out["td_mask"] = run_td_mask(cci, dev, stream, flush)
+    out["cci_vs_bbs"] = run_cci_vs_bbs(cci, dev, stream, flush)
     return out
+
+
+def run_cci_vs_bbs(cci, dev, stream, flush, reps=5):
+    """The paper's comparison format (Sec. 3.4) on the same shapes: balanced
+    sparsity (groups of G inputs per output channel) against CCI (groups of G
+    output channels per input), each on the tensor cores (decompression + the
+    same GEMM) and on CUDA cores (BBS: gather kernel; CCI: branch-free expand and
+    jump dispatch)."""
+    res = []
+    shapes = [("sweep_4096_G8_K2", wl.sweep_case(8, 2)), ("sweep_4096_G16_K4", wl.sweep_case(16, 4)),
+              ("bottleneck_1x1", wl.BOTTLENECK_1X1)]
+    for name, case in shapes:
+        X, W = wl.linear_inputs(case, device=str(dev))
+        G, K = case.G, case.K
+        Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
+        ws = cci.new_workspace(cci.ALGO_DENSE_TC_WS, X.dtype, case.Cout, case.R, dev)
+        cv, ci = cci.pack(W, G, K)
+        bv, bi = cci.bbs_pack(W, G, K)
+        row = {"shape": name, "G": G, "K": K, "dtype": case.dtype, "nz_gflop": case.nz_flops() / 1e9}
+        runs = {
+            "cci_tc_ms": lambda: cci.linear(X, cv, ci, case.Cout, G, K, out=Y, algo=cci.ALGO_DENSE_TC_WS,
+                                            workspace=ws),
+            "bbs_tc_ms": lambda: cci.bbs_linear(X, bv, bi, case.Cout, G, K, out=Y, algo=cci.ALGO_DENSE_TC_WS,
+                                                workspace=ws),
+            "bbs_cuda_core_gather_ms": lambda: cci.bbs_linear(X, bv, bi, case.Cout, G, K, out=Y,
+                                                              algo=cci.ALGO_GENERIC),
+            "cci_cuda_core_expand_ms": lambda: cci.linear(X, cv, ci, case.Cout, G, K, out=Y, algo=cci.ALGO_EXPAND),
+            "cci_cuda_core_jump_ms": lambda: cci.linear(X, cv, ci, case.Cout, G, K, out=Y, algo=cci.ALGO_REGTILE),
+        }
+        for key, fn in runs.items():
+            try:
+                fn()
+            except Exception as e:  # a family without this (G, K) or shape
+                row[key] = None
+                row[key.replace("_ms", "_why")] = str(e)[:80]
+                continue
+            ms = statistics.median(time_device(fn, reps, flush, stream))
+            row[key] = ms
+            row[key.replace("_ms", "_nz_tflops")] = case.nz_flops() / (ms * 1e-3) / 1e12
+        res.append(row)
+        del X, W, Y, ws, cv, ci, bv, bi
+    return res
 
 
 def run_td_mask(cci, dev, stream, flush, reps=10):

@@ -218,6 +218,32 @@ cci_status cci_td_mask(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, 
                        cci_stream_t stream);
 
 /*
+ * Balanced sparsity (Sec. 3.4), the format the paper compares CCI with: groups
+ * run along the INPUT dimension.  Per output channel co and group of G
+ * consecutive inputs r in [g*G, g*G + G) (R % G == 0), K weights are kept.
+ *
+ * cci_bbs_pack -- values[Cout][R/G][K] (dtype) and idx[Cout][R/G][K] (uint8,
+ * offsets inside the group): the K of largest |w| per group, ties to the lower
+ * index, in increasing index (the selection rule of cci_pack).  Errors as for
+ * cci_pack; R % G != 0 is CCI_ERR_GROUP.
+ *
+ * cci_bbs_linear -- Y[N][Cout] fp32 = sum over groups and slots of
+ * values[co][g][k] * X[n][g*G + idx[co][g][k]] (the gather form of the product).
+ * algo CCI_ALGO_DENSE_TC_WS: decompression into the workspace and the tensor-core
+ * product of the CCI path (Cin % 8 bf16 / % 4 fp32, Cout % 4, 16-byte aligned X,
+ * Y and workspace of cci_workspace_size(CCI_ALGO_DENSE_TC_WS, dtype, Cout, Cin)
+ * bytes); CCI_ALGO_GENERIC: the CUDA-core gather kernel (32 % G == 0); AUTO: the
+ * first when the layer and workspace allow, else the second; other families:
+ * CCI_ERR_UNSUPPORTED.  Index sets must be strictly increasing and < G
+ * (CCI_ERR_INDEX in dev_status).  Everything else as for cci_linear_ws.
+ */
+cci_status cci_bbs_pack(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K, void *values,
+                        uint8_t *idx, uint32_t *dev_status, cci_stream_t stream);
+cci_status cci_bbs_linear(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+                          const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
+                          cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream);
+
+/*
  * cci_pack_stats -- the allocation error of packing W (Sec. 4, Eq. 1, measured):
  * adds to counts[0] the number of nonzero weights of W[Cout][R] and to counts[1]
  * the number of them that cci_pack with (G, K) cannot keep (per group of G

@@ -201,6 +201,38 @@ def allocation_error_exact(G: int, Ps) -> Fraction:
     return total / si
 
 
+def bbs_pack(W, G: int, K: int):
+    """Balanced sparsity (Sec. 3.4, the comparison format): per output channel co
+    and group of G consecutive inputs r in [g*G, g*G + G), the K weights of largest
+    |w| (ties to the lower index) in increasing index; values[Cout][R/G][K] and
+    idx[Cout][R/G][K] (offsets inside the group).  The same selection as CCI's
+    pack on the transposed matrix, whose groups of G rows are G inputs."""
+    W = _f64(W)
+    Cout, R = W.shape
+    if R % G:
+        raise OracleError(2, "bbs_pack")
+    v, i = pack(np.ascontiguousarray(W.T), G, K)  # [R/G][Cout][K]
+    return np.ascontiguousarray(v.transpose(1, 0, 2)), np.ascontiguousarray(i.transpose(1, 0, 2))
+
+
+def bbs_decompress(values, idx, R: int):
+    """Dense Wd[Cout][R] and mask of a balanced-sparse matrix (repeated indices add)."""
+    values = _f64(values)
+    idx = np.asarray(idx)
+    Cout, ng, K = values.shape
+    G = R // ng
+    Wd = np.zeros((Cout, R))
+    mask = np.zeros((Cout, R), dtype=np.int32)
+    for g in range(ng):
+        for s in range(K):
+            j = idx[:, g, s].astype(np.int64)
+            if (j >= G).any():
+                raise OracleError(6, "bbs_decompress")
+            np.add.at(Wd, (np.arange(Cout), g * G + j), values[:, g, s])
+            np.add.at(mask, (np.arange(Cout), g * G + j), 1)
+    return Wd, mask
+
+
 def td_mask(W, G: int, K: int, rate: float, u):
     """Targeted dropout for CCI training (Sec. 5.1): the weights that packing keeps
     are protected; each other weight (a pruning candidate) is dropped when its

@@ -52,6 +52,9 @@ SIGNATURES = {
                                 _I32, _I32, _I32, _I32, _I32, _P, _I32, _I32, _P, _U32P, _P,
                                 ctypes.c_size_t, _P]),
     "cci_pack_stats": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, _P, _P]),
+    "cci_bbs_pack": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, _P, _P, _U32P, _P]),
+    "cci_bbs_linear": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P, _I32, _P,
+                              ctypes.c_size_t, _P]),
     "cci_td_mask": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, ctypes.c_float, _P, _P, _P, _U32P, _P]),
     "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
     "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
@@ -222,6 +225,36 @@ def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
                                G, K, Y.data_ptr(), status.data_ptr() if status is not None else None,
                                algo, wp, wb, _stream(X.device))
     _check(code, "cci_conv2d")
+    return Y
+
+
+def bbs_pack(W: torch.Tensor, G: int, K: int, *, status: Optional[torch.Tensor] = None):
+    """(values[Cout][R/G][K], idx[Cout][R/G][K]) of the balanced-sparse form of W
+    (groups of G consecutive inputs; ``cci_bbs_pack``)."""
+    _cuda_contig(W, "W")
+    Cout, R = W.shape
+    values = torch.empty((Cout, R // G, K), dtype=W.dtype, device=W.device)
+    idx = torch.empty((Cout, R // G, K), dtype=torch.uint8, device=W.device)
+    _check(lib().cci_bbs_pack(W.data_ptr(), _dtype_code(W), Cout, R, G, K, values.data_ptr(), idx.data_ptr(),
+                              status.data_ptr() if status is not None else None, _stream(W.device)),
+           "cci_bbs_pack")
+    return values, idx
+
+
+def bbs_linear(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int, *,
+               out: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
+               algo: int = ALGO_AUTO, workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Y[N][Cout] (fp32) = the balanced-sparse product (``cci_bbs_linear``); with AUTO
+    or ALGO_DENSE_TC_WS and no workspace, one is allocated here."""
+    _cuda_contig(X, "X")
+    N, Cin = X.shape
+    if workspace is None and algo in (ALGO_AUTO, ALGO_DENSE_TC_WS):
+        workspace = new_workspace(ALGO_DENSE_TC_WS, X.dtype, Cout, Cin, X.device)
+    Y = out if out is not None else torch.empty((N, Cout), dtype=torch.float32, device=X.device)
+    wp, wb = _ws(workspace)
+    _check(lib().cci_bbs_linear(X.data_ptr(), _dtype_code(X), N, Cin, values.data_ptr(), idx.data_ptr(), Cout,
+                                G, K, Y.data_ptr(), status.data_ptr() if status is not None else None, algo, wp,
+                                wb, _stream(X.device)), "cci_bbs_linear")
     return Y
 
 

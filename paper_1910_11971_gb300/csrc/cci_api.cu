@@ -261,6 +261,63 @@ cci_status cci_td_mask(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, 
                                     reinterpret_cast<cudaStream_t>(stream)));
 }
 
+cci_status cci_bbs_pack(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K, void *values,
+                        uint8_t *idx, uint32_t *dev_status, cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!W || !values || !idx) return CCI_ERR_NULL;
+    if (Cout < 1 || R < 1 || !mul_ok(Cout, R)) return CCI_ERR_SHAPE;
+    if (G < 1 || G > 256 || K < 1 || K > G || R % G != 0) return CCI_ERR_GROUP;
+    const size_t es = elem_size(dtype);
+    if (!aligned(W, es) || !aligned(values, es)) return CCI_ERR_ALIGN;
+    return to_status(launch_bbs_pack(W, dtype, Cout, R, G, K, values, idx, dev_status,
+                                     reinterpret_cast<cudaStream_t>(stream)));
+}
+
+cci_status cci_bbs_linear(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *values,
+                          const uint8_t *idx, int64_t Cout, int G, int K, float *Y, uint32_t *dev_status,
+                          cci_algo algo, void *workspace, size_t workspace_bytes, cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!values || !idx) return CCI_ERR_NULL;
+    if (N > 0 && (!X || !Y)) return CCI_ERR_NULL;
+    if (N < 0 || Cout < 1 || Cin < 1 || !mul_ok(N, Cout) || !mul_ok(N, Cin) || !mul_ok(Cout, Cin))
+        return CCI_ERR_SHAPE;
+    if (G < 1 || G > 256 || K < 1 || K > G || Cin % G != 0) return CCI_ERR_GROUP;
+    const size_t es = elem_size(dtype);
+    if (!aligned(values, es) || (X && !aligned(X, es)) || (Y && !aligned(Y, 4))) return CCI_ERR_ALIGN;
+    FwdParams p{};
+    p.X = X;
+    p.values = values;
+    p.idx = idx;
+    p.Y = Y;
+    p.status = dev_status;
+    p.N = N;
+    p.Cout = Cout;
+    p.R = Cin;
+    p.Cin = Cin;
+    p.H = p.W = p.P = p.Q = 1;
+    p.KH = p.KW = p.sh = p.sw = 1;
+    const int64_t v = dtype == CCI_F32 ? 4 : 8;  // elements per 16 bytes
+    const bool tc_ok = Cin % v == 0 && Cin < (int64_t(1) << 31) && Cout < (int64_t(1) << 31) &&
+                       Cout % 4 == 0 && aligned(X, 16) && aligned(Y, 16);
+    const bool ws_ok = workspace && workspace_bytes >= dense_ws_bytes(dtype, Cout, Cin) && aligned(workspace, 16);
+    if (algo == CCI_ALGO_AUTO) algo = (tc_ok && ws_ok) ? CCI_ALGO_DENSE_TC_WS : CCI_ALGO_GENERIC;
+    if (algo == CCI_ALGO_DENSE_TC_WS) {
+        if (!tc_ok) return CCI_ERR_UNSUPPORTED;
+        if (!ws_ok) return CCI_ERR_WORKSPACE;
+        if (N == 0) return CCI_OK;
+        p.wdense = workspace;
+        const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+        const cudaError_t e = launch_bbs_decompress(p, dtype, G, K, s);
+        if (e != cudaSuccess) return CCI_ERR_CUDA;
+        return to_status(launch_gemm_ws(p, dtype, s));
+    }
+    if (algo != CCI_ALGO_GENERIC || 32 % G != 0) return CCI_ERR_UNSUPPORTED;
+    if (N == 0) return CCI_OK;
+    return to_status(launch_bbs_gather(p, dtype, G, K, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 cci_status cci_pack_stats(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K,
                           unsigned long long *counts, cci_stream_t stream)
 {

@@ -9,6 +9,11 @@ cudaError_t launch_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G
                         uint8_t *idx, uint32_t *status, cudaStream_t stream);
 cudaError_t launch_td_mask(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K, float rate,
                            const float *u, void *Wout, uint8_t *mask, uint32_t *status, cudaStream_t stream);
+// balanced sparsity, the comparison format (cci_bbs.cu)
+cudaError_t launch_bbs_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K, void *values,
+                            uint8_t *idx, uint32_t *status, cudaStream_t stream);
+cudaError_t launch_bbs_decompress(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);
+cudaError_t launch_bbs_gather(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);
 cudaError_t launch_pack_stats(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K,
                               unsigned long long *counts, cudaStream_t stream);
 cudaError_t launch_generic(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);

@@ -216,3 +216,18 @@ def test_td_mask_rejects(lib):
     assert t(FAKE, 0, 16, 8, 8, 2, -0.1, FAKE, FAKE, None, None, None) == VALUE
     assert t(FAKE, 0, 16, 8, 8, 2, float("nan"), FAKE, FAKE, None, None, None) == VALUE
     assert t(FAKE + 2, 0, 16, 8, 8, 2, 0.5, FAKE, FAKE, None, None, None) == ALIGN
+
+
+def test_bbs_rejects(lib):
+    p, f = lib.cci_bbs_pack, lib.cci_bbs_linear
+    assert p(FAKE, 5, 16, 64, 8, 2, FAKE, FAKE, None, None) == DTYPE
+    assert p(None, 1, 16, 64, 8, 2, FAKE, FAKE, None, None) == NULL
+    assert p(FAKE, 1, 16, 60, 8, 2, FAKE, FAKE, None, None) == GROUP   # R % G
+    assert p(FAKE, 1, 16, 64, 8, 9, FAKE, FAKE, None, None) == GROUP
+    assert p(FAKE, 1, 0, 64, 8, 2, FAKE, FAKE, None, None) == SHAPE
+    assert p(FAKE + 1, 1, 16, 64, 8, 2, FAKE, FAKE, None, None) == ALIGN
+    assert f(FAKE, 1, 16, 60, FAKE, FAKE, 16, 8, 2, FAKE, None, 0, None, 0, None) == GROUP
+    assert f(FAKE, 1, 16, 64, FAKE, FAKE, 16, 64, 2, FAKE, None, 1, None, 0, None) == UNSUP  # gather: 32 % G
+    assert f(FAKE, 1, 16, 64, FAKE, FAKE, 16, 8, 2, FAKE, None, 2, None, 0, None) == UNSUP  # no such family
+    assert f(FAKE, 1, 16, 64, FAKE, FAKE, 16, 8, 2, FAKE, None, 5, None, 0, None) == 11     # workspace
+    assert f(FAKE, 1, 0, 64, FAKE, FAKE, 16, 8, 2, None, None, 1, None, 0, None) == OK      # empty
