@@ -58,7 +58,10 @@ __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
 
 // SPLIT: fp32 hi plane to w0, lo plane to w1; else the weights to w0.  Indices
 // must be strictly increasing inside a group and < G (else CCI_ERR_INDEX).
-template <typename TB, bool SPLIT>
+// GC > 0: G == GC known at compile time, the group assembled in registers and
+// written with 16-byte stores (G * element size a multiple of 16); GC == 0: any
+// G, element stores.
+template <typename TB, bool SPLIT, int GC>
 __global__ void bbs_decompress_kernel(const TB *__restrict__ values, const uint8_t *__restrict__ idx, int64_t Cout,
                                       int64_t R, int G, int K, TB *__restrict__ w0, TB *__restrict__ w1,
                                       uint32_t *status)
@@ -70,25 +73,62 @@ __global__ void bbs_decompress_kernel(const TB *__restrict__ values, const uint8
         const int64_t base = (t / ng) * R + (t % ng) * G;
         int s = 0, prev = -1;
         bool bad = false;
-        for (int j = 0; j < G; ++j) {
-            TB v = 0;
-            if (s < K) {
-                const int ij = idx[t * K + s];
-                bad |= ij >= G || ij <= prev;
-                if (ij == j) {
+        if constexpr (GC > 0) {
+            TB g[GC];
+            int ij = K > 0 ? idx[t * K] : -1;
+#pragma unroll
+            for (int j = 0; j < GC; ++j) {
+                TB v = 0;
+                if (s < K && ij == j) {
                     v = values[t * K + s];
+                    bad |= ij <= prev;
                     prev = ij;
                     ++s;
+                    ij = s < K ? idx[t * K + s] : -1;
+                }
+                g[j] = v;
+            }
+            bad |= s < K;  // an index >= G or out of order was never reached
+            constexpr int kV = 16 / static_cast<int>(sizeof(TB));  // elements per 16-byte store
+#pragma unroll
+            for (int q = 0; q < GC / kV; ++q) {
+                uint32_t h[4], l[4];
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    uint32_t word;
+                    if constexpr (sizeof(TB) == 4)
+                        word = static_cast<uint32_t>(g[q * kV + e]);
+                    else
+                        word = static_cast<uint32_t>(g[q * kV + 2 * e]) |
+                               (static_cast<uint32_t>(g[q * kV + 2 * e + 1]) << 16);
+                    h[e] = SPLIT ? hi_bits(word) : word;
+                    l[e] = SPLIT ? lo_bits(word) : 0u;
+                }
+                reinterpret_cast<uint4 *>(w0 + base)[q] = make_uint4(h[0], h[1], h[2], h[3]);
+                if constexpr (SPLIT) reinterpret_cast<uint4 *>(w1 + base)[q] = make_uint4(l[0], l[1], l[2], l[3]);
+            }
+        } else {
+            for (int j = 0; j < G; ++j) {
+                TB v = 0;
+                if (s < K) {
+                    const int ij = idx[t * K + s];
+                    bad |= ij >= G || ij <= prev;
+                    if (ij == j) {
+                        v = values[t * K + s];
+                        prev = ij;
+                        ++s;
+                    }
+                }
+                if constexpr (SPLIT) {
+                    w0[base + j] = hi_bits(v);
+                    w1[base + j] = lo_bits(v);
+                } else {
+                    w0[base + j] = v;
                 }
             }
-            if constexpr (SPLIT) {
-                w0[base + j] = hi_bits(v);
-                w1[base + j] = lo_bits(v);
-            } else {
-                w0[base + j] = v;
-            }
+            bad |= s < K;
         }
-        if (bad || s < K) report(status, CCI_ERR_INDEX);
+        if (bad) report(status, CCI_ERR_INDEX);
     }
 }
 
@@ -208,17 +248,31 @@ cudaError_t launch_bbs_pack(const void *W, int dtype, int64_t Cout, int64_t R, i
     return cudaGetLastError();
 }
 
+template <typename TB, bool SPLIT, int GC>
+static void bbs_decompress_launch(const FwdParams &p, int G, int K, int grid, cudaStream_t stream)
+{
+    TB *w0 = static_cast<TB *>(const_cast<void *>(p.wdense));
+    bbs::bbs_decompress_kernel<TB, SPLIT, GC><<<grid, 256, 0, stream>>>(
+        static_cast<const TB *>(p.values), p.idx, p.Cout, p.R, G, K, w0, SPLIT ? w0 + p.Cout * p.R : nullptr,
+        p.status);
+}
+
 cudaError_t launch_bbs_decompress(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream)
 {
     const int grid = grid_of(p.Cout * (p.R / G));
+    // the workspace is 16-byte aligned and R is a multiple of G, so every group
+    // of G * element size (a multiple of 16) bytes starts 16-byte aligned
     if (dtype == CCI_F32) {
-        uint32_t *w0 = static_cast<uint32_t *>(const_cast<void *>(p.wdense));
-        bbs::bbs_decompress_kernel<uint32_t, true><<<grid, 256, 0, stream>>>(
-            static_cast<const uint32_t *>(p.values), p.idx, p.Cout, p.R, G, K, w0, w0 + p.Cout * p.R, p.status);
+        if (G == 4) bbs_decompress_launch<uint32_t, true, 4>(p, G, K, grid, stream);
+        else if (G == 8) bbs_decompress_launch<uint32_t, true, 8>(p, G, K, grid, stream);
+        else if (G == 16) bbs_decompress_launch<uint32_t, true, 16>(p, G, K, grid, stream);
+        else if (G == 32) bbs_decompress_launch<uint32_t, true, 32>(p, G, K, grid, stream);
+        else bbs_decompress_launch<uint32_t, true, 0>(p, G, K, grid, stream);
     } else {
-        bbs::bbs_decompress_kernel<uint16_t, false><<<grid, 256, 0, stream>>>(
-            static_cast<const uint16_t *>(p.values), p.idx, p.Cout, p.R, G, K,
-            static_cast<uint16_t *>(const_cast<void *>(p.wdense)), nullptr, p.status);
+        if (G == 8) bbs_decompress_launch<uint16_t, false, 8>(p, G, K, grid, stream);
+        else if (G == 16) bbs_decompress_launch<uint16_t, false, 16>(p, G, K, grid, stream);
+        else if (G == 32) bbs_decompress_launch<uint16_t, false, 32>(p, G, K, grid, stream);
+        else bbs_decompress_launch<uint16_t, false, 0>(p, G, K, grid, stream);
     }
     return cudaGetLastError();
 }
