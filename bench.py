@@ -76,8 +76,8 @@ def parse():
                     help="only the warm-up and timed steps of the main path (for ncu)")
     ap.add_argument("--workload", default="bottleneck_1x1",
                     help="bottleneck_1x1 (default) or sweep_4096_G<G>_K<K>: the product timed; with "
-                         "--profile 1 also a convolution: conv3x3_28 or resnet50_lNN_K<K> (layer NN of "
-                         "the ResNet-50 stack)")
+                         "--profile 1 also a convolution: conv3x3_28, resnet50_lNN_K<K> (layer NN of "
+                         "the ResNet-50 stack) or mobilenetv2_pwNN (pointwise layer NN of MobileNetV2)")
     return ap.parse_args()
 
 
@@ -365,6 +365,8 @@ def conv_case(name: str):
     if name.startswith("resnet50_l") and "_K" in name:
         li, k = name[len("resnet50_l"):].split("_K")
         return wl.resnet50_layers(K=int(k))[int(li)]
+    if name.startswith("mobilenetv2_pw"):
+        return wl.mobilenetv2_pointwise_layers()[int(name[len("mobilenetv2_pw"):])]
     return None
 
 

@@ -296,7 +296,12 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
     // the CTAs (CG = 1) or the CTA pairs (CG = 2)
     const int64_t u0 = CG == 2 ? blockIdx.x / 2 : blockIdx.x;
     const int64_t ustep = CG == 2 ? gridDim.x / 2 : gridDim.x;
-    auto mtile = [&](int64_t u) -> int64_t { return CG == 2 ? 2 * (u / n_ct) + crank : u / n_ct; };
+    // unit u -> (M tile, N tile): one 64-bit division, the remainder by multiply-subtract
+    auto split_unit = [&](int64_t u, int64_t &mt, int64_t &ct) {
+        const int64_t q = u / n_ct;
+        ct = u - q * n_ct;
+        mt = CG == 2 ? 2 * q + crank : q;
+    };
 
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -361,8 +366,9 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
         int it = 0;
         bool ok = true;
         for (int64_t u = u0; u < n_tiles && ok; u += ustep) {
-            const int64_t mt = mtile(u);
-            const int64_t co0 = (u % n_ct) * kN + crank * C::kBRows;  // this CTA's B rows
+            int64_t mt, ct;
+            split_unit(u, mt, ct);
+            const int64_t co0 = ct * kN + crank * C::kBRows;  // this CTA's B rows
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d) bi = box_of(mt, box);
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
@@ -678,8 +684,9 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
         const uint32_t tmem_empty_remote = CG == 2 ? map_to_rank(tc::smem_u32(&S->tmem_empty[0]), 0) : 0u;
         for (int64_t u = u0 + eg * ustep; u < n_tiles && ok; u += kEG * ustep, t += kEG) {
             const int acc = t & 1;
-            const int64_t mt = mtile(u);
-            const int co0 = static_cast<int>((u % n_ct) * kN);
+            int64_t mt, ct;
+            split_unit(u, mt, ct);
+            const int co0 = static_cast<int>(ct * kN);
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d) bi = box_of(mt, box);
             ok = tc::mbar_wait(&S->tmem_full[acc], (t / 2) & 1, abort, p.status);
