@@ -5,7 +5,8 @@
 namespace cci {
 
 // ---------------------------------------------------------------------------
-// pack: one thread per (group gi, input feature r).  Sec. 3.1 / Sec. 5.1:
+// pack: one thread per (group gi, input feature r); this general form takes
+// any G <= 256 and re-reads the column from cache while ranking.  Sec. 3.1 / Sec. 5.1:
 // the K weights of largest |w| in W[gi*G .. gi*G+G)[r] survive, ties to the
 // lower index, and are written in increasing index.  |w| is compared on the
 // storage bits with the sign cleared (an order-preserving integer compare for
@@ -47,20 +48,76 @@ __global__ void pack_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, i
     }
 }
 
+// Register form for the group sizes of every workload (G <= 32, a power of
+// two): the G entries of the column are loaded once, coalesced across the
+// warp (consecutive threads take consecutive r), and ranked in registers.
+template <typename TB, int GT>
+__global__ void __launch_bounds__(128) pack_reg_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, int K,
+                                                       TB *__restrict__ values, uint8_t *__restrict__ idx,
+                                                       uint32_t *status)
+{
+    constexpr uint32_t kAbs = sizeof(TB) == 4 ? 0x7fffffffu : 0x7fffu;
+    constexpr uint32_t kInf = sizeof(TB) == 4 ? 0x7f800000u : 0x7f80u;
+    const int64_t total = (Cout / GT) * R;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gi = t / R;
+        const int64_t r = t - gi * R;
+        const TB *col = W + gi * GT * R + r;
+        TB w[GT];
+        uint32_t a[GT];
+#pragma unroll
+        for (int j = 0; j < GT; ++j) {
+            w[j] = __ldg(col + static_cast<int64_t>(j) * R);
+            a[j] = static_cast<uint32_t>(w[j]) & kAbs;
+        }
+        bool nan = false;
+        int s = 0;
+#pragma unroll
+        for (int j = 0; j < GT; ++j) {
+            nan |= a[j] > kInf;
+            int rank = 0;  // entries ranked ahead of j: larger |w|, or equal |w| at a lower index
+#pragma unroll
+            for (int j2 = 0; j2 < GT; ++j2)
+                rank += j2 < j ? (a[j2] >= a[j]) : (a[j2] > a[j]);
+            if (rank < K) {
+                values[t * K + s] = w[j];
+                idx[t * K + s] = static_cast<uint8_t>(j);
+                ++s;
+            }
+        }
+        if (nan) report(status, CCI_ERR_VALUE);
+    }
+}
+
+template <typename TB>
+cudaError_t launch_pack_t(const TB *W, int64_t Cout, int64_t R, int G, int K, TB *values, uint8_t *idx,
+                          uint32_t *status, cudaStream_t stream)
+{
+    const int64_t total = (Cout / G) * R;
+    const bool reg = G == 2 || G == 4 || G == 8 || G == 16 || G == 32;
+    const int threads = reg ? 128 : 256;
+    const int64_t blocks = (total + threads - 1) / threads;
+    const int grid = static_cast<int>(blocks < 65536 * 16 ? blocks : 65536 * 16);
+    switch (reg ? G : 0) {
+        case 2: pack_reg_kernel<TB, 2><<<grid, threads, 0, stream>>>(W, Cout, R, K, values, idx, status); break;
+        case 4: pack_reg_kernel<TB, 4><<<grid, threads, 0, stream>>>(W, Cout, R, K, values, idx, status); break;
+        case 8: pack_reg_kernel<TB, 8><<<grid, threads, 0, stream>>>(W, Cout, R, K, values, idx, status); break;
+        case 16: pack_reg_kernel<TB, 16><<<grid, threads, 0, stream>>>(W, Cout, R, K, values, idx, status); break;
+        case 32: pack_reg_kernel<TB, 32><<<grid, threads, 0, stream>>>(W, Cout, R, K, values, idx, status); break;
+        default: pack_kernel<TB><<<grid, threads, 0, stream>>>(W, Cout, R, G, K, values, idx, status);
+    }
+    return cudaGetLastError();
+}
+
 cudaError_t launch_pack(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K, void *values,
                         uint8_t *idx, uint32_t *status, cudaStream_t stream)
 {
-    const int64_t total = (Cout / G) * R;
-    const int threads = 256;
-    const int64_t blocks = (total + threads - 1) / threads;
-    const int grid = static_cast<int>(blocks < 65536 * 16 ? blocks : 65536 * 16);
     if (dtype == CCI_F32)
-        pack_kernel<uint32_t><<<grid, threads, 0, stream>>>(static_cast<const uint32_t *>(W), Cout, R, G, K,
-                                                            static_cast<uint32_t *>(values), idx, status);
-    else
-        pack_kernel<uint16_t><<<grid, threads, 0, stream>>>(static_cast<const uint16_t *>(W), Cout, R, G, K,
-                                                            static_cast<uint16_t *>(values), idx, status);
-    return cudaGetLastError();
+        return launch_pack_t(static_cast<const uint32_t *>(W), Cout, R, G, K, static_cast<uint32_t *>(values), idx,
+                             status, stream);
+    return launch_pack_t(static_cast<const uint16_t *>(W), Cout, R, G, K, static_cast<uint16_t *>(values), idx,
+                         status, stream);
 }
 
 // ---------------------------------------------------------------------------
@@ -101,22 +158,79 @@ __global__ void td_mask_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R
     }
 }
 
+// Register form of the same step for G <= 32, a power of two: the column and
+// its G uniform draws are loaded once (all loads in flight together) and the
+// ranking runs in registers.
+template <typename TB, int GT>
+__global__ void __launch_bounds__(128) td_mask_reg_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, int K,
+                                                          float rate, const float *__restrict__ u,
+                                                          TB *__restrict__ Wout, uint8_t *__restrict__ mask,
+                                                          uint32_t *status)
+{
+    constexpr uint32_t kAbs = sizeof(TB) == 4 ? 0x7fffffffu : 0x7fffu;
+    constexpr uint32_t kInf = sizeof(TB) == 4 ? 0x7f800000u : 0x7f80u;
+    const int64_t total = (Cout / GT) * R;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t gi = t / R;
+        const int64_t r = t - gi * R;
+        const int64_t base = gi * GT * R + r;
+        TB w[GT];
+        float uj[GT];
+        uint32_t a[GT];
+#pragma unroll
+        for (int j = 0; j < GT; ++j) {
+            w[j] = __ldg(W + base + static_cast<int64_t>(j) * R);
+            uj[j] = __ldg(u + base + static_cast<int64_t>(j) * R);
+            a[j] = static_cast<uint32_t>(w[j]) & kAbs;
+        }
+        bool nan = false;
+#pragma unroll
+        for (int j = 0; j < GT; ++j) {
+            nan |= a[j] > kInf;
+            int rank = 0;  // entries ranked ahead of j: larger |w|, or equal |w| at a lower index
+#pragma unroll
+            for (int j2 = 0; j2 < GT; ++j2)
+                rank += j2 < j ? (a[j2] >= a[j]) : (a[j2] > a[j]);
+            const bool keep = rank < K || !(uj[j] < rate);
+            const int64_t off = base + static_cast<int64_t>(j) * R;
+            Wout[off] = keep ? w[j] : static_cast<TB>(0);
+            if (mask) mask[off] = keep ? 1 : 0;
+        }
+        if (nan) report(status, CCI_ERR_VALUE);
+    }
+}
+
+template <typename TB>
+cudaError_t launch_td_mask_t(const TB *W, int64_t Cout, int64_t R, int G, int K, float rate, const float *u,
+                             TB *Wout, uint8_t *mask, uint32_t *status, cudaStream_t stream)
+{
+    const int64_t total = (Cout / G) * R;
+    const bool reg = G == 2 || G == 4 || G == 8 || G == 16 || G == 32;
+    const int threads = reg ? 128 : 256;
+    const int64_t blocks = (total + threads - 1) / threads;
+    const int grid = static_cast<int>(blocks < 65536 * 16 ? blocks : 65536 * 16);
+#define CCI_TD(GV) td_mask_reg_kernel<TB, GV><<<grid, threads, 0, stream>>>(W, Cout, R, K, rate, u, Wout, mask, status)
+    switch (reg ? G : 0) {
+        case 2: CCI_TD(2); break;
+        case 4: CCI_TD(4); break;
+        case 8: CCI_TD(8); break;
+        case 16: CCI_TD(16); break;
+        case 32: CCI_TD(32); break;
+        default: td_mask_kernel<TB><<<grid, threads, 0, stream>>>(W, Cout, R, G, K, rate, u, Wout, mask, status);
+    }
+#undef CCI_TD
+    return cudaGetLastError();
+}
+
 cudaError_t launch_td_mask(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K, float rate,
                            const float *u, void *Wout, uint8_t *mask, uint32_t *status, cudaStream_t stream)
 {
-    const int64_t total = (Cout / G) * R;
-    const int threads = 256;
-    const int64_t blocks = (total + threads - 1) / threads;
-    const int grid = static_cast<int>(blocks < 65536 * 16 ? blocks : 65536 * 16);
     if (dtype == CCI_F32)
-        td_mask_kernel<uint32_t><<<grid, threads, 0, stream>>>(static_cast<const uint32_t *>(W), Cout, R, G, K,
-                                                               rate, u, static_cast<uint32_t *>(Wout), mask,
-                                                               status);
-    else
-        td_mask_kernel<uint16_t><<<grid, threads, 0, stream>>>(static_cast<const uint16_t *>(W), Cout, R, G, K,
-                                                               rate, u, static_cast<uint16_t *>(Wout), mask,
-                                                               status);
-    return cudaGetLastError();
+        return launch_td_mask_t(static_cast<const uint32_t *>(W), Cout, R, G, K, rate, u,
+                                static_cast<uint32_t *>(Wout), mask, status, stream);
+    return launch_td_mask_t(static_cast<const uint16_t *>(W), Cout, R, G, K, rate, u, static_cast<uint16_t *>(Wout),
+                            mask, status, stream);
 }
 
 // ---------------------------------------------------------------------------
@@ -125,11 +239,12 @@ cudaError_t launch_td_mask(const void *W, int dtype, int64_t Cout, int64_t R, in
 // one thread per (group, r), warp sums, one 64-bit atomic per warp and counter.
 // A weight is nonzero when its magnitude bits are (so -0 is zero).
 // ---------------------------------------------------------------------------
-template <typename TB>
-__global__ void pack_stats_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, int G, int K,
+template <typename TB, int GT>  // GT = G known at compile time (all G loads in flight), or 0
+__global__ void pack_stats_kernel(const TB *__restrict__ W, int64_t Cout, int64_t R, int G_, int K,
                                   unsigned long long *counts)
 {
     constexpr uint32_t kMag = sizeof(TB) == 4 ? 0x7fffffffu : 0x7fffu;
+    const int G = GT ? GT : G_;
     const int64_t total = (Cout / G) * R;
     uint32_t nz_sum = 0, drop_sum = 0;
     for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
@@ -137,7 +252,8 @@ __global__ void pack_stats_kernel(const TB *__restrict__ W, int64_t Cout, int64_
         const int64_t gi = t / R, r = t - gi * R;
         const TB *w = W + gi * G * R + r;
         int nz = 0;
-        for (int j = 0; j < G; ++j) nz += (static_cast<uint32_t>(w[j * R]) & kMag) != 0;
+#pragma unroll
+        for (int j = 0; j < G; ++j) nz += (static_cast<uint32_t>(__ldg(w + j * R)) & kMag) != 0;
         nz_sum += static_cast<uint32_t>(nz);
         drop_sum += static_cast<uint32_t>(nz > K ? nz - K : 0);
     }
@@ -166,8 +282,9 @@ __global__ void pack_stats_kernel(const TB *__restrict__ W, int64_t Cout, int64_
     }
 }
 
-cudaError_t launch_pack_stats(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K,
-                              unsigned long long *counts, cudaStream_t stream)
+template <typename TB>
+void launch_pack_stats_t(const TB *W, int64_t Cout, int64_t R, int G, int K, unsigned long long *counts,
+                         cudaStream_t stream)
 {
     const int64_t total = (Cout / G) * R;
     const int threads = 256;
@@ -175,12 +292,22 @@ cudaError_t launch_pack_stats(const void *W, int dtype, int64_t Cout, int64_t R,
     // at most 8 blocks per SM with grid-stride loops: few atomics; a thread's
     // sums stay far below 2^32 for any matrix that fits in memory
     const int grid = static_cast<int>(blocks < 152 * 8 ? blocks : 152 * 8);
+    switch (G) {
+        case 4: pack_stats_kernel<TB, 4><<<grid, threads, 0, stream>>>(W, Cout, R, G, K, counts); break;
+        case 8: pack_stats_kernel<TB, 8><<<grid, threads, 0, stream>>>(W, Cout, R, G, K, counts); break;
+        case 16: pack_stats_kernel<TB, 16><<<grid, threads, 0, stream>>>(W, Cout, R, G, K, counts); break;
+        case 32: pack_stats_kernel<TB, 32><<<grid, threads, 0, stream>>>(W, Cout, R, G, K, counts); break;
+        default: pack_stats_kernel<TB, 0><<<grid, threads, 0, stream>>>(W, Cout, R, G, K, counts);
+    }
+}
+
+cudaError_t launch_pack_stats(const void *W, int dtype, int64_t Cout, int64_t R, int G, int K,
+                              unsigned long long *counts, cudaStream_t stream)
+{
     if (dtype == CCI_F32)
-        pack_stats_kernel<uint32_t><<<grid, threads, 0, stream>>>(static_cast<const uint32_t *>(W), Cout, R, G, K,
-                                                                  counts);
+        launch_pack_stats_t(static_cast<const uint32_t *>(W), Cout, R, G, K, counts, stream);
     else
-        pack_stats_kernel<uint16_t><<<grid, threads, 0, stream>>>(static_cast<const uint16_t *>(W), Cout, R, G, K,
-                                                                  counts);
+        launch_pack_stats_t(static_cast<const uint16_t *>(W), Cout, R, G, K, counts, stream);
     return cudaGetLastError();
 }
 

@@ -681,7 +681,8 @@ def test_fused_identity_equals_plain_product(dev):
 # ---------------------------------------------------------------------------
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("Cout,R,G,K,Ps", [(64, 33, 8, 2, 0.75), (48, 1000, 16, 4, 0.5), (1024, 4096, 8, 2, 0.75),
-                                           (4, 7, 4, 1, 0.3), (512, 96, 32, 8, 0.9)])
+                                           (4, 7, 4, 1, 0.3), (512, 96, 32, 8, 0.9),
+                                           (90, 21, 3, 1, 0.4), (128, 40, 64, 16, 0.5)])
 def test_pack_stats_exact(dev, dtype, Cout, R, G, K, Ps):
     rng = np.random.default_rng(Cout + R + G)
     W = rng.standard_normal((Cout, R)).astype(np.float32)

@@ -69,7 +69,8 @@ def test_drop_rate_schedule():
 @pytest.mark.gpu
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16])
 @pytest.mark.parametrize("Cout,R,G,K,rate", [(64, 37, 8, 2, 0.5), (96, 1000, 16, 4, 0.9), (4096, 1024, 8, 2, 0.75),
-                                             (32, 9, 32, 8, 1.0), (12, 5, 4, 3, 0.0)])
+                                             (32, 9, 32, 8, 1.0), (12, 5, 4, 3, 0.0),
+                                             (30, 41, 3, 1, 0.6), (128, 19, 64, 9, 0.8)])
 def test_td_mask_matches_oracle(dtype, Cout, R, G, K, rate):
     from paper_1910_11971_gb300 import build as cci_build
     cci_build.build()
