@@ -489,7 +489,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
             advance(t2, k2);
         }
         if constexpr (!C::kATma) {
-            for (int64_t tile = blockIdx.x; tile < n_tiles && ok; tile += gridDim.x) {
+            // the same work units, in the same order, as the TMA issuers and the MMAs
+            for (int64_t tile = u0; tile < n_tiles && ok; tile += ustep) {
                 const int64_t n0 = (tile / n_ct) * kM;
                 ColumnSite site[8];
                 bool colok[8];
@@ -616,7 +617,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
         };
         for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
             const int acc = t & 1;
-            if (t >= 2) ok = tc::mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
+            // CG = 2: the phase includes arrivals of the odd CTA's epilogue
+            if (t >= 2) ok = tc::mbar_wait<CG == 2>(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);

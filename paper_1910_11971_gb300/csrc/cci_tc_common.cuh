@@ -40,21 +40,46 @@ __device__ __forceinline__ void mbar_arrive(uint64_t *bar)
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
-// bounded wait for the phase with the given parity; false on timeout or abort
+// one test of the phase with the given parity (kCluster: acquire at cluster
+// scope, for phases that include arrivals released by the other CTA of a pair).
+// A waiting thread is suspended in hardware until the phase completes (or the
+// hint elapses) instead of spinning: the kernels hold a dozen warps that spend
+// most of their time waiting, and spinning ones take issue slots from the warps
+// issuing MMAs and copies on the same scheduler.
+constexpr uint32_t kSuspendNs = 1000000;
+template <bool kCluster>
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity)
+{
+    uint32_t done;
+    if constexpr (kCluster)
+        asm volatile(
+            "{\n.reg .pred p;\n"
+            "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2, %3;\n"
+            "selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(a), "r"(parity), "n"(kSuspendNs)
+            : "memory");
+    else
+        asm volatile(
+            "{\n.reg .pred p;\n"
+            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+            "selp.u32 %0, 1, 0, p;\n}\n"
+            : "=r"(done)
+            : "r"(a), "r"(parity), "n"(kSuspendNs)
+            : "memory");
+    return done != 0;
+}
+
+// bounded wait for the phase with the given parity; false on timeout or abort.
+// A phase already complete costs one test (no clock read).
+template <bool kCluster = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, volatile int *abort, uint32_t *status)
 {
     const uint32_t a = smem_u32(bar);
+    if (mbar_try<kCluster>(a, parity)) return true;
     const long long t0 = clock64();
     while (true) {
-        uint32_t done;
-        asm volatile(
-            "{\n.reg .pred p;\n"
-            "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-            "selp.u32 %0, 1, 0, p;\n}\n"
-            : "=r"(done)
-            : "r"(a), "r"(parity)
-            : "memory");
-        if (done) return true;
+        if (mbar_try<kCluster>(a, parity)) return true;
         if (*abort) return false;
         if (clock64() - t0 > kWaitLimit) {
             *abort = 1;

@@ -585,6 +585,33 @@ def test_pair_tiles_conv(dev, B, H, Cin, Cout, stride):
         assert_within_tol(Yg, Yo, S, f"pair conv B={B} H={H} s={stride} image {b}")
 
 
+# fp32 layers (three tf32 passes) with long reductions: odd M tile counts,
+# ragged reductions and N tails, both N tiles, 2-D and 4-D copies, checked on
+# sampled outputs (products) or every output (convolutions).
+@pytest.mark.parametrize("N,Cin,Cout,G,K", [(16429, 256, 1024, 8, 2), (5000, 300, 192, 16, 4), (300, 512, 64, 4, 1)])
+def test_tf32x3_long_reduction_product(dev, N, Cin, Cout, G, K):
+    X, W = wl.random_small(N + Cin + 1, "f32", N, Cin, Cout)
+    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    rows = np.unique(np.concatenate([sample_rows(N, 768, seed=N), np.arange(N - 200, N)]))
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, f"tf32x3 product {N}x{Cin}->{Cout}")
+
+
+@pytest.mark.parametrize("B,H,Cin,Cout,stride", [(9, 14, 64, 128, 1), (8, 28, 32, 64, 2), (3, 7, 256, 256, 1)])
+def test_tf32x3_long_reduction_conv(dev, B, H, Cin, Cout, stride):
+    G, K = 8, 2
+    g = torch.Generator().manual_seed(B * 37 + H + Cin)
+    X = torch.randn((B, H, H, Cin), generator=g).clamp_min(0)
+    W = torch.randn((Cout, 9 * Cin), generator=g)
+    Y = run_conv(dev, X, W, (3, 3, (stride, stride), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, 3, 3, (stride, stride), (1, 1))
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, f"tf32x3 conv B={B} H={H} s={stride}")
+
+
 # ---------------------------------------------------------------------------
 # fused output epilogue: + bias, ReLU, fp32 or bf16 (round to nearest even)
 # output, on every activation source and tile form of the workspace family
