@@ -17,6 +17,15 @@
 //               TMA over X[B][H][W][Cin] with a box of QB x PB x BB output
 //               pixels (QB*PB*BB <= 128 rows), shifted by the tap (kh, kw); the
 //               zero padding is the copy's out-of-range fill;
+//     kAHalo    bf16 3x3 convolutions with unit stride and padding 1: per tile
+//               and 64-channel chunk one TMA copy of the input halo, rows
+//               (p, q) of PB input rows + 2 by Q + 2 columns (the padding is the
+//               copy's out-of-range fill); the tile's output rows are laid out on
+//               the same Q + 2 wide grid (two unused columns per row), so tap
+//               (kh, kw) reads the halo from row kh * (Q + 2) + kw on: the A
+//               operand of every tap is the same buffer at a row offset (the
+//               128-byte swizzle follows the address, so any row offset works);
+//               per stage only the tap's weight tile is copied;
 //     kAGather  other convolutions: the producer warps gather rows (cp.async for
 //               bf16; registers, two stages ahead, then the hi/lo split, for fp32).
 //   fp32 activations copied by TMA land raw in shared memory; the producer warps
@@ -44,16 +53,19 @@
 namespace cci {
 namespace ws {
 
-enum ASrc { kA2d = 0, kA4d = 1, kAGather = 2 };
+enum ASrc { kA2d = 0, kA4d = 1, kAGather = 2, kAHalo = 3 };
 
 // output-pixel box of one M tile of a convolution whose activations are copied
 // by 4-D TMA: rows m = (bi*PB + pi)*QB + qi of the tile are the pixels
-// (b0 + bi, p0 + pi, q0 + qi); rows >= QB*PB*BB are unused
+// (b0 + bi, p0 + pi, q0 + qi); rows >= QB*PB*BB are unused.  Halo copies: QB = Q,
+// BB = 1, rows m = pi*(Q + 2) + qi (qi >= Q unused), rows = PB*(Q + 2)
 struct ConvBox {
     int QB, PB, BB;  // box extent along q, p and the batch
     int nQ, nP;      // boxes along q and p (the batch index is the rest)
     int rows;        // QB * PB * BB
     int64_t B;       // batch size
+    int hrows;       // halo copies: rows of one halo buffer (a multiple of 8)
+    int nh;          // halo copies: buffers in the ring (0 otherwise)
 };
 
 // activation tensor maps: [0] for products (2-D over X[N][Cin]); for a
@@ -76,13 +88,19 @@ struct Cfg {
     static constexpr int kBRows = kN / CG;  // B rows held by one CTA
     static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
+    static constexpr bool kHalo = ASRC == kAHalo;  // A: per-chunk halo buffers, stages hold B only
+    static_assert(!kHalo || (!TF32 && CG == 1), "halo copies: bf16 single-CTA tiles");
     // raw fp32 A by TMA; the producers split it into hi / lo and write both to
     // tensor memory, where the MMAs read A (no A planes in shared memory)
     static constexpr bool kARaw = TF32 && ASRC != kAGather;
     static constexpr int kAPlanes = (TF32 && !kARaw) ? 2 : 1, kBPlanes = TF32 ? 2 : 1;
     static constexpr int kAPlane = kM * 128;                    // bytes: 128-byte rows
     static constexpr int kBPlane = kBRows * 128;
-    static constexpr int kStage = kAPlanes * kAPlane + kBPlanes * kBPlane;
+    static constexpr int kBOff = kHalo ? 0 : kAPlanes * kAPlane;  // B planes within a stage
+    static constexpr int kStage = kBOff + kBPlanes * kBPlane;
+    // halo copies: fewer weight stages, the rest of shared memory for a ring of
+    // halo buffers whose size and count the host sets per layer (ConvBox)
+    static constexpr int kHaloStages = kBPlane <= 8192 ? 6 : (kBPlane <= 16384 ? 4 : 3);
     static constexpr int kYBuf = kM * 128;  // one output staging buffer: [128 rows][32 fp32]
     // epilogue groups: warps 0-3, and warps 4-7 too when they have no producer work
     // (TMA-copied bf16 activations); two staging buffers per group
@@ -90,12 +108,13 @@ struct Cfg {
     static constexpr int kYBufs = 2 * kEG;
     static_assert(EPI == 1 || EPI == 2, "epilogue groups");
     static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - kYBufs * kYBuf - 1024;
-    static constexpr int kStages = (kBudget / kStage) < tc::kMaxStages ? (kBudget / kStage) : tc::kMaxStages;
+    static constexpr int kStagesFit = (kBudget / kStage) < tc::kMaxStages ? (kBudget / kStage) : tc::kMaxStages;
+    static constexpr int kStages = kHalo ? kHaloStages : kStagesFit;
     // accumulators: 2 x kN columns; kARaw adds per stage A hi and A lo (32 columns each)
     static constexpr int kAColBase = 2 * kN;
     static constexpr int kTmemCols = kARaw ? 512 : 2 * kN;
     static constexpr size_t kSmem =
-        1024 + static_cast<size_t>(kStages) * kStage + kYBufs * kYBuf + sizeof(tc::Smem) + 64;
+        1024 + static_cast<size_t>(kStages) * kStage + kYBufs * kYBuf + sizeof(tc::Smem) + 64;  // + halo ring
     static constexpr uint32_t kBBytes = kBPlanes * kBPlane;
     static constexpr uint32_t kIdesc = (1u << 4)                                           // D f32
                                        | (TF32 ? (2u << 7) | (2u << 10) : (1u << 7) | (1u << 10))  // tf32 / bf16
@@ -109,9 +128,11 @@ struct Cfg {
     // thread's copies are processed one box at a time, so several issuers keep
     // more boxes moving.  kIssuers <= kStages keeps every empty-barrier wait
     // within one phase of the barrier (no parity aliasing).
-    static constexpr int kIssuers = ASRC == kAGather ? 1 : (kStages < 4 ? kStages : 4);
+    // (kAHalo: one more warp, which copies the halos)
+    static constexpr int kIssuers = ASRC == kAGather ? 1 : (kStages < 4 ? kStages : 4) + (kHalo ? 1 : 0);
     static constexpr int kThreads = 32 * (9 + kIssuers);
-    static_assert(kIssuers >= 1 && kIssuers <= kStages, "issuers must not outnumber the stages");
+    static_assert(kIssuers - (kHalo ? 1 : 0) >= 1 && kIssuers - (kHalo ? 1 : 0) <= kStages,
+                  "stage issuers must not outnumber the stages");
 };
 
 template <bool TF32, int CG>
@@ -145,6 +166,32 @@ __device__ __forceinline__ void mma_tf32_ta(uint32_t d, uint32_t a_tmem, uint64_
         "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
         "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
         "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        : "memory");
+}
+
+// ---- one pipeline stage of bf16 MMAs ----
+// Every lane of the MMA warp executes the block; the lane with `issue` set
+// issues the four 16-deep MMAs of a 64-wide stage (descriptors advance by 32
+// bytes, 2 units of 16 bytes, per MMA) and commits the stage to `bar`.  Kept in
+// one block with the descriptors precomputed: the MMA warp's own instruction
+// latency per stage bounds layers whose MMAs are short (measured on GB300: a
+// 64-wide N tile stage is 192 tensor cycles, and the issue path was 400-700).
+template <uint32_t kIdesc>
+__device__ __forceinline__ void stage_f16(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t acc0, uint32_t issue,
+                                          uint32_t bar)
+{
+    asm volatile(
+        "{\n.reg .pred pe, pa, pt;\n.reg .b64 ad, bd;\n"
+        "setp.ne.b32 pe, %4, 0;\nsetp.ne.b32 pa, %3, 0;\nsetp.eq.b32 pt, 0, 0;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %5, pa;\n"
+        "add.s64 ad, %1, 2;\nadd.s64 bd, %2, 2;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %5, pt;\n"
+        "add.s64 ad, %1, 4;\nadd.s64 bd, %2, 4;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %5, pt;\n"
+        "add.s64 ad, %1, 6;\nadd.s64 bd, %2, 6;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %5, pt;\n"
+        "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%6];\n}\n" ::"r"(d),
+        "l"(adesc), "l"(bdesc), "r"(acc0), "r"(issue), "n"(kIdesc), "r"(bar)
         : "memory");
 }
 
@@ -286,8 +333,13 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
     extern __shared__ __align__(16) unsigned char smem_raw[];
     const uint32_t raw = tc::smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
-    const uint32_t ybuf = base + kStages * C::kStage;  // output staging buffers, two per epilogue group
-    tc::Smem *S = reinterpret_cast<tc::Smem *>(smem_raw + (base - raw) + kStages * C::kStage + C::kYBufs * C::kYBuf);
+    const uint32_t hbuf = base + kStages * C::kStage;  // halo ring (kAHalo: box.nh buffers)
+    const uint32_t hbytes = static_cast<uint32_t>(box.hrows) * 128u;
+    const uint32_t hring = C::kHalo ? static_cast<uint32_t>(box.nh) * hbytes : 0u;
+    const uint32_t ybuf = hbuf + hring;  // output staging buffers, two per epilogue group
+    tc::Smem *S = reinterpret_cast<tc::Smem *>(smem_raw + (base - raw) + kStages * C::kStage + hring +
+                                               C::kYBufs * C::kYBuf);
+    const int taps = p.KH * p.KW;  // kAHalo: stages run chunk by chunk, the taps of a chunk in turn
     volatile int *abort = &S->abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nks = static_cast<int>((p.R + kKS - 1) / kKS);
@@ -314,6 +366,10 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
             tc::mbar_init(&S->tmem_empty[a], 128 * CG);
         }
         tc::mbar_init(&S->drain, 1);
+        for (int h = 0; h < tc::kMaxHalo; ++h) {
+            tc::mbar_init(&S->hfull[h], 1);
+            tc::mbar_init(&S->hempty[h], 1);
+        }
         S->abort = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -343,6 +399,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
         if constexpr (ASRC == kA2d) tc::tma_prefetch_desc(&tmA.m[0]);
         if constexpr (ASRC == kA4d)
             for (int i = 0; i < p.sh * p.sw; ++i) tc::tma_prefetch_desc(&tmA.m[i]);
+        if constexpr (ASRC == kAHalo) tc::tma_prefetch_desc(&tmA.m[0]);
         tc::tma_prefetch_desc(&tmB0);
         if constexpr (C::kBPlanes > 1) tc::tma_prefetch_desc(&tmB1);
         tc::tma_prefetch_desc(&tmY);
@@ -362,20 +419,57 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
         // ------------------------------------------------------------ TMA issuers
         const uint32_t a_bytes = ASRC == kA4d ? static_cast<uint32_t>(box.rows) * 128u : C::kAPlane;
         const int cpt = static_cast<int>(p.Cin / kKS);  // stages per tap (kA4d)
-        const int issuer = warp - 9;
+        const uint32_t halo_bytes =
+            static_cast<uint32_t>((box.QB + p.KW - 1) * (box.PB + p.KH - 1)) * 128u;  // kAHalo
+        // kAHalo: warp 9 copies the halos, as far ahead as the halo ring allows;
+        // the other issuer warps copy the weight stages in turn
+        const int issuer = warp - (C::kHalo ? 10 : 9);
+        constexpr int kBIssuers = C::kHalo ? C::kIssuers - 1 : C::kIssuers;
         int it = 0;
         bool ok = true;
+        if (C::kHalo && warp == 9) {
+            int hc = 0;
+            const int chunks = nks / taps;
+            for (int64_t u = u0; u < n_tiles && ok; u += ustep) {
+                int64_t mt, ct;
+                split_unit(u, mt, ct);
+                const BoxIdx bi = box_of(mt, box);
+                for (int c = 0; c < chunks && ok; ++c, ++hc) {
+                    // buffer hb is free once the MMAs of chunk hc - nh completed; this
+                    // warp waited for chunk hc - 1 - nh before, so the phase cannot alias
+                    const int hb = hc % box.nh;
+                    if (hc >= box.nh) ok = tc::mbar_wait(&S->hempty[hb], ((hc / box.nh) - 1) & 1, abort, p.status);
+                    if (!ok) break;
+                    if (lane == 0) {
+                        tc::mbar_arrive_expect_tx(&S->hfull[hb], halo_bytes);
+                        tc::tma_load_4d(hbuf + hb * hbytes, &tmA.m[0], c * 64, -p.pw, bi.pb * box.PB - p.ph,
+                                        static_cast<int>(bi.bb), &S->hfull[hb]);
+                    }
+                    __syncwarp();
+                }
+            }
+        } else
         for (int64_t u = u0; u < n_tiles && ok; u += ustep) {
             int64_t mt, ct;
             split_unit(u, mt, ct);
             const int64_t co0 = ct * kN + crank * C::kBRows;  // this CTA's B rows
             BoxIdx bi{0, 0, 0};
-            if constexpr (ASRC == kA4d) bi = box_of(mt, box);
+            if constexpr (ASRC == kA4d || ASRC == kAHalo) bi = box_of(mt, box);
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
-                if (it % C::kIssuers != issuer) continue;
+                if (it % kBIssuers != issuer) continue;
                 const int s = it % kStages;
                 if (it >= kStages) ok = tc::mbar_wait(&S->empty[s], ((it / kStages) - 1) & 1, abort, p.status);
                 if (!ok) break;
+                if constexpr (ASRC == kAHalo) {
+                    const int c = ks / taps, t = ks - c * taps;  // stages: chunk by chunk, taps in turn
+                    if (lane == 0) {
+                        tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes);
+                        tc::tma_load_2d(base + s * C::kStage, &tmB0, static_cast<int>(t * p.Cin) + c * 64,
+                                        static_cast<int>(ct * kN), &S->full[s]);
+                    }
+                    __syncwarp();
+                    continue;
+                }
                 if (lane == 0 && CG == 2) {
                     // both CTAs' copies complete on the even CTA's full barrier, which
                     // expects the bytes of the pair
@@ -398,7 +492,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                     }
                 } else if (lane == 0) {
                     const uint32_t st = base + s * C::kStage;
-                    const uint32_t bst = st + C::kAPlanes * C::kAPlane;
+                    const uint32_t bst = st + C::kBOff;
                     // the activation copy completes on aux (raw fp32, split afterwards) or full
                     uint64_t *abar = C::kARaw ? &S->aux[s] : &S->full[s];
                     if constexpr (C::kARaw) tc::mbar_arrive_expect_tx(abar, a_bytes);
@@ -609,6 +703,13 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
         // the drain)
         int it = 0, t = 0;
         bool ok = CG == 1 || crank == 0;
+        // kAHalo: stage and halo-ring positions with their phase parities
+        int hs = 0, hb = 0;
+        uint32_t hsph = 0u, hph = 0u;
+        const int hchunks = ASRC == kAHalo ? nks / taps : 0;
+        const uint64_t hdesc0 = tc::sw128_desc(hbuf), bdesc0 = tc::sw128_desc(base);
+        const uint32_t empty0 = tc::smem_u32(&S->empty[0]);
+        const uint32_t issue = lane == 0 ? 1u : 0u;  // the lane that issues (a predicate in the stage block)
         auto commit = [&](uint64_t *bar) {
             if constexpr (CG == 2)
                 mma_commit_pair(bar);
@@ -622,6 +723,39 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
+            if constexpr (ASRC == kAHalo) {
+                // chunk by chunk (halo buffer hb of the ring), the taps in turn: tap
+                // (kh, kw) reads the halo from row kh * (Q + 2) + kw on.  Counters
+                // advance by increments (no division in the issue loop).
+                // descriptors in 16-byte units: + wq_units per halo row of taps,
+                // + 8 per column, + hunits per halo buffer, + sunits per stage
+                const uint64_t wq_units = static_cast<uint64_t>(box.QB + p.KW - 1) * 8u;
+                const uint64_t hunits = hbytes >> 4, sunits = C::kStage >> 4;
+                for (int c = 0; c < hchunks && ok; ++c) {
+                    ok = tc::mbar_wait(&S->hfull[hb], hph, abort, p.status);
+                    const uint64_t hdesc = hdesc0 + static_cast<uint64_t>(hb) * hunits;
+                    for (int kh = 0; kh < p.KH && ok; ++kh) {
+                        for (int kw = 0; kw < p.KW && ok; ++kw, ++it) {
+                            ok = tc::mbar_wait(&S->full[hs], hsph, abort, p.status);
+                            if (!ok) break;
+                            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                            stage_f16<C::kIdesc>(d, hdesc + static_cast<uint64_t>(kh) * wq_units + kw * 8u,
+                                                 bdesc0 + static_cast<uint64_t>(hs) * sunits,
+                                                 (c | kh | kw) != 0 ? 1u : 0u, issue, empty0 + 8u * hs);
+                            if (kh == p.KH - 1 && kw == p.KW - 1 && lane == 0) commit(&S->hempty[hb]);
+                            __syncwarp();
+                            if (++hs == kStages) {
+                                hs = 0;
+                                hsph ^= 1u;
+                            }
+                        }
+                    }
+                    if (++hb == box.nh) {
+                        hb = 0;
+                        hph ^= 1u;
+                    }
+                }
+            } else
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
                 const int s = it % kStages;
                 ok = tc::mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
@@ -629,7 +763,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 if (lane == 0) {
                     const uint32_t st = base + s * C::kStage;
-                    const uint32_t bst = st + C::kAPlanes * C::kAPlane;
+                    const uint32_t bst = st + C::kBOff;
                     if constexpr (C::kARaw) {
 #pragma unroll
                         for (int k = 0; k < kKS / 8; ++k) {
@@ -652,14 +786,18 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                             mma<TF32, CG>(d, ah, bl, C::kIdesc, 1u);
                             mma<TF32, CG>(d, ah, bh, C::kIdesc, 1u);
                         }
-                    } else {
+                    } else if constexpr (CG == 2) {
 #pragma unroll
                         for (int k = 0; k < kKS / 16; ++k)
                             mma<TF32, CG>(d, tc::sw128_desc(st + k * 32), tc::sw128_desc(bst + k * 32), C::kIdesc,
                                           (ks > 0 || k > 0) ? 1u : 0u);
                     }
-                    commit(&S->empty[s]);
+                    if constexpr (TF32 || CG == 2) commit(&S->empty[s]);
                 }
+                if constexpr (!TF32 && CG == 1)
+                    stage_f16<C::kIdesc>(d, bdesc0 + static_cast<uint64_t>(s) * (C::kStage >> 4),
+                                         bdesc0 + static_cast<uint64_t>(s) * (C::kStage >> 4) + (C::kBOff >> 4),
+                                         ks > 0 ? 1u : 0u, issue, empty0 + 8u * s);
                 __syncwarp();
             }
             if (ok && lane == 0) commit(&S->tmem_full[acc]);
@@ -690,7 +828,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
             split_unit(u, mt, ct);
             const int co0 = static_cast<int>(ct * kN);
             BoxIdx bi{0, 0, 0};
-            if constexpr (ASRC == kA4d) bi = box_of(mt, box);
+            if constexpr (ASRC == kA4d || ASRC == kAHalo) bi = box_of(mt, box);
             ok = tc::mbar_wait(&S->tmem_full[acc], (t / 2) & 1, abort, p.status);
             ok = tc::named_and(ebar, 128, ok);
             if (!ok) break;
@@ -729,13 +867,25 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                 const uint32_t buf = ybuf + static_cast<uint32_t>(2 * eg + (chunk_no & 1)) * C::kYBuf;
                 if (etid == 0) tc::bulk_wait_read<1>();
                 tc::named_sync(ebar, 128);
+                // halo tiles: row m = pi * (Q + 2) + qi goes to staged row pi * Q + qi
+                // (the box of the store), the two unused columns of each row nowhere
+                int srow = m;
+                bool stage_row = true;
+                if constexpr (ASRC == kAHalo) {
+                    const int wq = box.QB + p.KW - 1;
+                    const int pi = m / wq, qi = m - (m / wq) * wq;
+                    srow = pi * box.QB + qi;
+                    stage_row = pi < box.PB && qi < box.QB;
+                }
+                if (stage_row) {
 #pragma unroll
-                for (int q = 0; q < 8; ++q)
-                    st_shared_v4(buf + sw_chunk(m, q), v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                    for (int q = 0; q < 8; ++q)
+                        st_shared_v4(buf + sw_chunk(srow, q), v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 tc::named_sync(ebar, 128);
                 if (etid == 0) {
-                    if constexpr (ASRC == kA4d)
+                    if constexpr (ASRC == kA4d || ASRC == kAHalo)
                         tc::tma_store_4d(&tmY, buf, co0 + c0, bi.qb * box.QB, bi.pb * box.PB,
                                          static_cast<int>(bi.bb * box.BB));
                     else
@@ -826,6 +976,14 @@ inline bool build_a_maps(const FwdParams &p, const ConvBox &box, int asrc, bool 
         const int bx[2] = {ks, 128};
         return make_map(&am->m[0], p.X, dt, static_cast<int>(e), 2, dims, bx);
     }
+    if (asrc == kAHalo) {
+        // the halo of PB output rows: Q + KW - 1 columns by PB + KH - 1 rows of
+        // input pixels, 64 channels, from (q, p) = (-pw, p0 - ph) on
+        const int64_t dims[4] = {p.Cin, p.W, p.H, box.B};
+        const int64_t strides[3] = {p.Cin * e, p.W * p.Cin * e, p.H * p.W * p.Cin * e};
+        const int bx[4] = {64, box.QB + p.KW - 1, box.PB + p.KH - 1, 1};
+        return make_map_strided(&am->m[0], p.X, dt, 4, dims, strides, bx);
+    }
     if (asrc != kA4d) return true;
     for (int rh = 0; rh < p.sh; ++rh)
         for (int rw = 0; rw < p.sw; ++rw) {
@@ -905,12 +1063,23 @@ inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn, int cg = 1)
 }
 
 template <bool TF32, int ASRC, int BN, int CG, int EPI = 1>
-cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA, cudaStream_t stream)
+cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &tmA, cudaStream_t stream)
 {
     using C = Cfg<TF32, ASRC, BN, CG, EPI>;
     auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG, EPI>;
-    static const cudaError_t attr =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(C::kSmem));
+    ConvBox box = box_in;
+    size_t smem = C::kSmem;
+    if constexpr (C::kHalo) {
+        // the halo ring takes the shared memory left: up to kMaxHalo buffers, two at least
+        const size_t hb = static_cast<size_t>(box.hrows) * 128;
+        const size_t left = kMaxSmemPerBlock - C::kSmem;
+        box.nh = static_cast<int>(left / hb < static_cast<size_t>(tc::kMaxHalo) ? left / hb : tc::kMaxHalo);
+        if (box.nh < 2) return cudaErrorInvalidValue;
+        smem += static_cast<size_t>(box.nh) * hb;
+    }
+    static const cudaError_t attr = cudaFuncSetAttribute(
+        kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        static_cast<int>(C::kHalo ? static_cast<size_t>(kMaxSmemPerBlock) : C::kSmem));
     if (attr != cudaSuccess) return attr;
     CUtensorMap tmB0{}, tmB1{}, tmY{};
     const CUtensorMapDataType dt = TF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
@@ -925,7 +1094,7 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
     // output rows of 128 bytes: 32 fp32 or 64 bf16 channels
     const CUtensorMapDataType ydt = p.out_bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
     const int yel = p.out_bf16 ? 2 : 4, ysc = p.out_bf16 ? 64 : 32;
-    if constexpr (ASRC == kA4d) {
+    if constexpr (ASRC == kA4d || ASRC == kAHalo) {
         const int64_t dims[4] = {p.Cout, p.Q, p.P, box.B};
         const int bx[4] = {ysc, box.QB, box.PB, box.BB};
         if (!make_map(&tmY, p.Y, ydt, yel, 4, dims, bx)) return cudaErrorInvalidValue;
@@ -935,7 +1104,8 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
         if (!make_map(&tmY, p.Y, ydt, yel, 2, dims, bx)) return cudaErrorInvalidValue;
     }
     const int64_t n_ct = (p.Cout + C::kN - 1) / C::kN;
-    const int64_t m_tiles = ASRC == kA4d ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)
+    const int64_t m_tiles = (ASRC == kA4d || ASRC == kAHalo)
+                                ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)
                                          : (p.N + C::kM - 1) / C::kM;
     // CG = 2: units are pair tiles (two M tiles), one per CTA pair
     const int64_t n_tiles = n_ct * (CG == 2 ? (m_tiles + 1) / 2 : m_tiles);
@@ -947,7 +1117,7 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box, const AMaps &tmA,
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(static_cast<unsigned>(grid));
     cfg.blockDim = dim3(C::kThreads);
-    cfg.dynamicSmemBytes = C::kSmem;
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute la[2];
     la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -969,11 +1139,40 @@ struct Plan {
     ConvBox box;
     AMaps am;
 };
+// halo box of a bf16 3x3, stride-1, padding-1 convolution: PB output rows of
+// the full width per tile.  Used for layers of 256 input channels or more (four
+// chunks or more per tile: the per-tap copies there move 9 x the halo's bytes,
+// and the halo copies measured 7-11 % faster on the 14 x 14 ResNet-50 layers;
+// with 64 or 128 channels the tile is bound by the MMAs' shared-memory reads
+// and the per-tap form measured faster) whose output rows per tile are at
+// least three quarters of the 4-D box's (images narrower than the tile fit
+// several per 4-D box, not per halo)
+inline bool halo_box(const FwdParams &p, const ConvBox &a4d, ConvBox *hb)
+{
+    if (!(p.is_conv && p.KH == 3 && p.KW == 3 && p.sh == 1 && p.sw == 1 && p.ph == 1 && p.pw == 1 &&
+          p.Cin % 64 == 0 && p.Cin >= 256 && p.P == p.H && p.Q == p.W && p.Q + 2 <= 66))
+        return false;
+    const int wq = static_cast<int>(p.Q) + 2;
+    const int pb = static_cast<int>(p.P < 128 / wq ? p.P : 128 / wq);
+    if (pb < 1 || 4 * pb * p.Q < 3 * a4d.rows) return false;
+    const int64_t B = p.N / (p.P * p.Q);
+    // rows an MMA can read: 128 from the largest tap offset 2 * wq + 2 on, in
+    // whole 1024-byte swizzle patterns
+    const int hrows = (128 + 2 * wq + 2 + 7) / 8 * 8;
+    *hb = ConvBox{static_cast<int>(p.Q), pb, 1, 1, static_cast<int>((p.P + pb - 1) / pb), pb * wq, B, hrows, 0};
+    return true;
+}
+
 inline void plan_layer(const FwdParams &p, bool tf32, int ks, Plan *pl)
 {
     pl->asrc = a_source(p, ks);
     pl->box = ConvBox{1, 1, 1, 1, 1, 1, 1};
     if (pl->asrc == kA4d) pl->box = choose_box(p.N / (p.P * p.Q), p.P, p.Q);
+    ConvBox hb;
+    if (pl->asrc == kA4d && !tf32 && halo_box(p, pl->box, &hb)) {
+        pl->asrc = kAHalo;
+        pl->box = hb;
+    }
     if (!build_a_maps(p, pl->box, pl->asrc, tf32, ks, &pl->am)) {
         pl->asrc = kAGather;
         pl->box = ConvBox{1, 1, 1, 1, 1, 1, 1};
@@ -983,7 +1182,8 @@ inline void plan_layer(const FwdParams &p, bool tf32, int ks, Plan *pl)
 // m tiles of the layer for the chosen activation source
 inline int64_t m_tiles_of(const FwdParams &p, int asrc, const ConvBox &box)
 {
-    if (asrc == kA4d) return static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB);
+    if (asrc == kA4d || asrc == kAHalo)
+        return static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB);
     return (p.N + 127) / 128;
 }
 

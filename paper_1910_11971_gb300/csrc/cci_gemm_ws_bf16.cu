@@ -16,12 +16,18 @@ cudaError_t launch_gemm_ws_bf16(const FwdParams &p, cudaStream_t stream)
     // CTA pairs (256-row tiles, B split over the pair) halve each SM's B traffic,
     // which pays on long reductions with 256-wide N tiles; shorter or narrower
     // layers run faster on single CTAs (measured on the ResNet-50 stack)
-    const bool pair = asrc != kAGather && nks >= 16 && choose_bn(m_tiles, p.Cout, 256, 2) == 256;
+    const bool pair = (asrc == kA2d || asrc == kA4d) && nks >= 16 && choose_bn(m_tiles, p.Cout, 256, 2) == 256;
     if (pair) {
         if (asrc == kA2d) return launch_cfg<false, kA2d, 256, 2>(p, pl.box, pl.am, stream);
         return launch_cfg<false, kA4d, 256, 2>(p, pl.box, pl.am, stream);
     }
     const int bn = choose_bn(m_tiles, p.Cout, 256, 1);
+    if (asrc == kAHalo) {
+        // 3x3 convolutions from halo copies (tiles of nine stages per chunk at least)
+        if (bn == 64) return launch_cfg<false, kAHalo, 64, 1>(p, pl.box, pl.am, stream);
+        if (bn == 128) return launch_cfg<false, kAHalo, 128, 1>(p, pl.box, pl.am, stream);
+        return launch_cfg<false, kAHalo, 256, 1>(p, pl.box, pl.am, stream);
+    }
     // tiles of at most 4 stages: the output write dominates, two epilogue groups
     // with two staging buffers each; longer ones keep the shared memory for stages
     const bool short_k = nks <= 4 && asrc != kAGather;

@@ -10,6 +10,7 @@ namespace tc {
 constexpr long long kWaitLimit = 1ll << 31;  // clock cycles (about 1 s) per bounded wait
 
 constexpr int kMaxStages = 8;
+constexpr int kMaxHalo = 4;  // halo buffers of a 3x3 convolution tile ring
 
 // barriers and TMEM slot of a tensor-core kernel (after its 1024-byte aligned
 // stage buffers); up to kMaxStages pipeline stages
@@ -20,6 +21,8 @@ struct Smem {
     uint64_t tmem_full[2];
     uint64_t tmem_empty[2];
     uint64_t drain;
+    uint64_t hfull[kMaxHalo];   // halo copies (3x3 convolutions): halo buffer landed
+    uint64_t hempty[kMaxHalo];  // halo buffer free again (its chunk's MMAs completed)
     uint32_t tmem_base;
     int abort;
 };

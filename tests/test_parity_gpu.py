@@ -549,6 +549,46 @@ def test_dense_tc_ws_conv_tma_equals_gather_bitwise(dev):
 
 
 # ---------------------------------------------------------------------------
+# 3x3 convolutions (stride 1, padding 1, 256 input channels or more) from halo
+# copies: one copy of the input halo per tile and 64-channel chunk, every tap
+# reading it at a row offset; 56, 28 and 14 wide images, a ragged last row
+# block, a 62-wide image (64-row halo lines), 4-6 chunks per tile (the ring of
+# halo buffers wraps within and across tiles), N tiles of 64, 128 and 256.
+# Every output checked.
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("B,H,Wi,Cin,Cout", [(1, 56, 56, 256, 64), (2, 28, 28, 256, 128), (9, 14, 14, 256, 256),
+                                             (2, 30, 30, 320, 96), (1, 17, 62, 256, 64), (3, 20, 20, 384, 192)])
+def test_halo_conv3x3(dev, B, H, Wi, Cin, Cout):
+    G, K = 8, 2
+    g = torch.Generator().manual_seed(B * 53 + H + Cin + Cout)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (3, 3, (1, 1), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, 3, 3, (1, 1), (1, 1))
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, f"halo conv B={B} {H}x{Wi} {Cin}->{Cout}")
+
+
+def test_halo_conv3x3_wide_tiles(dev):
+    """Enough tiles that the 256-wide N tile wins (three stages of 32 KB beside
+    the two halo buffers); sampled outputs of the first and last images."""
+    B, H, Cin, Cout, G, K = 64, 14, 256, 512, 8, 2
+    g = torch.Generator().manual_seed(4242)
+    X = torch.randn((B, H, H, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (3, 3, (1, 1), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    per = H * H
+    for b in (0, B - 1):
+        pts = np.unique(np.concatenate([np.arange(40), np.arange(per - 40, per),
+                                        np.random.default_rng(b).choice(per, size=48)]))
+        Yo, S = oracle.conv2d(f64(X[b:b + 1]), Wd, mask, 3, 3, (1, 1), (1, 1), pts=pts)
+        Yg = f64(Y[b].reshape(-1, Cout)[torch.from_numpy(pts).to(dev)])
+        assert_within_tol(Yg, Yo, S, f"halo conv wide tiles image {b}")
+
+
+# ---------------------------------------------------------------------------
 # CTA-pair tiles (tcgen05 cta_group::2): bf16 layers with at least 16 stages of
 # 64 reduction indices and 256-wide N tiles run as 256-row tiles split over two
 # SMs.  Sizes below make the tile-round model pick that form; checked on sampled
@@ -653,6 +693,7 @@ def test_fused_product(dev, case):
 # lattices, row gather (stride 3), fp32 input
 FUSED_CONVS = [
     (3, 9, 7, 64, 64, 3, 3, (1, 1), (1, 1), 8, 2, "bf16"),
+    (3, 14, 14, 256, 128, 3, 3, (1, 1), (1, 1), 8, 2, "bf16"),  # halo copies
     (2, 9, 7, 64, 128, 3, 3, (2, 2), (1, 1), 8, 2, "bf16"),
     (1, 10, 10, 64, 64, 3, 3, (3, 3), (1, 1), 8, 2, "bf16"),
     (2, 9, 7, 32, 64, 3, 3, (1, 1), (1, 1), 8, 2, "f32"),
