@@ -159,13 +159,40 @@ __device__ __forceinline__ void mma(uint32_t d, uint64_t a, uint64_t b, uint32_t
     }
 }
 
-// tf32 MMA with A read from tensor memory (lane = row m, one column per k)
-__device__ __forceinline__ void mma_tf32_ta(uint32_t d, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc)
+// ---- one pipeline stage of three-pass tf32 MMAs, A in tensor memory ----
+// Per 8 r (k = 0..3 of a 32-wide stage): lo(A) * hi(B) + hi(A) * lo(B) + hi(A) * hi(B),
+// A hi at TMEM column a0 + 8k and A lo 32 columns on, B hi at descriptor bh + 2k
+// (32 bytes per step) and B lo one plane (kBLo 16-byte units) further.  Every
+// lane of the MMA warp executes the block; the lane with `issue` set issues the
+// twelve MMAs and commits the stage to `bar`.  One block with the addresses
+// formed by adds: the MMA warp's instruction stream per stage bounds this
+// product (measured on GB300 with clock stamps: the MMAs waited ~130 cycles per
+// stage for their operands while the issue of a stage took ~850).
+template <uint32_t kIdesc, uint32_t kBLo>
+__device__ __forceinline__ void stage_tf32x3(uint32_t d, uint32_t a0, uint64_t bh, uint32_t acc0, uint32_t issue,
+                                             uint32_t bar)
 {
     asm volatile(
-        "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
-        "tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d),
-        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
+        "{\n.reg .pred pe, pa, pt;\n.reg .b32 ah, al;\n.reg .b64 bh, bl;\n"
+        "setp.ne.b32 pe, %4, 0;\nsetp.ne.b32 pa, %3, 0;\nsetp.eq.b32 pt, 0, 0;\n"
+        "add.u32 al, %1, 32;\nadd.s64 bl, %2, %6;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], %2, %5, pa;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], bl, %5, pt;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %5, pt;\n"
+        "add.u32 ah, %1, 8;\nadd.u32 al, %1, 40;\nadd.s64 bh, %2, 2;\nadd.s64 bl, bl, 2;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], bh, %5, pt;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bl, %5, pt;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bh, %5, pt;\n"
+        "add.u32 ah, %1, 16;\nadd.u32 al, %1, 48;\nadd.s64 bh, %2, 4;\nadd.s64 bl, bl, 2;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], bh, %5, pt;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bl, %5, pt;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bh, %5, pt;\n"
+        "add.u32 ah, %1, 24;\nadd.u32 al, %1, 56;\nadd.s64 bh, %2, 6;\nadd.s64 bl, bl, 2;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], bh, %5, pt;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bl, %5, pt;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bh, %5, pt;\n"
+        "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%7];\n}\n" ::"r"(d),
+        "r"(a0), "l"(bh), "r"(acc0), "r"(issue), "n"(kIdesc), "n"(static_cast<uint64_t>(kBLo)), "r"(bar)
         : "memory");
 }
 
@@ -716,6 +743,32 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
             else
                 tc::mma_commit(bar);
         };
+        if constexpr (C::kARaw) {
+            // one thread runs the whole issue loop: no per-stage divergence or warp
+            // reconvergence between the stages' MMAs (the gaps between stages, not
+            // the MMAs, bounded this product)
+            if (lane == 0) {
+                for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
+                    const int acc = t & 1;
+                    if (t >= 2) ok = tc::mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
+                    if (!ok) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
+                    for (int ks = 0; ks < nks; ++ks, ++it) {
+                        const int s = it % kStages;
+                        ok = tc::mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
+                        if (!ok) break;
+                        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                        stage_tf32x3<C::kIdesc, (C::kBPlane >> 4)>(
+                            d, tmem + static_cast<uint32_t>(C::kAColBase + s * 64),
+                            bdesc0 + static_cast<uint64_t>(s) * (C::kStage >> 4) + (C::kBOff >> 4), ks > 0 ? 1u : 0u,
+                            1u, empty0 + 8u * s);
+                    }
+                    if (ok) commit(&S->tmem_full[acc]);
+                }
+            }
+            ok = false;  // the generic loop below is not entered
+        }
         for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
             const int acc = t & 1;
             // CG = 2: the phase includes arrivals of the odd CTA's epilogue
@@ -764,18 +817,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                 if (lane == 0) {
                     const uint32_t st = base + s * C::kStage;
                     const uint32_t bst = st + C::kBOff;
-                    if constexpr (C::kARaw) {
-#pragma unroll
-                        for (int k = 0; k < kKS / 8; ++k) {
-                            const uint32_t ah = tmem + static_cast<uint32_t>(C::kAColBase + s * 64 + k * 8);
-                            const uint32_t al = ah + 32;
-                            const uint64_t bh = tc::sw128_desc(bst + k * 32);
-                            const uint64_t bl = tc::sw128_desc(bst + C::kBPlane + k * 32);
-                            mma_tf32_ta(d, al, bh, C::kIdesc, (ks > 0 || k > 0) ? 1u : 0u);
-                            mma_tf32_ta(d, ah, bl, C::kIdesc, 1u);
-                            mma_tf32_ta(d, ah, bh, C::kIdesc, 1u);
-                        }
-                    } else if constexpr (TF32) {
+                    if constexpr (TF32) {
 #pragma unroll
                         for (int k = 0; k < kKS / 8; ++k) {
                             const uint64_t ah = tc::sw128_desc(st + k * 32);
