@@ -25,8 +25,8 @@
  *                                  P = (H + 2*pad_h - KH)/stride_h + 1, Q likewise
  *
  * Ownership and execution: the caller allocates every buffer; all data pointers
- * are DEVICE pointers; the library allocates nothing and keeps no state between
- * calls.  Every call is asynchronous on `stream` (NULL = the legacy default
+ * are DEVICE pointers (except the X_host / Y_host of cci_linear_host); the
+ * library allocates nothing and keeps no state between calls.  Every call is asynchronous on `stream` (NULL = the legacy default
  * stream) and returns once its kernels are enqueued.  Calls on different
  * streams may run concurrently when their outputs do not overlap.
  *
@@ -197,6 +197,44 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
                          int KH, int KW, int stride_h, int stride_w, int pad_h, int pad_w,
                          int G, int K, float *Y, uint32_t *dev_status, cci_algo algo,
                          void *workspace, size_t workspace_bytes, cci_stream_t stream);
+
+/*
+ * cci_linear_host -- the product H = W-hat x X of Alg. 2 (Sec. 3.2) with the
+ * activations and the output in HOST memory: Y_host[N][Cout] (fp32) =
+ * X_host[N][Cin] * Wd^T, Wd the dense matrix of the packed weights (which stay
+ * on the device).  The columns are processed in chunks of `chunk_cols`; chunk c
+ * is copied in on `copy_in_stream`, multiplied on `stream` (the dense
+ * tensor-core family, CCI_ALGO_DENSE_TC_WS; the weights are decompressed once,
+ * by the first chunk) and copied out on `copy_out_stream`, so that the copies of
+ * neighbouring chunks overlap the product.  The result equals cci_linear_ws
+ * with CCI_ALGO_DENSE_TC_WS on the same data bit for bit.
+ *
+ *   X_host, Y_host  host memory; page-locked (cudaHostAlloc / registered) for the
+ *                   copies to overlap; pageable memory is correct but serialises
+ *   values, idx     device, as cci_linear
+ *   chunk_cols      columns per chunk, >= 1 (a multiple of 128 keeps the
+ *                   product's tiles full)
+ *   device_buffer   device, 256-byte aligned, at least
+ *                   cci_linear_host_buffer_size(dtype, Cin, Cout, chunk_cols)
+ *                   bytes: the workspace and two staging slots per direction;
+ *                   overwritten
+ *   copy_in_stream, copy_out_stream  may be NULL: that copy then runs on `stream`
+ * Ordering: the copies start after the work enqueued on `stream` before the
+ * call; `stream` waits for the last copy-out, so Y_host is complete once `stream`
+ * has reached the end of the call's work (synchronise `stream` before reading
+ * it).  Calls that overlap on the GPU must use different device buffers.
+ * Errors: as cci_linear; CCI_ERR_SHAPE for chunk_cols < 1; CCI_ERR_UNSUPPORTED
+ * for layers without the dense tensor-core kernel (it needs Cin % 4 == 0 for
+ * fp32, % 8 for bf16, and G in {4, 8, 16, 32} with K <= G/2); CCI_ERR_WORKSPACE for a missing,
+ * short or misaligned device buffer; CCI_ERR_CUDA if an event, copy or launch
+ * fails (chunks already enqueued still complete on the streams).
+ */
+size_t cci_linear_host_buffer_size(cci_dtype dtype, int64_t Cin, int64_t Cout, int64_t chunk_cols);
+cci_status cci_linear_host(const void *X_host, cci_dtype dtype, int64_t N, int64_t Cin,
+                           const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
+                           float *Y_host, int64_t chunk_cols, void *device_buffer,
+                           size_t device_buffer_bytes, uint32_t *dev_status, cci_stream_t stream,
+                           cci_stream_t copy_in_stream, cci_stream_t copy_out_stream);
 
 /*
  * cci_td_mask -- one step of the improved targeted dropout used to train CCI

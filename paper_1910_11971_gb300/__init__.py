@@ -57,6 +57,9 @@ SIGNATURES = {
                               ctypes.c_size_t, _P]),
     "cci_td_mask": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, ctypes.c_float, _P, _P, _P, _U32P, _P]),
     "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
+    "cci_linear_host_buffer_size": (ctypes.c_size_t, [_I32, _I64, _I64, _I64]),
+    "cci_linear_host": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _I64, _P,
+                               ctypes.c_size_t, _U32P, _P, _P, _P]),
     "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
                                           _P]),
     "cci_kernel_name": (ctypes.c_char_p, [_I32, _I64, _I64, _I64, _I32, _I32, _I32]),
@@ -200,6 +203,53 @@ def linear(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
                                status.data_ptr() if status is not None else None, algo, wp, wb,
                                _stream(X.device))
     _check(code, "cci_linear")
+    return Y
+
+
+_copy_streams = {}
+
+
+def host_chunk(N: int) -> int:
+    """Default columns per chunk of ``linear_host``: about an eighth of N, in
+    whole 128-column tiles."""
+    return max(128, -(-(-(-N // 8)) // 128) * 128)
+
+
+def host_buffer(dtype: torch.dtype, Cin: int, Cout: int, chunk: int, device) -> torch.Tensor:
+    """A device buffer for ``linear_host`` (the library allocates nothing)."""
+    n = lib().cci_linear_host_buffer_size(F32 if dtype == torch.float32 else BF16, Cin, Cout, chunk)
+    if not n:
+        raise ValueError("cci_linear_host_buffer_size: invalid shape")
+    return torch.empty(n, dtype=torch.uint8, device=device)
+
+
+def linear_host(X_host: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, G: int, K: int, *,
+                out: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
+                chunk: Optional[int] = None, buffer: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """``linear`` with X and Y in host memory (``cci_linear_host``): column chunks
+    are copied in, multiplied and copied out on three streams, overlapping.
+    X_host should be pinned; the result ``out`` (pinned fp32 [N][Cout], allocated
+    when not given) is complete once the device's current stream has been
+    synchronised."""
+    if X_host.is_cuda or not X_host.is_contiguous():
+        raise ValueError("X_host must be a contiguous host tensor")
+    dev = values.device
+    N, Cin = X_host.shape
+    chunk = chunk or host_chunk(N)
+    if buffer is None:
+        buffer = host_buffer(X_host.dtype, Cin, Cout, chunk, dev)
+    Y = out if out is not None else torch.empty((N, Cout), dtype=torch.float32).pin_memory()
+    if Y.is_cuda or not Y.is_contiguous() or Y.dtype != torch.float32:
+        raise ValueError("out must be a contiguous fp32 host tensor")
+    key = (dev.index if dev.index is not None else torch.cuda.current_device())
+    if key not in _copy_streams:
+        _copy_streams[key] = (torch.cuda.Stream(dev), torch.cuda.Stream(dev))
+    s_in, s_out = _copy_streams[key]
+    code = lib().cci_linear_host(X_host.data_ptr(), _dtype_code(X_host), N, Cin, values.data_ptr(),
+                                 idx.data_ptr(), Cout, G, K, Y.data_ptr(), chunk, buffer.data_ptr(),
+                                 buffer.numel(), status.data_ptr() if status is not None else None,
+                                 _stream(dev), s_in.cuda_stream, s_out.cuda_stream)
+    _check(code, "cci_linear_host")
     return Y
 
 

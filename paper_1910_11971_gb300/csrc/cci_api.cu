@@ -210,21 +210,15 @@ struct Epilogue {
     int out_bf16;
 };
 
-cci_status linear_impl(const void *X, int dtype, int64_t N, int64_t Cin, const void *values, const uint8_t *idx,
-                       int64_t Cout, int G, int K, void *Y, uint32_t *dev_status, cci_algo algo, void *workspace,
-                       size_t workspace_bytes, cci_stream_t stream, Epilogue e)
+// parameters of the product Y[N][Cout] = X[N][Cin] * Wd^T (fp32 output, no epilogue)
+FwdParams linear_params(const void *X, int64_t N, int64_t Cin, const void *values, const uint8_t *idx,
+                        int64_t Cout, float *Y, uint32_t *dev_status)
 {
-    const cci_status st = check_common(X, dtype, values, idx, static_cast<float *>(Y), N, Cout, Cin, G, K);
-    if (st != CCI_OK) return st;
-    if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
     FwdParams p{};
     p.X = X;
     p.values = values;
     p.idx = idx;
-    p.Y = static_cast<float *>(Y);
-    p.bias = e.bias;
-    p.relu = e.relu;
-    p.out_bf16 = e.out_bf16;
+    p.Y = Y;
     p.status = dev_status;
     p.N = N;
     p.Cout = Cout;
@@ -234,6 +228,20 @@ cci_status linear_impl(const void *X, int dtype, int64_t N, int64_t Cin, const v
     p.KH = p.KW = p.sh = p.sw = 1;
     p.ph = p.pw = 0;
     p.is_conv = 0;
+    return p;
+}
+
+cci_status linear_impl(const void *X, int dtype, int64_t N, int64_t Cin, const void *values, const uint8_t *idx,
+                       int64_t Cout, int G, int K, void *Y, uint32_t *dev_status, cci_algo algo, void *workspace,
+                       size_t workspace_bytes, cci_stream_t stream, Epilogue e)
+{
+    const cci_status st = check_common(X, dtype, values, idx, static_cast<float *>(Y), N, Cout, Cin, G, K);
+    if (st != CCI_OK) return st;
+    if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
+    FwdParams p = linear_params(X, N, Cin, values, idx, Cout, static_cast<float *>(Y), dev_status);
+    p.bias = e.bias;
+    p.relu = e.relu;
+    p.out_bf16 = e.out_bf16;
     return forward(p, dtype, G, K, algo, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream));
 }
 
@@ -569,4 +577,130 @@ extern "C" cci_status cci_linear_dense_tc_static(const void *X, cci_dtype dtype,
     if (a != CCI_OK) return a;
     return cci_linear_ws(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, CCI_ALGO_DENSE_TC_WS, ws,
                          kStaticWsBytes, stream);
+}
+
+// ---------------------------------------------------------------------------
+// The product over host buffers: X read from host memory and Y written back to
+// it, in chunks of columns pipelined over three streams (copy in, product, copy
+// out) so that the copies of one chunk overlap the product of another.  The
+// caller's device buffer holds the dense-weight workspace and two staging slots
+// per direction.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr int kHostSlots = 2;  // staging slots per direction: chunk c + 1 in, c computed, c - 1 out
+
+size_t round256(size_t b) { return (b + 255) / 256 * 256; }
+
+struct HostLayout {
+    size_t ws, xslot, yslot, total;
+};
+
+bool host_layout(int dtype, int64_t Cin, int64_t Cout, int64_t chunk, HostLayout *l)
+{
+    if (!valid_dtype(dtype) || Cin < 1 || Cout < 1 || chunk < 1 || !mul_ok(chunk, Cin) || !mul_ok(chunk, Cout) ||
+        !mul_ok(Cout, Cin))
+        return false;
+    l->ws = round256(dense_ws_bytes(dtype, Cout, Cin));
+    l->xslot = round256(static_cast<size_t>(chunk) * static_cast<size_t>(Cin) * elem_size(dtype));
+    l->yslot = round256(static_cast<size_t>(chunk) * static_cast<size_t>(Cout) * 4);
+    l->total = l->ws + kHostSlots * (l->xslot + l->yslot);
+    return true;
+}
+
+}  // namespace
+
+extern "C" size_t cci_linear_host_buffer_size(cci_dtype dtype, int64_t Cin, int64_t Cout, int64_t chunk_cols)
+{
+    HostLayout l;
+    return host_layout(dtype, Cin, Cout, chunk_cols, &l) ? l.total : 0;
+}
+
+extern "C" cci_status cci_linear_host(const void *X_host, cci_dtype dtype, int64_t N, int64_t Cin,
+                                      const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
+                                      float *Y_host, int64_t chunk_cols, void *device_buffer,
+                                      size_t device_buffer_bytes, uint32_t *dev_status, cci_stream_t stream,
+                                      cci_stream_t copy_in_stream, cci_stream_t copy_out_stream)
+{
+    const cci_status st = check_common(X_host, dtype, values, idx, Y_host, N, Cout, Cin, G, K);
+    if (st != CCI_OK) return st;
+    if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
+    if (chunk_cols < 1) return CCI_ERR_SHAPE;
+    const bool tc_fits = Cin < (int64_t(1) << 31) && Cout < (int64_t(1) << 31);
+    if (!tc_fits || !dense_tc_shape_ok(dtype, G, K, Cin, Cin)) return CCI_ERR_UNSUPPORTED;
+    HostLayout l;
+    if (!host_layout(dtype, Cin, Cout, chunk_cols, &l)) return CCI_ERR_SHAPE;
+    if (!device_buffer || device_buffer_bytes < l.total || !aligned(device_buffer, 256)) return CCI_ERR_WORKSPACE;
+    if (N == 0) return CCI_OK;
+
+    const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    const cudaStream_t si = copy_in_stream ? reinterpret_cast<cudaStream_t>(copy_in_stream) : cs;
+    const cudaStream_t so = copy_out_stream ? reinterpret_cast<cudaStream_t>(copy_out_stream) : cs;
+    // events: [0] the call's start on `stream`; per slot k: chunk in (1 + k),
+    // product done (1 + S + k), chunk out (1 + 2S + k)
+    constexpr int kEv = 1 + 3 * kHostSlots;
+    cudaEvent_t ev[kEv] = {};
+    for (int i = 0; i < kEv; ++i) {
+        if (cudaEventCreateWithFlags(&ev[i], cudaEventDisableTiming) != cudaSuccess) {
+            for (int j = 0; j < i; ++j) cudaEventDestroy(ev[j]);
+            return CCI_ERR_CUDA;
+        }
+    }
+    cudaEvent_t *ev_in = ev + 1, *ev_done = ev + 1 + kHostSlots, *ev_out = ev + 1 + 2 * kHostSlots;
+    char *const base = static_cast<char *>(device_buffer);
+    void *const ws = base;
+    char *const xs = base + l.ws;
+    char *const ys = xs + kHostSlots * l.xslot;
+    const size_t es = elem_size(dtype);
+    const int64_t chunks = (N + chunk_cols - 1) / chunk_cols;
+
+    // the copy streams start after the work the caller enqueued on `stream` before this call
+    cudaError_t e = cudaEventRecord(ev[0], cs);
+    if (e == cudaSuccess && si != cs) e = cudaStreamWaitEvent(si, ev[0], 0);
+    if (e == cudaSuccess && so != cs) e = cudaStreamWaitEvent(so, ev[0], 0);
+    cci_status result = to_status(e);
+    int64_t issued = 0;  // chunks whose copy-out was enqueued
+    for (int64_t c = 0; c < chunks && result == CCI_OK; ++c) {
+        const int k = static_cast<int>(c % kHostSlots);
+        const int64_t n0 = c * chunk_cols;
+        const int64_t nc = (N - n0) < chunk_cols ? (N - n0) : chunk_cols;
+        char *const xd = xs + k * l.xslot;
+        float *const yd = reinterpret_cast<float *>(ys + k * l.yslot);
+        // copy in, once the product of the chunk that last used this slot has read it
+        if (c >= kHostSlots) e = cudaStreamWaitEvent(si, ev_done[k], 0);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(xd, static_cast<const char *>(X_host) + static_cast<size_t>(n0) * Cin * es,
+                                static_cast<size_t>(nc) * Cin * es, cudaMemcpyHostToDevice, si);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_in[k], si);
+        // product, once the chunk is in and the copy-out of this slot's last output is done
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, ev_in[k], 0);
+        if (e == cudaSuccess && c >= kHostSlots) e = cudaStreamWaitEvent(cs, ev_out[k], 0);
+        result = to_status(e);
+        if (result != CCI_OK) break;
+        FwdParams p = linear_params(xd, nc, Cin, values, idx, Cout, yd, dev_status);
+        if (c == 0) {
+            // the first chunk decompresses the weights into the workspace
+            result = forward(p, dtype, G, K, CCI_ALGO_DENSE_TC_WS, ws, l.ws, cs);
+        } else {
+            p.wdense = ws;
+            result = to_status(launch_gemm_ws(p, dtype, cs));
+        }
+        if (result != CCI_OK) break;
+        e = cudaEventRecord(ev_done[k], cs);
+        // copy out, once the product is done
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(so, ev_done[k], 0);
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(Y_host + static_cast<size_t>(n0) * Cout, yd, static_cast<size_t>(nc) * Cout * 4,
+                                cudaMemcpyDeviceToHost, so);
+        if (e == cudaSuccess) e = cudaEventRecord(ev_out[k], so);
+        result = to_status(e);
+        if (result == CCI_OK) issued = c + 1;
+    }
+    // the call completes on `stream`: it waits for every copy-out enqueued
+    for (int k = 0; k < kHostSlots && k < issued; ++k) {
+        const cudaError_t w = cudaStreamWaitEvent(cs, ev_out[k], 0);
+        if (result == CCI_OK) result = to_status(w);
+    }
+    for (int i = 0; i < kEv; ++i) cudaEventDestroy(ev[i]);  // released once their last record completes
+    return result;
 }
