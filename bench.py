@@ -232,11 +232,13 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 def oracle_rate(case: wl.LinearCase, seconds: float):
     """Nonzero TFLOP/s of the oracle on the first `rows` columns of the workload,
-    with `rows` grown until one call takes about `seconds`."""
+    with `rows` grown until one call takes about `seconds`; when the whole
+    workload takes less, whole passes repeat until `seconds` have elapsed.
+    Returns (rate, rows, passes, seconds spent, threads)."""
     import numpy as np
 
     import oracle
-    X, W = wl.linear_inputs(case, N=min(case.N, 65536))
+    X, W = wl.linear_inputs(case)
     Xf = X.to(torch.float64).numpy()
     v, i = oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
     Wd, mask = oracle.decompress(v, i, case.Cout, case.G)
@@ -248,8 +250,14 @@ def oracle_rate(case: wl.LinearCase, seconds: float):
         if dt >= seconds or rows >= Xf.shape[0]:
             break
         rows = min(Xf.shape[0], int(rows * max(2.0, 1.2 * seconds / max(dt, 1e-3))))
-    flops = 2.0 * rows * case.R * case.Cout * case.K / case.G
-    return flops / dt / 1e12, rows, dt, oracle.threads()
+    passes, total = 1, dt
+    while total < seconds:
+        t0 = time.perf_counter()
+        oracle.linear(Xf[:rows], Wd, mask)
+        total += time.perf_counter() - t0
+        passes += 1
+    flops = 2.0 * rows * case.R * case.Cout * case.K / case.G * passes
+    return flops / total / 1e12, rows, passes, total, oracle.threads()
 
 
 def run_reference(args, rank, world):
@@ -498,6 +506,14 @@ def run_ours(args, rank, world, local):
     metric_roofline = {"definition": "max(nonzero flops / CUDA-core FMA peak, compressed bytes / 8 TB/s)",
                        "floor_us": floor_s * 1e6, "frac": floor_s / (lin_avg * 1e-3),
                        "fma_peak_tflops": ALU_PEAK_TFLOPS}
+    # the product's absolute rates (decompression + GEMM time): nonzero and
+    # dense-equivalent flops, algorithmic bytes
+    gbs = alg_bytes / (lin_avg * 1e-3) / 1e9
+    absolute = {"nonzero_tflops": achieved,
+                "dense_equiv_tflops": case.dense_flops() / (lin_avg * 1e-3) / 1e12,
+                "gbs": gbs, "gbs_frac_of_measured_hbm": gbs / measured_peaks()["hbm_gbs"],
+                "gbs_frac_of_8tbs": gbs / HBM_ROOF_GBS,
+                "nonzero_frac_of_fma_peak": achieved / ALU_PEAK_TFLOPS}
 
     # ---- end to end through the public API: W host -> device and packed, then
     # cci_linear_host: X from pinned host memory, Y back to it, in column chunks
@@ -550,10 +566,10 @@ def run_ours(args, rank, world, local):
 
     cpu = None
     if rank == 0 and world == 1:
-        rate, rows, dt, cores = oracle_rate(case, args.cpu_sample_seconds)
+        rate, rows, passes, dt, cores = oracle_rate(case, args.cpu_sample_seconds)
         cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"first {rows} of {case.N} columns, one fp64 dense-mask product "
-                         f"({dt:.1f} s), nonzero flops counted"}
+               "sample": f"{passes} pass(es) of the fp64 dense-mask product over the first {rows} of "
+                         f"{case.N} columns ({dt:.1f} s in all), nonzero flops counted"}
 
     if rank == 0:
         line = {
@@ -562,13 +578,21 @@ def run_ours(args, rank, world, local):
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": config_of(case), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
             "gpu_launches": (3 if on_tc else 2) * args.steps, "clocks": clk.summary(),
-            "metric_roofline": metric_roofline,
+            "metric_roofline": metric_roofline, "absolute": absolute,
             "breakdown_ms": {"pack": statistics.mean(pack_ms), "linear": lin_avg,
                              "wall_per_step_incl_flush": t_wall * 1e3 / args.steps},
             "dense_reference": dense, "cuda_core_families": families, **extras,
         }
         print(json.dumps(line), flush=True)
     return 0
+
+
+def algorithmic_bytes(case, elem: int) -> int:
+    """Bytes a product or convolution must move at least: its input once (the
+    NHWC tensor for a convolution), its fp32 output once and the packed weights
+    (values and uint8 indices)."""
+    x = case.B * case.H * case.W * case.Cin if isinstance(case, wl.ConvCase) else case.N * case.Cin
+    return x * elem + case.N * case.Cout * 4 + (case.Cout // case.G) * case.R * case.K * (elem + 1)
 
 
 def run_extras(cci, dev, stream, flush):
@@ -609,8 +633,9 @@ def run_extras(cci, dev, stream, flush):
                                   "dense_tc_ws_ms": ms_ws,
                                   "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
                                   "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
+                                  "gbs": algorithmic_bytes(case, 2) / (ms * 1e-3) / 1e9,
                                   "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R,
-                                                            case.Cout, G, K)})
+                                                            case.Cout, G, K, cci.ALGO_DENSE_TC_WS)})
         del X, W, v, i, Y, Wm, ws
     case = wl.CONV3X3_28
     X, W = wl.conv_inputs(case, device=str(dev))
@@ -640,8 +665,10 @@ def run_extras(cci, dev, stream, flush):
                          "dense_tc_ws_ms": ms_ws, "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
                          "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
                          "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
+                         "dense_equiv_tflops": case.dense_flops() / (ms * 1e-3) / 1e12,
+                         "gbs": algorithmic_bytes(case, 2) / (ms * 1e-3) / 1e9,
                          "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R, case.Cout,
-                                                   case.G, case.K)}
+                                                   case.G, case.K, cci.ALGO_DENSE_TC_WS)}
     out["resnet50_stack"] = run_resnet_stack(cci, dev, stream, flush)
     out["mobilenetv2_pointwise"] = run_pointwise_stack(cci, dev, stream, flush)
     out["allocation_error"] = run_allocation_error(cci, dev, stream, flush)
