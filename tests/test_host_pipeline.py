@@ -124,3 +124,30 @@ def test_host_product_orders_after_prior_work_and_reuses_the_buffer():
         _, _, Wo, mask = oracle_reference(W, G, K)
         Yo, S = oracle.linear(f64(X), Wo, mask)
         assert_within_tol(f64(Yh), Yo, S, f"call {seed}")
+
+
+@pytest.mark.gpu
+def test_host_product_bottleneck_full():
+    """The benchmark's end-to-end call at full size (N = 100352, 256 -> 1024, G = 8,
+    K = 2, fp32, 12544-column chunks): every output equals the device-resident
+    product, and sampled rows (tile and chunk edges, the tail, random ones) are
+    within tolerance of the oracle."""
+    from parity_util import sample_rows
+    cci_build.build()
+    dev = torch.device("cuda:0")
+    case = wl.BOTTLENECK_1X1
+    X, W = wl.linear_inputs(case)
+    v, i = cci.pack(W.to(dev), case.G, case.K)
+    chunk = cci.host_chunk(case.N)
+    assert chunk == 12544
+    st = cci.new_status(dev)
+    Yh = cci.linear_host(X.pin_memory(), v, i, case.Cout, case.G, case.K, status=st, chunk=chunk)
+    torch.cuda.current_stream(dev).synchronize()
+    assert cci.read_status(st) == 0
+    Yd = cci.linear(X.to(dev), v, i, case.Cout, case.G, case.K, algo=cci.ALGO_DENSE_TC_WS).cpu()
+    assert bool((Yh.view(torch.int32) == Yd.view(torch.int32)).all())
+    edges = np.concatenate([np.arange(c * chunk - 2, c * chunk + 2) for c in range(1, case.N // chunk)])
+    rows = np.unique(np.concatenate([sample_rows(case.N, 1024, seed=5), edges]))
+    _, _, Wo, mask = oracle_reference(W, case.G, case.K)
+    Yo, S = oracle.linear(f64(X[rows]), Wo, mask)
+    assert_within_tol(f64(Yh[torch.from_numpy(rows)]), Yo, S, "bottleneck_1x1 through cci_linear_host")
