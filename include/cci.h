@@ -386,6 +386,21 @@ int cci_version(void);
  */
 cci_status cci_fma_probe(float *out, int blocks, int threads, int iters, cci_stream_t stream);
 
+/*
+ * cci_wait_probe -- diagnostic of the bounded waits inside the tensor-core
+ * kernels (a safety mechanism of this library; the paper has no counterpart).
+ * One thread initialises an mbarrier that expects one arrival, arrives on it if
+ * `arrive` is nonzero, and waits for the barrier's phase exactly as the kernels
+ * wait for their copies and MMAs.  With the arrival the wait returns at once and
+ * nothing is reported.  Without it nothing can complete the phase: the wait
+ * gives up after 2^31 SM clock cycles (about one second), ORs bit
+ * (1u << CCI_ERR_TIMEOUT) into *dev_status and the kernel returns, leaving the
+ * context usable.
+ *   dev_status  device uint32, required
+ * Errors: CCI_ERR_NULL, CCI_ERR_CUDA.
+ */
+cci_status cci_wait_probe(uint32_t *dev_status, int arrive, cci_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -67,6 +67,7 @@ SIGNATURES = {
     "cci_decode_device_status": (_I32, [ctypes.c_uint32]),
     "cci_version": (_I32, []),
     "cci_fma_probe": (_I32, [_P, _I32, _I32, _I32, _P]),
+    "cci_wait_probe": (_I32, [_U32P, _I32, _P]),
 }
 
 _lib = None

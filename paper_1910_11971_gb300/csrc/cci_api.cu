@@ -528,6 +528,12 @@ cci_status cci_fma_probe(float *out, int blocks, int threads, int iters, cci_str
     return to_status(launch_fma_probe(out, blocks, threads, iters, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+cci_status cci_wait_probe(uint32_t *dev_status, int arrive, cci_stream_t stream)
+{
+    if (!dev_status) return CCI_ERR_NULL;
+    return to_status(launch_wait_probe(dev_status, arrive, reinterpret_cast<cudaStream_t>(stream)));
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------------------

@@ -299,7 +299,31 @@ cudaError_t launch(const FwdParams &p, cudaStream_t stream)
     return cudaGetLastError();
 }
 
+// Diagnostic of the bounded waits above: one thread initialises an mbarrier that
+// expects one arrival, arrives on it when `arrive` is set, and waits for its
+// phase with mbar_wait.  Without the arrival nothing can complete the phase, the
+// wait gives up after kWaitLimit cycles and reports CCI_ERR_TIMEOUT; nothing is
+// in flight, so the kernel then simply returns.
+__global__ void wait_probe_kernel(uint32_t *status, int arrive)
+{
+    __shared__ uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        if (arrive) mbar_arrive(&bar);
+        mbar_wait(&bar, 0, &abort_flag, status);
+    }
+}
+
 }  // namespace tc
+
+cudaError_t launch_wait_probe(uint32_t *status, int arrive, cudaStream_t stream)
+{
+    tc::wait_probe_kernel<<<1, 32, 0, stream>>>(status, arrive);
+    return cudaGetLastError();
+}
 
 // ===========================================================================
 // One-pass decompression of the packed weights into the workspace of

@@ -18,6 +18,8 @@ cudaError_t launch_pack_stats(const void *W, int dtype, int64_t Cout, int64_t R,
                               unsigned long long *counts, cudaStream_t stream);
 cudaError_t launch_generic(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);
 cudaError_t launch_fma_probe(float *out, int blocks, int threads, int iters, cudaStream_t stream);
+// bounded-wait diagnostic (cci_dense_tc.cu): arrive = 0 lets the wait expire
+cudaError_t launch_wait_probe(uint32_t *status, int arrive, cudaStream_t stream);
 
 // dense tensor-core comparison kernel (tcgen05, bf16 only)
 bool dense_tc_supported(int dtype, int G, int K);

@@ -467,6 +467,28 @@ def test_tf32x3_small(dev, case):
     assert_within_tol(f64(Y), Yo, S, str(case))
 
 
+@pytest.mark.parametrize("algo", [cci.ALGO_DENSE_TC_WS, cci.ALGO_GENERIC], ids=["tf32x3", "generic"])
+def test_fp32_wide_exponent_range(dev, algo):
+    """Every activation row and every group of G output channels of W carries its
+    own power-of-two scale (2^-30 .. 2^30), so the per-output scale S spans ~35 orders of
+    magnitude: the product must hold |err| <= 1e-5 * S for each output (no absolute
+    error floor; for the three-pass tf32 split, hi and lo keep fp32's exponent
+    range)."""
+    N, Cin, Cout, G, K = 700, 256, 256, 8, 2
+    g = torch.Generator().manual_seed(2024)
+    X = torch.randn((N, Cin), generator=g) * torch.pow(2.0, torch.randint(-30, 31, (N, 1), generator=g).float())
+    # one scale per group of G output channels: every channel keeps weights (a scale
+    # per channel would let the two largest-scaled channels of a group win every r)
+    wsc = torch.pow(2.0, torch.randint(-30, 31, (Cout // G, 1, 1), generator=g).float())
+    W = (torch.randn((Cout // G, G, Cin), generator=g) * wsc).reshape(Cout, Cin)
+    X[::7, ::5] = 0.0  # exact zeros among the activations (ReLU-like)
+    Y = run_linear(dev, X, W, G, K, algo)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert float(S[S > 0].max() / S[S > 0].min()) > 1e30  # this draw: ~4e35
+    assert_within_tol(f64(Y), Yo, S, "fp32 wide exponent range")
+
+
 def test_tf32x3_bottleneck_full(dev):
     case = wl.BOTTLENECK_1X1
     X, W = wl.linear_inputs(case)
