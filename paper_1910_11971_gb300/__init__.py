@@ -213,7 +213,8 @@ _copy_streams = {}
 def host_chunk(N: int) -> int:
     """Default columns per chunk of ``linear_host``: about an eighth of N, in
     whole 128-column tiles."""
-    return max(128, -(-(-(-N // 8)) // 128) * 128)
+    eighth = (N + 7) // 8
+    return max(128, (eighth + 127) // 128 * 128)
 
 
 def host_buffer(dtype: torch.dtype, Cin: int, Cout: int, chunk: int, device) -> torch.Tensor:
