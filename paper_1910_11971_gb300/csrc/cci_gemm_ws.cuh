@@ -41,7 +41,8 @@
 // overlaps the producers' work), stage by stage in turn: the copies one thread
 // issues are processed one box after another (measured on GB300: about 0.5 us
 // per box of 16-64 KB from one issuer; copy throughput grows with the number of
-// issuing warps), so up to four warps issue.  Every mbarrier wait is bounded
+// issuing warps), so up to six warps issue (one per stage in flight).  Every
+// mbarrier wait is bounded
 // (CCI_ERR_TIMEOUT, abort flag, drain, TMEM freed).
 #pragma once
 
@@ -129,7 +130,7 @@ struct Cfg {
     // more boxes moving.  kIssuers <= kStages keeps every empty-barrier wait
     // within one phase of the barrier (no parity aliasing).
     // (kAHalo: one more warp, which copies the halos)
-    static constexpr int kIssuers = ASRC == kAGather ? 1 : (kStages < 4 ? kStages : 4) + (kHalo ? 1 : 0);
+    static constexpr int kIssuers = ASRC == kAGather ? 1 : (kStages < 6 ? kStages : 6) + (kHalo ? 1 : 0);
     static constexpr int kThreads = 32 * (9 + kIssuers);
     static_assert(kIssuers - (kHalo ? 1 : 0) >= 1 && kIssuers - (kHalo ? 1 : 0) <= kStages,
                   "stage issuers must not outnumber the stages");
