@@ -1,21 +1,23 @@
 """Benchmark of the CCI-sparse forward layer (arXiv 1910.11971) on GB300.
 
-Default workload: the ResNet 1x1 bottleneck as a CCI product, fp32:
-N = 32*56*56 = 100352 columns, 256 -> 1024 channels, G = 8, K = 2 (75% sparse),
-W ~ N(0, 2/256), X = ReLU(N(0, 1)), seeded synthetic data.
+Headline workload: the K/G sweep, a 4096 -> 4096 product over N = 8192 columns
+in bf16 (W ~ N(0, 1/4096), X ~ N(0, 1), seeded synthetic data), at its middle
+point G = 8, K = 2 (75 % sparse).  One step = the whole hot path on one batch:
+cci_pack of the dense weights (per-group top-K, Sec. 3.1 / 5.1) + the product
+(Alg. 2) through the library's production path, inputs resident in HBM.  The
+metric is nonzero TFLOP/s (2*N*R*Cout*K/G per step).  L2 (129 MB) is flushed
+between timed steps by writing a 256 MB buffer outside the timed events.
 
-One step = the whole hot path on one batch: cci_pack of the dense weights
-(per-group top-K) + cci_linear (scatter-accumulate), inputs resident in HBM.
-The metric is nonzero TFLOP/s (2*N*R*Cout*K/G per step); the roofline is the
-CUDA-core FMA peak (the path is bound by fp32 FMA, not HBM).  L2 (129 MB) is
-flushed between timed steps by writing a 256 MB buffer outside the timed events.
+stdout gets ONE short JSON line, last: the headline with its roofline, CPU
+baseline (the fp64 oracle on a bounded sample), end-to-end figure (host buffers,
+copies inside the timed region), clocks, and a compact per-(G, K) array of the
+sweep.  Every other measurement (fp32 bottleneck, 3x3 convolution, ResNet-50 and
+MobileNetV2 stacks, Eq. 1, targeted dropout, CCI against balanced sparsity) is
+printed to stderr, one JSON line each.
 
 ``--impl reference`` times the fp64 CPU oracle on a bounded sample of the same
-workload instead (the reported CPU baseline).
-
-Prints one JSON line (rank 0).  Multi-GPU (torchrun): every rank runs its own
-batch (weak scaling, no collective on the data path); the step time is the max
-over ranks.
+workload instead.  Multi-GPU (torchrun): every rank runs its own batch (weak
+scaling, no collective on the data path); the step time is the max over ranks.
 """
 from __future__ import annotations
 
@@ -46,6 +48,9 @@ N_SM, FMA_LANES, SM_MAX_GHZ = 152, 128, 2.070
 ALU_PEAK_TFLOPS = N_SM * FMA_LANES * 2 * SM_MAX_GHZ / 1e3
 L2_FLUSH_BYTES = 256 << 20
 HBM_ROOF_GBS = 8000.0  # the workload's stated memory roof (8 TB/s)
+HEADLINE = wl.sweep_case(8, 2)  # the middle point of the K/G sweep
+# --algo names -> cci_algo values (profiling runs only)
+ALGOS = {"auto": 0, "generic": 1, "regtile": 2, "fused": 3, "expand": 4, "ws": 5}
 
 
 def measured_peaks():
@@ -67,17 +72,20 @@ def tensor_peak(dtype_name: str) -> float:
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--extras", type=int, default=1, help="also measure the sweep / conv workloads")
+    ap.add_argument("--extras", type=int, default=1,
+                    help="also measure the other workloads (stderr, one JSON line each)")
     ap.add_argument("--cpu-sample-seconds", type=float, default=12.0)
     ap.add_argument("--profile", type=int, default=0,
                     help="only the warm-up and timed steps of the main path (for ncu)")
-    ap.add_argument("--workload", default="bottleneck_1x1",
-                    help="bottleneck_1x1 (default) or sweep_4096_G<G>_K<K>: the product timed; with "
+    ap.add_argument("--workload", default=HEADLINE.name,
+                    help="sweep_4096_G<G>_K<K> (default G8_K2) or bottleneck_1x1: the product timed; with "
                          "--profile 1 also a convolution: conv3x3_28, resnet50_lNN_K<K> (layer NN of "
                          "the ResNet-50 stack) or mobilenetv2_pwNN (pointwise layer NN of MobileNetV2)")
+    ap.add_argument("--algo", default="auto", choices=sorted(ALGOS),
+                    help="with --profile 1: the kernel family of the timed product")
     return ap.parse_args()
 
 
@@ -206,7 +214,7 @@ class ClockSampler:
                         reasons.add(name)
             return {"sm_mhz": statistics.median(s[0] for s in self.samples),
                     "sm_max_mhz": max(s[1] for s in self.samples), "reasons": sorted(reasons),
-                    "samples": len(self.samples), "source": "nvml"}
+                    "samples": len(self.samples)}
         sm, smax, reasons = [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
         for ln in self.smi_lines:
@@ -261,29 +269,30 @@ def oracle_rate(case: wl.LinearCase, seconds: float):
 
 
 def run_reference(args, rank, world):
-    case = wl.BOTTLENECK_1X1
+    """The reference arm: the fp64 oracle (pack, decompression, dense-mask product)
+    on the host cores, on a bounded sample of the headline workload per step."""
+    case = workload_case(args.workload)
     if rank != 0:
         return 0
-    import numpy as np  # noqa: F401
-
     import oracle
     X, W = wl.linear_inputs(case, N=4096)
     Xf = X.to(torch.float64).numpy()
+    Wf = W.to(torch.float64).numpy()
     # size one step's sample so that warmup + steps stay within a few minutes
-    v, i = oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
+    v, i = oracle.pack(Wf, case.G, case.K)
     Wd, mask = oracle.decompress(v, i, case.Cout, case.G)
-    rows = 256
+    rows = 16
     t0 = time.perf_counter()
     oracle.linear(Xf[:rows], Wd, mask)
     dt = time.perf_counter() - t0
     budget = 90.0 / max(1, args.steps + args.warmup)
-    rows = max(16, min(Xf.shape[0], int(rows * budget / max(dt, 1e-4))))
+    rows = max(4, min(Xf.shape[0], int(rows * budget / max(dt, 1e-4))))
     for _ in range(args.warmup):
-        oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
+        oracle.pack(Wf, case.G, case.K)
         oracle.linear(Xf[:rows], Wd, mask)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        vv, ii = oracle.pack(W.to(torch.float64).numpy(), case.G, case.K)
+        vv, ii = oracle.pack(Wf, case.G, case.K)
         Wd, mask = oracle.decompress(vv, ii, case.Cout, case.G)
         oracle.linear(Xf[:rows], Wd, mask)
     dt = (time.perf_counter() - t0) / args.steps
@@ -292,26 +301,40 @@ def run_reference(args, rank, world):
     sample = (f"{rows} of {case.N} columns per step (pack + decompress + dense-mask product in "
               f"fp64), {case.Cin}->{case.Cout}, G={case.G}, K={case.K}")
     line = {
-        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+        "impl": "reference", "metric": METRIC, "value": sig(value), "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": sig(dt * 1e3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": config_of(case, extra={"sample_columns": rows}),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+        "cpu_baseline": {"value": sig(value), "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
                          "sample": sample},
-        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "e2e": {"value": sig(value), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
 
 
+def sig(x, n: int = 4):
+    """x rounded to n significant digits (keeps the headline line short)."""
+    if x is None or not isinstance(x, (int, float)) or x == 0 or not math.isfinite(x):
+        return x
+    return float(f"{x:.{n}g}")
+
+
 def config_of(case, extra=None):
     c = {"workload": case.name, "N": case.N, "Cin": case.Cin, "Cout": case.Cout, "G": case.G,
-         "K": case.K, "sparsity": 1 - case.K / case.G, "dtype_in": case.dtype,
-         "l2": "flushed between timed steps (256 MB write outside the timed events)",
-         "parallelism": "one independent batch per GPU"}
+         "K": case.K, "dtype_in": case.dtype, "l2": "flushed (256 MB write, untimed)",
+         "parallelism": "one batch/GPU"}
+    if case.name.startswith("sweep_4096"):
+        c["workload"] = f"sweep_4096 (K/G sweep, 11 points); value at G={case.G} K={case.K}"
     if extra:
         c.update(extra)
     return c
+
+
+def extra(name: str, payload) -> None:
+    """One measurement beside the headline, as its own JSON line on stderr (the
+    headline stays the last, short line on stdout)."""
+    print(json.dumps({"extra": name, "data": payload}), file=sys.stderr, flush=True)
 
 
 # ---------------------------------------------------------------------------
@@ -385,7 +408,7 @@ def profile_conv(cci, case, args, dev, stream):
     values = torch.empty((case.Cout // case.G, case.R, case.K), dtype=X.dtype, device=dev)
     idx = torch.empty((case.Cout // case.G, case.R, case.K), dtype=torch.uint8, device=dev)
     Y = torch.empty((case.B, case.P, case.Q, case.Cout), dtype=torch.float32, device=dev)
-    ws = cci.new_workspace(cci.ALGO_AUTO, X.dtype, case.Cout, case.R, dev)
+    ws = cci.auto_workspace(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, dev)
     status = cci.new_status(dev)
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
 
@@ -402,6 +425,24 @@ def profile_conv(cci, case, args, dev, stream):
     print(json.dumps({"workload": case.name, "ms_per_step": statistics.mean(ms), "steps": args.steps,
                       "note": "profiling helper: pack + convolution per step"}), flush=True)
     return 0
+
+
+def dense_planes(W: torch.Tensor) -> torch.Tensor:
+    """Unpruned weights in the dense family's layout, for the same-kernel dense
+    line: bf16 as is; fp32 as the hi / lo tf32 planes (hi = low 13 mantissa bits
+    cleared, lo = w - hi)."""
+    if W.dtype == torch.bfloat16:
+        return W.contiguous()
+    hi = (W.view(torch.int32) & -8192).view(torch.float32)
+    return torch.stack([hi, W - hi]).contiguous()
+
+
+def launches_per_product(cci, dtype, case) -> int:
+    """Kernels one product launches on the production path (AUTO): the workspace
+    family runs a decompression and the GEMM, every other family one kernel."""
+    name = cci.kernel_name(dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
+                           workspace=True)
+    return 2 if name.startswith("dense_tc_ws") else 1
 
 
 def run_ours(args, rank, world, local):
@@ -427,29 +468,34 @@ def run_ours(args, rank, world, local):
     values = torch.empty((case.Cout // case.G, case.R, case.K), dtype=Xd.dtype, device=dev)
     idx = torch.empty((case.Cout // case.G, case.R, case.K), dtype=torch.uint8, device=dev)
     Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
-    # the library's production path: AUTO with a workspace (the dense tensor-core
-    # family when the layer has one, else the CUDA-core family)
-    ws = cci.new_workspace(cci.ALGO_AUTO, Xd.dtype, case.Cout, case.R, dev)
-    kname = cci.kernel_name(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_DENSE_TC_WS)
-    on_tc = bool(kname) and ws is not None
-    if not on_tc:
-        kname = cci.kernel_name(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K)
+    # the library's production path: AUTO (with the workspace it asks for, if any)
+    algo = ALGOS[args.algo] if args.profile else cci.ALGO_AUTO
+    if algo == cci.ALGO_AUTO:
+        ws = cci.auto_workspace(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K, dev)
+    else:
+        ws = cci.new_workspace(algo, Xd.dtype, case.Cout, case.R, dev)
+    kname = cci.kernel_name(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
+                            workspace=ws is not None)
+    on_tc = kname.startswith("dense_tc")
     status = cci.new_status(dev)
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
 
     def flush():
         flush_buf.fill_(1.0)
 
+    def product():
+        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status, algo=algo, workspace=ws)
+
     def step():
         cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
-        cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status, workspace=ws)
+        product()
 
     for _ in range(max(3, args.warmup)):
         step()
     torch.cuda.synchronize(dev)
     assert cci.read_status(status) == 0
 
-    # ---- timed region: K steps, per-step events (pack | linear), L2 flushed between ----
+    # ---- timed region: K steps, per-step events (pack | product), L2 flushed between ----
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
            torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     barrier(world)
@@ -462,7 +508,7 @@ def run_ours(args, rank, world, local):
             a.record(stream)
             cci.pack(Wd, case.G, case.K, status=status, check=False, out=(values, idx))
             b.record(stream)
-            cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, status=status, workspace=ws)
+            product()
             c.record(stream)
         torch.cuda.synchronize(dev)
         t_wall = time.perf_counter() - t_wall0
@@ -478,42 +524,25 @@ def run_ours(args, rank, world, local):
     value = world * nzf / (ms_step * 1e-3) / 1e12
     lin_avg = statistics.mean(lin_ms)
     achieved = nzf / (lin_avg * 1e-3) / 1e12
-    alg_bytes = (case.N * case.Cin * X.element_size() + case.N * case.Cout * 4
-                 + (case.Cout // case.G) * case.R * case.K * (X.element_size() + 1))
+    es = X.element_size()
+    alg_bytes = algorithmic_bytes(case, es)
+    tdt = "bf16" if X.dtype == torch.bfloat16 else "tf32"
     if on_tc:
-        tdt = "bf16" if X.dtype == torch.bfloat16 else "tf32"
         passes = 1 if tdt == "bf16" else 3
         peak = tensor_peak(tdt)
         executed = passes * case.dense_flops()
-        roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                    "frac": achieved / peak, "traffic": measured_traffic(kname), "kernel": kname,
-                    "peak_source": f"measured bf16 burst {measured_peaks()['bf16_tflops']} TFLOP/s"
-                                   + (" x nominal tf32/bf16 ratio 1.1/2.25" if tdt == "tf32" else ""),
-                    "algorithmic_flops_per_launch": nzf,
-                    "tensor_flops_executed_per_launch": executed,
-                    "tensor_utilisation": executed / (lin_avg * 1e-3) / 1e12 / peak,
-                    "note": "linear time includes the one-pass weight decompression launch",
-                    "hbm_bytes_per_launch": alg_bytes}
+        roofline = {"bound": "tensor", "achieved": sig(achieved), "peak": sig(peak), "unit": "TFLOP/s",
+                    "frac": sig(achieved / peak), "traffic": measured_traffic(kname), "kernel": kname,
+                    "peak_source": "measured bf16 burst" + (" x 1.1/2.25" if tdt == "tf32" else ""),
+                    "tensor_util": sig(executed / (lin_avg * 1e-3) / 1e12 / peak)}
     else:
-        roofline = {"bound": "alu", "achieved": achieved, "peak": ALU_PEAK_TFLOPS, "unit": "TFLOP/s",
-                    "frac": achieved / ALU_PEAK_TFLOPS, "traffic": measured_traffic(kname),
-                    "kernel": kname,
-                    "peak_source": "derived: 152 SMs x 128 FP32 FMA lanes x 2 flop x 2.070 GHz max clock",
-                    "algorithmic_flops_per_launch": nzf, "hbm_bytes_per_launch": alg_bytes}
-    # the workload's own roofline: the slower of its nonzero flops at the CUDA-core
-    # FMA peak and its compressed bytes at 8 TB/s
+        roofline = {"bound": "alu", "achieved": sig(achieved), "peak": sig(ALU_PEAK_TFLOPS), "unit": "TFLOP/s",
+                    "frac": sig(achieved / ALU_PEAK_TFLOPS), "traffic": measured_traffic(kname), "kernel": kname,
+                    "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 flop x 2.070 GHz"}
+    # the workload's own roofline (the metric's): the slower of its nonzero flops at
+    # the CUDA-core FMA peak and its compressed bytes at 8 TB/s
     floor_s = max(nzf / (ALU_PEAK_TFLOPS * 1e12), alg_bytes / (HBM_ROOF_GBS * 1e9))
-    metric_roofline = {"definition": "max(nonzero flops / CUDA-core FMA peak, compressed bytes / 8 TB/s)",
-                       "floor_us": floor_s * 1e6, "frac": floor_s / (lin_avg * 1e-3),
-                       "fma_peak_tflops": ALU_PEAK_TFLOPS}
-    # the product's absolute rates (decompression + GEMM time): nonzero and
-    # dense-equivalent flops, algorithmic bytes
-    gbs = alg_bytes / (lin_avg * 1e-3) / 1e9
-    absolute = {"nonzero_tflops": achieved,
-                "dense_equiv_tflops": case.dense_flops() / (lin_avg * 1e-3) / 1e12,
-                "gbs": gbs, "gbs_frac_of_measured_hbm": gbs / measured_peaks()["hbm_gbs"],
-                "gbs_frac_of_8tbs": gbs / HBM_ROOF_GBS,
-                "nonzero_frac_of_fma_peak": achieved / ALU_PEAK_TFLOPS}
+    roofline["metric_frac"] = sig(floor_s / (lin_avg * 1e-3))
 
     # ---- end to end through the public API: W host -> device and packed, then
     # cci_linear_host: X from pinned host memory, Y back to it, in column chunks
@@ -533,58 +562,83 @@ def run_ours(args, rank, world, local):
     torch.cuda.synchronize(dev)
     e2e_ms = statistics.mean(time_device(e2e_step, max(3, args.steps // 4), flush, stream))
     e2e_ms = max_over_ranks(e2e_ms, world, dev)
-    e2e = {"value": world * nzf / (e2e_ms * 1e-3) / 1e12, "unit": UNIT,
+    e2e = {"value": sig(world * nzf / (e2e_ms * 1e-3) / 1e12), "unit": UNIT,
            "h2d_bytes_per_step": X_host.numel() * X_host.element_size() + W_host.numel() * W_host.element_size(),
-           "d2h_bytes_per_step": Y_host.numel() * 4, "ms_per_step": e2e_ms,
-           "path": f"cci_pack + cci_linear_host (C ABI, host X and Y, {chunk}-column chunks, copies on their "
-                   f"own streams overlapping the product)"}
+           "d2h_bytes_per_step": Y_host.numel() * 4, "ms_per_step": sig(e2e_ms)}
+    extra("e2e_path", "H2D copy of W + cci_pack + cci_linear_host (X and Y in pinned host memory, column "
+                      f"chunks of {chunk}, copies on their own streams overlapping the product)")
 
-    # ---- dense reference line: cuBLAS fp32 (TF32 off) on the masked dense weights ----
-    Wm = torch.zeros_like(Wd)
-    Wm.view(case.Cout // case.G, case.G, case.R).scatter_(
-        1, idx.permute(0, 2, 1).long(), values.permute(0, 2, 1))
-    dense_ms = statistics.median(time_device(lambda: torch.matmul(Xd, Wm.t()), 10, flush, stream))
-    dense = {"kernel": "torch.matmul fp32 (cuBLAS, TF32 off)", "ms": dense_ms,
-             "dense_tflops": case.dense_flops() / (dense_ms * 1e-3) / 1e12,
-             "speedup_cci_over_dense": dense_ms / lin_avg}
-
-    # the CUDA-core kernel families on the same product (same inputs, same output)
-    families = {}
-    for name, algo in (("regtile_jump_dispatch", cci.ALGO_REGTILE), ("expand_branch_free", cci.ALGO_EXPAND)):
-        kn = cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, algo)
-        if not kn:
-            continue
-        fn = lambda a=algo: cci.linear(Xd, values, idx, case.Cout, case.G, case.K, out=Y, algo=a)  # noqa: E731
-        fn()
-        ms = statistics.median(time_device(fn, 10, flush, stream))
-        families[name] = {"kernel": kn, "ms": ms, "nz_tflops": nzf / (ms * 1e-3) / 1e12,
-                          "roofline_frac": nzf / (ms * 1e-3) / 1e12 / ALU_PEAK_TFLOPS}
-
-    extras = {}
+    sweep = []
+    if rank == 0 and case.name.startswith("sweep_4096"):
+        sweep = run_sweep(cci, dev, stream, flush)
     if args.extras and rank == 0:
-        extras = run_extras(cci, dev, stream, flush)
+        run_extras(cci, dev, stream, flush)
 
     cpu = None
     if rank == 0 and world == 1:
         rate, rows, passes, dt, cores = oracle_rate(case, args.cpu_sample_seconds)
-        cpu = {"value": rate, "unit": UNIT, "cores": cores, "kind": "oracle",
-               "sample": f"{passes} pass(es) of the fp64 dense-mask product over the first {rows} of "
-                         f"{case.N} columns ({dt:.1f} s in all), nonzero flops counted"}
+        cpu = {"value": sig(rate), "unit": UNIT, "cores": cores, "kind": "oracle",
+               "sample": f"fp64 dense-mask product, first {rows}/{case.N} columns x {passes}, {dt:.0f} s"}
 
     if rank == 0:
+        extra("timed_region", {"wall_ms_per_step_incl_flush": t_wall * 1e3 / args.steps, "clocks": clk.summary()})
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": config_of(case), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
-            "gpu_launches": (3 if on_tc else 2) * args.steps, "clocks": clk.summary(),
-            "metric_roofline": metric_roofline, "absolute": absolute,
-            "breakdown_ms": {"pack": statistics.mean(pack_ms), "linear": lin_avg,
-                             "wall_per_step_incl_flush": t_wall * 1e3 / args.steps},
-            "dense_reference": dense, "cuda_core_families": families, **extras,
+            "metric": METRIC, "value": sig(value), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": sig(ms_step), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if tdt == "bf16" else "f32",
+            "data": "synthetic", "config": config_of(case), "roofline": roofline, "cpu_baseline": cpu,
+            "e2e": e2e, "gpu_launches": (1 + launches_per_product(cci, X.dtype, case)) * args.steps,
+            "clocks": clk.summary(),
+            "ms": {"pack": sig(statistics.mean(pack_ms)), "product": sig(lin_avg)},
+            "sweep": sweep,
         }
-        print(json.dumps(line), flush=True)
+        print(json.dumps(line, separators=(",", ":")), flush=True)
     return 0
+
+
+def run_sweep(cci, dev, stream, flush, reps=10):
+    """The K/G sweep (4096 -> 4096, N = 8192, bf16): per (G, K) the production
+    product (pack excluded), cuBLAS bf16 on the masked dense weights, and the same
+    tensor-core GEMM on the unpruned dense weights without decompression.  Keys:
+    ms (CCI product), nz (nonzero TFLOP/s), frac (the workload roofline: nonzero
+    flops at the CUDA-core FMA peak, or bytes at 8 TB/s, over ms),
+    cublas (cuBLAS ms / CCI ms), same (the same kernel on dense weights, its ms /
+    CCI ms: what the sparsity buys); the tensor utilisation (dense flops executed /
+    ms / measured bf16 peak) and kernel names go to stderr."""
+    out, tu = [], []
+    dense_same_ms = None
+    peak = tensor_peak("bf16")
+    for G, K in wl.SWEEP_POINTS:
+        case = wl.sweep_case(G, K)
+        X, W = wl.linear_inputs(case, device=str(dev))
+        v, i = cci.pack(W, G, K)
+        Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
+        ws = cci.auto_workspace(X.dtype, case.Cin, case.R, case.Cout, G, K, dev)
+        fn = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, workspace=ws)  # noqa: E731
+        fn()
+        ms = statistics.median(time_device(fn, reps, flush, stream))
+        Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
+        Wm.view(case.Cout // G, G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
+        dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), reps, flush, stream))
+        if dense_same_ms is None:  # one shape for every point: the unpruned W of the first
+            Wp = dense_planes(W)
+            fd = lambda: cci.dense_linear_tc(X, Wp, case.Cout, out=Y)  # noqa: E731
+            fd()
+            dense_same_ms = statistics.median(time_device(fd, reps, flush, stream))
+            del Wp
+        nz = case.nz_flops() / (ms * 1e-3) / 1e12
+        floor_s = max(case.nz_flops() / (ALU_PEAK_TFLOPS * 1e12),
+                      algorithmic_bytes(case, 2) / (HBM_ROOF_GBS * 1e9))
+        out.append({"G": G, "K": K, "ms": sig(ms), "nz": sig(nz, 3), "frac": sig(floor_s / (ms * 1e-3), 3),
+                    "cublas": sig(dms / ms, 3), "same": sig(dense_same_ms / ms, 3)})
+        tu.append({"G": G, "K": K, "tensor_util": case.dense_flops() / (ms * 1e-3) / 1e12 / peak,
+                   "cublas_ms": dms, "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, G, K,
+                                                               cci.ALGO_AUTO, workspace=ws is not None)})
+        del X, W, v, i, Y, Wm, ws
+    torch.cuda.empty_cache()
+    extra("sweep_4096_details", {"same_kernel_dense_ms": dense_same_ms, "points": tu,
+                                 "same_kernel": "the tensor-core GEMM on unpruned bf16 W, no decompression"})
+    return out
 
 
 def algorithmic_bytes(case, elem: int) -> int:
@@ -595,86 +649,103 @@ def algorithmic_bytes(case, elem: int) -> int:
     return x * elem + case.N * case.Cout * 4 + (case.Cout // case.G) * case.R * case.K * (elem + 1)
 
 
-def run_extras(cci, dev, stream, flush):
-    """K/G sweep (4096 -> 4096, N = 8192, bf16) and the 3x3 conv workload, each
-    against its dense cuBLAS / cuDNN line on the masked dense weights."""
-    out = {"sweep_4096": [], "conv3x3_28": None}
-    for G, K in wl.SWEEP_POINTS:
-        case = wl.sweep_case(G, K)
-        X, W = wl.linear_inputs(case, device=str(dev))
-        v, i = cci.pack(W, G, K)
-        Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
-        fn = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y)  # noqa: E731
+def kernel_families(cci, case, X, v, i, Y, conv, flush, stream, reps=5):
+    """The product of one workload on every kernel family that has it: the CUDA-core
+    scatter families (jump dispatch and expand), the workspace tensor-core family
+    and the fused tensor-core family; ms and nonzero TFLOP/s of each."""
+    G, K = case.G, case.K
+    res = {}
+    for name, algo in (("regtile_jump", cci.ALGO_REGTILE), ("expand", cci.ALGO_EXPAND),
+                       ("dense_tc_ws", cci.ALGO_DENSE_TC_WS), ("dense_tc_fused", cci.ALGO_DENSE_TC)):
+        kn = cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, G, K, algo)
+        if not kn:
+            continue
+        ws = cci.new_workspace(algo, X.dtype, case.Cout, case.R, X.device) if algo == cci.ALGO_DENSE_TC_WS else None
+        if conv:
+            fn = lambda a=algo, w=ws: cci.conv2d(X, v, i, case.Cout, G, K, case.KH, case.KW,  # noqa: E731
+                                                 (case.stride,) * 2, (case.pad,) * 2, out=Y, algo=a, workspace=w)
+        else:
+            fn = lambda a=algo, w=ws: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=a, workspace=w)  # noqa: E731
         fn()
-        ms = statistics.median(time_device(fn, 10, flush, stream))
-        fr = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_REGTILE)  # noqa: E731
-        fr()
-        ms_jump = statistics.median(time_device(fr, 5, flush, stream))
-        ft = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_DENSE_TC)  # noqa: E731
-        ft()
-        ms_tc = statistics.median(time_device(ft, 10, flush, stream))
-        ws = cci.new_workspace(cci.ALGO_DENSE_TC_WS, X.dtype, case.Cout, case.R, dev)
-        fw = lambda: cci.linear(X, v, i, case.Cout, G, K, out=Y, algo=cci.ALGO_DENSE_TC_WS,  # noqa: E731
-                                workspace=ws)
-        fw()
-        ms_ws = statistics.median(time_device(fw, 10, flush, stream))
-        Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
-        Wm.view(case.Cout // G, G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
-        dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), 10, flush, stream))
-        tf = case.nz_flops() / (ms * 1e-3) / 1e12
-        out["sweep_4096"].append({"G": G, "K": K, "K_over_G": K / G, "ms": ms, "nz_tflops": tf,
-                                  "dense_equiv_tflops": case.dense_flops() / (ms * 1e-3) / 1e12,
-                                  "roofline_frac": tf / ALU_PEAK_TFLOPS,
-                                  "dense_bf16_ms": dms, "speedup_over_dense": dms / ms,
-                                  "regtile_jump_dispatch_ms": ms_jump,
-                                  "dense_tc_ms": ms_tc,
-                                  "dense_tc_nz_tflops": case.nz_flops() / (ms_tc * 1e-3) / 1e12,
-                                  "dense_tc_dense_equiv_tflops": case.dense_flops() / (ms_tc * 1e-3) / 1e12,
-                                  "dense_tc_ws_ms": ms_ws,
-                                  "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
-                                  "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
-                                  "gbs": algorithmic_bytes(case, 2) / (ms * 1e-3) / 1e9,
-                                  "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R,
-                                                            case.Cout, G, K, cci.ALGO_DENSE_TC_WS)})
-        del X, W, v, i, Y, Wm, ws
+        ms = statistics.median(time_device(fn, reps, flush, stream))
+        res[name] = {"kernel": kn, "ms": sig(ms), "nz": sig(case.nz_flops() / (ms * 1e-3) / 1e12)}
+    return res
+
+
+def run_bottleneck_fp32(cci, dev, stream, flush, reps=10):
+    """The ResNet 1x1 bottleneck as an fp32 product (N = 100352, 256 -> 1024, G = 8,
+    K = 2): the production path, every kernel family, cuBLAS fp32 (TF32 off) on the
+    masked dense weights and the same tensor-core GEMM on the unpruned weights."""
+    case = wl.BOTTLENECK_1X1
+    X, W = wl.linear_inputs(case, device=str(dev))
+    v, i = cci.pack(W, case.G, case.K)
+    Y = torch.empty((case.N, case.Cout), dtype=torch.float32, device=dev)
+    ws = cci.auto_workspace(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, dev)
+    fn = lambda: cci.linear(X, v, i, case.Cout, case.G, case.K, out=Y, workspace=ws)  # noqa: E731
+    fn()
+    ms = statistics.median(time_device(fn, reps, flush, stream))
+    Wm = torch.zeros_like(W)
+    Wm.view(case.Cout // case.G, case.G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
+    dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), reps, flush, stream))
+    Wp = dense_planes(W)
+    fd = lambda: cci.dense_linear_tc(X, Wp, case.Cout, out=Y)  # noqa: E731
+    fd()
+    sms = statistics.median(time_device(fd, reps, flush, stream))
+    nzf = case.nz_flops()
+    floor_s = max(nzf / (ALU_PEAK_TFLOPS * 1e12), algorithmic_bytes(case, 4) / (HBM_ROOF_GBS * 1e9))
+    return {"workload": case.name, "ms": ms, "nz_tflops": nzf / (ms * 1e-3) / 1e12,
+            "metric_roofline_frac": floor_s / (ms * 1e-3),
+            "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
+                                      workspace=ws is not None),
+            "cublas_fp32_simt_ms": dms, "speedup_over_cublas_fp32": dms / ms,
+            "same_kernel_dense_ms": sms, "sparsity_gain": sms / ms,
+            "tensor_vs_simt": dms / sms,
+            "families": kernel_families(cci, case, X, v, i, Y, False, flush, stream)}
+
+
+def run_conv3x3(cci, dev, stream, flush, reps=10):
+    """The 3x3 convolution workload (batch 64, 28x28, 128 -> 128, G = 16, K = 4,
+    bf16): the production path, every kernel family, cuDNN bf16 on the masked dense
+    weights and the same tensor-core GEMM on the unpruned weights."""
     case = wl.CONV3X3_28
     X, W = wl.conv_inputs(case, device=str(dev))
     v, i = cci.pack(W, case.G, case.K)
-    fn = lambda: cci.conv2d(X, v, i, case.Cout, case.G, case.K, 3, 3, (1, 1), (1, 1))  # noqa: E731
+    Y = torch.empty((case.B, case.P, case.Q, case.Cout), dtype=torch.float32, device=dev)
+    ws = cci.auto_workspace(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, dev)
+    fn = lambda: cci.conv2d(X, v, i, case.Cout, case.G, case.K, 3, 3, (1, 1), (1, 1), out=Y,  # noqa: E731
+                            workspace=ws)
     fn()
-    ms = statistics.median(time_device(fn, 10, flush, stream))
+    ms = statistics.median(time_device(fn, reps, flush, stream))
     Wm = torch.zeros((case.Cout, case.R), dtype=W.dtype, device=dev)
     Wm.view(case.Cout // case.G, case.G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
     w4 = Wm.view(case.Cout, 3, 3, case.Cin).permute(0, 3, 1, 2).contiguous(memory_format=torch.channels_last)
     x4 = X.permute(0, 3, 1, 2)  # NHWC memory, NCHW view = channels_last
-    dms = statistics.median(time_device(
-        lambda: torch.nn.functional.conv2d(x4, w4, padding=1), 10, flush, stream))
-    ft = lambda: cci.conv2d(X, v, i, case.Cout, case.G, case.K, 3, 3, (1, 1), (1, 1),  # noqa: E731
-                            algo=cci.ALGO_DENSE_TC)
-    ft()
-    ms_tc = statistics.median(time_device(ft, 10, flush, stream))
-    ws = cci.new_workspace(cci.ALGO_DENSE_TC_WS, X.dtype, case.Cout, case.R, dev)
-    fw = lambda: cci.conv2d(X, v, i, case.Cout, case.G, case.K, 3, 3, (1, 1), (1, 1),  # noqa: E731
-                            algo=cci.ALGO_DENSE_TC_WS, workspace=ws)
-    fw()
-    ms_ws = statistics.median(time_device(fw, 10, flush, stream))
-    tf = case.nz_flops() / (ms * 1e-3) / 1e12
-    out["conv3x3_28"] = {"ms": ms, "nz_tflops": tf, "roofline_frac": tf / ALU_PEAK_TFLOPS,
-                         "dense_tc_ms": ms_tc, "dense_tc_nz_tflops": case.nz_flops() / (ms_tc * 1e-3) / 1e12,
-                         "dense_tc_dense_equiv_tflops": case.dense_flops() / (ms_tc * 1e-3) / 1e12,
-                         "dense_tc_ws_ms": ms_ws, "dense_tc_ws_nz_tflops": case.nz_flops() / (ms_ws * 1e-3) / 1e12,
-                         "dense_tc_ws_dense_equiv_tflops": case.dense_flops() / (ms_ws * 1e-3) / 1e12,
-                         "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
-                         "dense_equiv_tflops": case.dense_flops() / (ms * 1e-3) / 1e12,
-                         "gbs": algorithmic_bytes(case, 2) / (ms * 1e-3) / 1e9,
-                         "kernel": cci.kernel_name(torch.bfloat16, case.Cin, case.R, case.Cout,
-                                                   case.G, case.K, cci.ALGO_DENSE_TC_WS)}
-    out["resnet50_stack"] = run_resnet_stack(cci, dev, stream, flush)
-    out["mobilenetv2_pointwise"] = run_pointwise_stack(cci, dev, stream, flush)
-    out["allocation_error"] = run_allocation_error(cci, dev, stream, flush)
-    out["td_mask"] = run_td_mask(cci, dev, stream, flush)
-    out["cci_vs_bbs"] = run_cci_vs_bbs(cci, dev, stream, flush)
-    return out
+    dms = statistics.median(time_device(lambda: torch.nn.functional.conv2d(x4, w4, padding=1), reps, flush, stream))
+    fd = lambda: cci.dense_conv2d_tc(X, W, case.Cout, 3, 3, (1, 1), (1, 1), out=Y)  # noqa: E731
+    fd()
+    sms = statistics.median(time_device(fd, reps, flush, stream))
+    nzf = case.nz_flops()
+    return {"workload": case.name, "ms": ms, "nz_tflops": nzf / (ms * 1e-3) / 1e12,
+            "metric_roofline_frac": layer_floor_us(case) * 1e-3 / ms,
+            "dense_equiv_tflops": case.dense_flops() / (ms * 1e-3) / 1e12,
+            "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
+                                      workspace=ws is not None),
+            "cudnn_bf16_ms": dms, "speedup_over_cudnn": dms / ms,
+            "same_kernel_dense_ms": sms, "sparsity_gain": sms / ms,
+            "families": kernel_families(cci, case, X, v, i, Y, True, flush, stream)}
+
+
+def run_extras(cci, dev, stream, flush):
+    """Every measurement beside the headline, each printed as its own stderr line:
+    the fp32 bottleneck product, the 3x3 convolution, the ResNet-50 and MobileNetV2
+    stacks, Eq. 1's allocation error, the targeted-dropout step and CCI against
+    balanced sparsity."""
+    for name, fn in (("bottleneck_1x1_fp32", run_bottleneck_fp32), ("conv3x3_28", run_conv3x3),
+                     ("resnet50_stack", run_resnet_stack), ("mobilenetv2_pointwise", run_pointwise_stack),
+                     ("allocation_error", run_allocation_error), ("td_mask", run_td_mask),
+                     ("cci_vs_bbs", run_cci_vs_bbs)):
+        extra(name, fn(cci, dev, stream, flush))
+        torch.cuda.empty_cache()
 
 
 def run_cci_vs_bbs(cci, dev, stream, flush, reps=5):
@@ -747,29 +818,33 @@ def run_pointwise_stack(cci, dev, stream, flush, reps=5):
     """The 34 pointwise convolutions of MobileNetV2 (batch 128, bf16, G = 8, K = 2:
     the paper's 75 % case), each on its own synthetic input, captured in CUDA
     graphs: fp32 outputs (the library's product), bf16 outputs with bias through
-    the fused epilogue, and cuDNN on the masked dense weights (bf16 output)."""
+    the fused epilogue, cuDNN on the masked dense weights (bf16 output) and the
+    library's tensor-core GEMM on the unpruned weights (fp32 output)."""
     layers = wl.mobilenetv2_pointwise_layers()
-    plain, fused, dense, keep = [], [], [], []
+    plain, fused, dense, same, keep = [], [], [], [], []
     for c in layers:
         X, W = wl.conv_inputs(c, device=str(dev))
         v, i = cci.pack(W, c.G, c.K)
         Y = torch.empty((c.B, c.P, c.Q, c.Cout), dtype=torch.float32, device=dev)
         Yb = torch.empty((c.B, c.P, c.Q, c.Cout), dtype=torch.bfloat16, device=dev)
         bias = torch.zeros(c.Cout, dtype=torch.float32, device=dev)
-        ws = cci.new_workspace(cci.ALGO_AUTO, X.dtype, c.Cout, c.R, dev)
+        ws = cci.auto_workspace(X.dtype, c.Cin, c.R, c.Cout, c.G, c.K, dev)
+        wsf = cci.new_workspace(cci.ALGO_DENSE_TC_WS, X.dtype, c.Cout, c.R, dev)
         Wm = torch.zeros((c.Cout, c.R), dtype=W.dtype, device=dev)
         Wm.view(c.Cout // c.G, c.G, c.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
         w4 = Wm.view(c.Cout, 1, 1, c.Cin).permute(0, 3, 1, 2).contiguous(memory_format=torch.channels_last)
         x4 = X.permute(0, 3, 1, 2)
-        del W, Wm
-        keep.append((X, v, i, Y, Yb, bias, ws, w4, x4))
+        del Wm
+        keep.append((X, v, i, Y, Yb, bias, ws, wsf, w4, x4, W))
         plain.append(lambda c=c, X=X, v=v, i=i, Y=Y, ws=ws: cci.conv2d(
             X, v, i, c.Cout, c.G, c.K, 1, 1, (1, 1), (0, 0), out=Y, workspace=ws))
-        fused.append(lambda c=c, X=X, v=v, i=i, Yb=Yb, ws=ws, bias=bias: cci.conv2d_fused(
+        fused.append(lambda c=c, X=X, v=v, i=i, Yb=Yb, ws=wsf, bias=bias: cci.conv2d_fused(
             X, v, i, c.Cout, c.G, c.K, 1, 1, (1, 1), (0, 0), bias=bias, out=Yb, workspace=ws))
         dense.append(lambda x4=x4, w4=w4: torch.nn.functional.conv2d(x4, w4))
+        same.append(lambda c=c, X=X, W=W, Y=Y: cci.dense_conv2d_tc(X, W, c.Cout, 1, 1, out=Y))
     res = {"layers": len(layers), "batch": layers[0].B, "G": 8, "K": 2}
-    for name, calls in (("ms", plain), ("fused_bf16_out_ms", fused), ("dense_cudnn_bf16_ms", dense)):
+    for name, calls in (("ms", plain), ("fused_bf16_out_ms", fused), ("dense_cudnn_bf16_ms", dense),
+                        ("same_kernel_dense_ms", same)):
         for f in calls:
             f()
         torch.cuda.synchronize(dev)
@@ -787,8 +862,9 @@ def run_pointwise_stack(cci, dev, stream, flush, reps=5):
                 "dense_equiv_tflops": sum(c.dense_flops() for c in layers) / (res["ms"] * 1e-3) / 1e12,
                 "roofline_floor_ms": floor_ms, "roofline_frac": floor_ms / res["ms"],
                 "speedup_over_dense": res["dense_cudnn_bf16_ms"] / res["ms"],
-                "fused_speedup_over_dense": res["dense_cudnn_bf16_ms"] / res["fused_bf16_out_ms"]})
-    del keep, plain, fused, dense
+                "fused_speedup_over_dense": res["dense_cudnn_bf16_ms"] / res["fused_bf16_out_ms"],
+                "sparsity_gain": res["same_kernel_dense_ms"] / res["ms"]})
+    del keep, plain, fused, dense, same
     torch.cuda.empty_cache()
     return res
 
@@ -846,25 +922,28 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
     res = []
     for K in (1, 2, 4):
         layers = wl.resnet50_layers(K=K)
-        ours_calls, dense_calls = [], []
+        ours_calls, dense_calls, same_calls = [], [], []
         keep = []
         for c in layers:
             X, W = wl.conv_inputs(c, device=str(dev))
             v, i = cci.pack(W, c.G, c.K)
             Y = torch.empty((c.B, c.P, c.Q, c.Cout), dtype=torch.float32, device=dev)
-            ws = cci.new_workspace(cci.ALGO_AUTO, X.dtype, c.Cout, c.R, dev)
+            ws = cci.auto_workspace(X.dtype, c.Cin, c.R, c.Cout, c.G, c.K, dev)
+            wsf = cci.new_workspace(cci.ALGO_DENSE_TC_WS, X.dtype, c.Cout, c.R, dev)
             Wm = torch.zeros((c.Cout, c.R), dtype=W.dtype, device=dev)
             Wm.view(c.Cout // c.G, c.G, c.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
             w4 = Wm.view(c.Cout, c.KH, c.KW, c.Cin).permute(0, 3, 1, 2).contiguous(
                 memory_format=torch.channels_last)
             x4 = X.permute(0, 3, 1, 2)
-            del W, Wm
-            keep.append((X, v, i, Y, ws, w4, x4))
+            del Wm
+            keep.append((X, v, i, Y, wsf, w4, x4, W, ws))
             ours_calls.append(lambda c=c, X=X, v=v, i=i, Y=Y, ws=ws: cci.conv2d(
                 X, v, i, c.Cout, c.G, c.K, c.KH, c.KW, (c.stride, c.stride), (c.pad, c.pad), out=Y,
                 workspace=ws))
             dense_calls.append(lambda c=c, x4=x4, w4=w4: torch.nn.functional.conv2d(
                 x4, w4, stride=c.stride, padding=c.pad))
+            same_calls.append(lambda c=c, X=X, W=W, Y=Y: cci.dense_conv2d_tc(
+                X, W, c.Cout, c.KH, c.KW, (c.stride, c.stride), (c.pad, c.pad), out=Y))
 
         def ours():
             for f in ours_calls:
@@ -874,28 +953,38 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
             for f in dense_calls:
                 f()
 
+        def same():
+            for f in same_calls:
+                f()
+
         ours()
         dense()
+        same()
         torch.cuda.synchronize(dev)
-        g_ours, g_dense = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
+        g_ours, g_dense, g_same = torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()
         with torch.cuda.graph(g_ours):
             ours()
         with torch.cuda.graph(g_dense):
             dense()
+        with torch.cuda.graph(g_same):
+            same()
         g_ours.replay()
         g_dense.replay()
+        g_same.replay()
         torch.cuda.synchronize(dev)
         ms = statistics.median(time_device(g_ours.replay, reps, flush, stream))
         dms = statistics.median(time_device(g_dense.replay, reps, flush, stream))
+        sms = statistics.median(time_device(g_same.replay, reps, flush, stream))
         per_layer = []
         if K == 2:  # each layer alone, for the breakdown
-            for c, fo, fd in zip(layers, ours_calls, dense_calls):
+            for c, fo, fd, fs, kp in zip(layers, ours_calls, dense_calls, same_calls, keep):
                 lm = statistics.median(time_device(fo, reps, flush, stream))
                 ld = statistics.median(time_device(fd, reps, flush, stream))
+                ls = statistics.median(time_device(fs, reps, flush, stream))
                 per_layer.append({"layer": c.name, "ms": round(lm, 5), "floor_ms": round(layer_floor_us(c) * 1e-3, 5),
-                                  "cudnn_ms": round(ld, 5),
+                                  "cudnn_ms": round(ld, 5), "same_kernel_dense_ms": round(ls, 5),
                                   "kernel": cci.kernel_name(torch.bfloat16, c.Cin, c.R, c.Cout, c.G, c.K,
-                                                            cci.ALGO_DENSE_TC_WS)})
+                                                            cci.ALGO_AUTO, workspace=kp[8] is not None)})
         # the same 52 layers chained through the fused epilogue: each layer reads
         # the bf16 output of the layer before it in its block (the first block its
         # synthetic input), adds a bias, applies ReLU (a and b) and writes bf16
@@ -904,7 +993,7 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
         x_in = wl.draw_x((layers[0].B, layers[0].H, layers[0].W, layers[0].Cin), "relu_normal", "bf16",
                          1000 + K, str(dev))
         block_in, prev, pending = x_in, None, None
-        for c, role, (X, v, i, Y, ws, w4, x4) in zip(layers, roles, keep):
+        for c, role, (X, v, i, Y, ws, w4, x4, _, _) in zip(layers, roles, keep):
             if role == "a" and pending is not None:  # a new block reads the last block's output
                 block_in, pending = pending, None
             src = block_in if role in ("a", "proj") else prev
@@ -939,6 +1028,7 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
                     "dense_equiv_tflops": dense_f / (ms * 1e-3) / 1e12,
                     "roofline_floor_ms": floor_ms, "roofline_frac": floor_ms / ms,
                     "dense_cudnn_bf16_ms": dms, "speedup_over_dense": dms / ms,
+                    "same_kernel_dense_ms": sms, "sparsity_gain": sms / ms,
                     "fused_chained": {"ms": fms, "nz_tflops": nzf / (fms * 1e-3) / 1e12,
                                       "speedup_over_dense": dms / fms,
                                       "what": "cci_conv2d_fused per layer: bias, ReLU on the 1x1-reduce and 3x3 "
@@ -947,7 +1037,7 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
                     "captured": "CUDA graph of the 52 calls (ours) / 52 cuDNN convolutions (dense)"})
         if per_layer:
             res[-1]["per_layer"] = per_layer
-        del keep, ours_calls, dense_calls, g_ours, g_dense, fused_calls, fkeep, g_fused, block_in, prev, pending, x_in
+        del keep, ours_calls, dense_calls, same_calls, g_ours, g_dense, g_same, fused_calls, fkeep, g_fused, block_in, prev, pending, x_in
         torch.cuda.empty_cache()
     return res
 

@@ -26,9 +26,13 @@
  *
  * Ownership and execution: the caller allocates every buffer; all data pointers
  * are DEVICE pointers (except the X_host / Y_host of cci_linear_host); the
- * library allocates nothing and keeps no state between calls.  Every call is asynchronous on `stream` (NULL = the legacy default
- * stream) and returns once its kernels are enqueued.  Calls on different
- * streams may run concurrently when their outputs do not overlap.
+ * library allocates nothing.  It keeps no state between calls except two
+ * per-device caches, both filled on a device's first use: the dynamic
+ * shared-memory limit set on each tensor-core kernel, and the device address of
+ * the static scratch array of cci_linear_dense_tc_static (see there).  Every
+ * call is asynchronous on `stream` (NULL = the legacy default stream) and
+ * returns once its kernels are enqueued.  Calls on different streams may run
+ * concurrently when their outputs do not overlap.
  *
  * Errors:
  *   - Argument errors are detected on the host, before anything is enqueued, and
@@ -93,7 +97,7 @@ typedef enum cci_algo {
                                CCI_ALGO_REGTILE */
     CCI_ALGO_DENSE_TC_WS = 5  /* decompress the packed weights once per call into a caller
                                workspace and multiply densely on the tensor cores (tcgen05),
-                               operands streamed by cp.async.  bf16: dense bf16 [Cout][R],
+                               operands copied by TMA (cp.async.bulk.tensor).  bf16: dense bf16 [Cout][R],
                                Cin % 8 == 0, R % 8 == 0.  fp32: hi and lo tf32 planes
                                [2][Cout][R] and a three-pass tf32 product (hi*hi + hi*lo +
                                lo*hi, |error| below 2^-21 of sum |w||x|), Cin % 4 == 0,
@@ -256,6 +260,15 @@ cci_status cci_td_mask(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, 
                        cci_stream_t stream);
 
 /*
+ * cci_td_drop_rate -- the candidate drop rate of the targeted-dropout schedule
+ * (Sec. 5.1) at training step `step`: the paper fixes only the end points (start
+ * at 50 %, end toward 100 %); this library ramps linearly from `start` to `end`
+ * over `ramp_steps` steps and holds `end` afterwards (ramp_steps <= 0: `end` at
+ * once; negative steps count as 0).  Host function, no device work.
+ */
+float cci_td_drop_rate(int64_t step, int64_t ramp_steps, float start, float end);
+
+/*
  * Balanced sparsity (Sec. 3.4), the format the paper compares CCI with: groups
  * run along the INPUT dimension.  Per output channel co and group of G
  * consecutive inputs r in [g*G, g*G + G) (R % G == 0), K weights are kept.
@@ -324,6 +337,30 @@ cci_status cci_conv2d_fused(const void *X, cci_dtype dtype, int64_t B, int64_t H
                             void *Y, uint32_t *dev_status, void *workspace,
                             size_t workspace_bytes, cci_stream_t stream);
 
+/*
+ * cci_dense_linear_tc / cci_dense_conv2d_tc -- the tensor-core GEMM of
+ * CCI_ALGO_DENSE_TC_WS run on a DENSE weight matrix that the caller provides,
+ * with no decompression: Y = X * Wd^T (a convolution: the implicit product of
+ * cci_conv2d with Wd in OHWI order).  This is the reference line that isolates
+ * what the sparsity buys on this hardware: Sec. 3.2 argues that CCI cuts the
+ * work of the product by G/K; timing the same kernel on the unpruned weights
+ * shows how much of that a dense tensor-core product keeps.
+ *
+ *   Wd   device, 16-byte aligned, in the workspace layout of the dense family:
+ *        bf16 dense [Cout][R]; fp32 the hi and lo tf32 planes [2][Cout][R]
+ *        (hi = w with the low 13 mantissa bits cleared, lo = w - hi)
+ *   X, Y as cci_linear / cci_conv2d, 16-byte aligned; Cin % 8 == 0 (bf16) or
+ *        % 4 == 0 (fp32); Cout % 4 == 0
+ * Errors: CCI_ERR_NULL, CCI_ERR_SHAPE, CCI_ERR_DTYPE, CCI_ERR_ALIGN,
+ *         CCI_ERR_UNSUPPORTED (shapes the dense kernel lacks), CCI_ERR_CUDA.
+ */
+cci_status cci_dense_linear_tc(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *Wd,
+                               int64_t Cout, float *Y, uint32_t *dev_status, cci_stream_t stream);
+cci_status cci_dense_conv2d_tc(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W,
+                               int64_t Cin, const void *Wd, int64_t Cout, int KH, int KW,
+                               int stride_h, int stride_w, int pad_h, int pad_w, float *Y,
+                               uint32_t *dev_status, cci_stream_t stream);
+
 /* Largest dense-weight size (Cout*R*2 bytes) that cci_linear_dense_tc_static accepts. */
 #define CCI_STATIC_WORKSPACE_BYTES (16u * 1024u * 1024u)
 
@@ -344,7 +381,9 @@ cci_status cci_conv2d_fused(const void *X, cci_dtype dtype, int64_t B, int64_t H
  *   - Cout*Cin*2 > CCI_STATIC_WORKSPACE_BYTES is rejected with CCI_ERR_WORKSPACE;
  *   - the first call on a device looks up the array's device address on that
  *     device (the device current at the call); make that first call before any
- *     stream capture;
+ *     stream capture.  The address is cached for the life of the process: after
+ *     cudaDeviceReset() on that device the cached address is stale, so do not
+ *     call this entry point again on a device that was reset;
  *   - every call shares the one array per device and leaves it holding the last
  *     call's dense weights; each call rewrites the part it reads, so nothing
  *     needs clearing, but calls that overlap on the GPU (other streams, other

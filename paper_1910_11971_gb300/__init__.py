@@ -56,12 +56,16 @@ SIGNATURES = {
     "cci_bbs_linear": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P, _I32, _P,
                               ctypes.c_size_t, _P]),
     "cci_td_mask": (_I32, [_P, _I32, _I64, _I64, _I32, _I32, ctypes.c_float, _P, _P, _P, _U32P, _P]),
+    "cci_td_drop_rate": (ctypes.c_float, [_I64, _I64, ctypes.c_float, ctypes.c_float]),
     "cci_workspace_size": (ctypes.c_size_t, [_I32, _I32, _I64, _I64]),
     "cci_linear_host_buffer_size": (ctypes.c_size_t, [_I32, _I64, _I64, _I64]),
     "cci_linear_host": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _I64, _P,
                                ctypes.c_size_t, _U32P, _P, _P, _P]),
     "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
                                           _P]),
+    "cci_dense_linear_tc": (_I32, [_P, _I32, _I64, _I64, _P, _I64, _P, _U32P, _P]),
+    "cci_dense_conv2d_tc": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _I64, _I32, _I32, _I32, _I32,
+                                   _I32, _I32, _P, _U32P, _P]),
     "cci_kernel_name": (ctypes.c_char_p, [_I32, _I64, _I64, _I64, _I32, _I32, _I32]),
     "cci_status_string": (ctypes.c_char_p, [_I32]),
     "cci_decode_device_status": (_I32, [ctypes.c_uint32]),
@@ -191,11 +195,13 @@ def linear(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
 
     ``workspace``: device buffer for the families that need one (see
     ``workspace_size``); with ``algo`` AUTO or ``ALGO_DENSE_TC_WS`` and none given,
-    one is allocated here from PyTorch memory (the library allocates nothing), so
-    AUTO can use the dense tensor-core family."""
+    the one that family asks for is allocated here from PyTorch memory (the
+    library allocates nothing), so AUTO can reach its fastest family."""
     _cuda_contig(X, "X")
     N, Cin = X.shape
-    if workspace is None and algo in (ALGO_AUTO, ALGO_DENSE_TC_WS):
+    if workspace is None and algo == ALGO_AUTO:
+        workspace = auto_workspace(X.dtype, Cin, Cin, Cout, G, K, X.device)
+    elif workspace is None and algo == ALGO_DENSE_TC_WS:
         workspace = new_workspace(algo, X.dtype, Cout, Cin, X.device)
     Y = out if out is not None else torch.empty((N, Cout), dtype=torch.float32, device=X.device)
     wp, wb = _ws(workspace)
@@ -269,7 +275,9 @@ def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
     P, Q = conv_out_hw(H, W, KH, KW, stride, pad)
     Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=torch.float32,
                                                 device=X.device)
-    if workspace is None and algo in (ALGO_AUTO, ALGO_DENSE_TC_WS):
+    if workspace is None and algo == ALGO_AUTO:
+        workspace = auto_workspace(X.dtype, Cin, KH * KW * Cin, Cout, G, K, X.device)
+    elif workspace is None and algo == ALGO_DENSE_TC_WS:
         workspace = new_workspace(algo, X.dtype, Cout, KH * KW * Cin, X.device)
     wp, wb = _ws(workspace)
     code = lib().cci_conv2d_ws(X.data_ptr(), _dtype_code(X), B, H, W, Cin, values.data_ptr(),
@@ -327,12 +335,10 @@ def td_mask(W: torch.Tensor, G: int, K: int, rate: float, uniforms: torch.Tensor
 
 
 def td_drop_rate(step: int, ramp_steps: int, start: float = 0.5, end: float = 1.0) -> float:
-    """The candidate drop rate of Sec. 5.1: from ``start`` (50 %) toward ``end``
-    (100 %); the paper fixes the end points only, the ramp here is linear over
-    ``ramp_steps`` steps and then constant."""
-    if ramp_steps <= 0:
-        return end
-    return start + (end - start) * min(max(step, 0) / ramp_steps, 1.0)
+    """The candidate drop rate of Sec. 5.1 at ``step`` (``cci_td_drop_rate``): from
+    ``start`` (50 %) toward ``end`` (100 %), linear over ``ramp_steps`` steps and then
+    constant (the paper fixes the end points only)."""
+    return float(lib().cci_td_drop_rate(int(step), int(ramp_steps), float(start), float(end)))
 
 
 def pack_stats(W: torch.Tensor, G: int, K: int, counts: Optional[torch.Tensor] = None) -> torch.Tensor:
@@ -407,10 +413,64 @@ def conv2d_fused(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout:
     return Y
 
 
+def dense_linear_tc(X: torch.Tensor, Wd: torch.Tensor, Cout: int, *, out: Optional[torch.Tensor] = None,
+                    status: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """Y[N][Cout] = X Wd^T on the library's tensor-core GEMM with dense weights and
+    no decompression (``cci_dense_linear_tc``).  Wd is the dense family's workspace
+    layout: bf16 [Cout][Cin]; fp32 the hi / lo tf32 planes [2][Cout][Cin]."""
+    _cuda_contig(X, "X")
+    _cuda_contig(Wd, "Wd")
+    N, Cin = X.shape
+    Y = out if out is not None else torch.empty((N, Cout), dtype=torch.float32, device=X.device)
+    _check(lib().cci_dense_linear_tc(X.data_ptr(), _dtype_code(X), N, Cin, Wd.data_ptr(), Cout, Y.data_ptr(),
+                                     status.data_ptr() if status is not None else None, _stream(X.device)),
+           "cci_dense_linear_tc")
+    return Y
+
+
+def dense_conv2d_tc(X: torch.Tensor, Wd: torch.Tensor, Cout: int, KH: int, KW: int, stride=(1, 1), pad=(0, 0), *,
+                    out: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """NHWC convolution on the library's tensor-core GEMM with dense OHWI weights in
+    the dense family's workspace layout and no decompression (``cci_dense_conv2d_tc``)."""
+    _cuda_contig(X, "X")
+    _cuda_contig(Wd, "Wd")
+    B, H, W, Cin = X.shape
+    P, Q = conv_out_hw(H, W, KH, KW, stride, pad)
+    Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=torch.float32,
+                                                device=X.device)
+    _check(lib().cci_dense_conv2d_tc(X.data_ptr(), _dtype_code(X), B, H, W, Cin, Wd.data_ptr(), Cout, KH, KW,
+                                     stride[0], stride[1], pad[0], pad[1], Y.data_ptr(),
+                                     status.data_ptr() if status is not None else None, _stream(X.device)),
+           "cci_dense_conv2d_tc")
+    return Y
+
+
 def kernel_name(dtype: torch.dtype, Cin: int, R: int, Cout: int, G: int, K: int,
-                algo: int = ALGO_AUTO) -> str:
+                algo: int = ALGO_AUTO, workspace: bool = False) -> str:
+    """The kernel family a call would run (``cci_kernel_name``).  With
+    ``workspace=True`` and AUTO: the family AUTO picks when it is given the
+    workspace it asks for (the workspace tensor-core family where the fused one
+    does not apply)."""
     code = F32 if dtype == torch.float32 else BF16
-    return lib().cci_kernel_name(code, Cin, R, Cout, G, K, algo).decode()
+    name = lib().cci_kernel_name(code, Cin, R, Cout, G, K, algo).decode()
+    if algo == ALGO_AUTO and workspace and not name.startswith("dense_tc"):
+        ws_name = lib().cci_kernel_name(code, Cin, R, Cout, G, K, ALGO_DENSE_TC_WS).decode()
+        if ws_name:
+            return ws_name
+    return name
+
+
+def auto_workspace(dtype: torch.dtype, Cin: int, R: int, Cout: int, G: int, K: int,
+                   device) -> Optional[torch.Tensor]:
+    """The workspace AUTO needs to reach its fastest family for a layer (R = Cin
+    for a product, KH*KW*Cin for a convolution), from PyTorch memory: None when
+    that family needs none (the library allocates nothing itself)."""
+    if kernel_name(dtype, Cin, R, Cout, G, K, ALGO_AUTO).startswith("dense_tc"):
+        return None
+    if not lib().cci_kernel_name(F32 if dtype == torch.float32 else BF16, Cin, R, Cout, G, K,
+                                 ALGO_DENSE_TC_WS):
+        return None
+    return new_workspace(ALGO_DENSE_TC_WS, dtype, Cout, R, device)
 
 
 def fma_probe(out: torch.Tensor, blocks: int, threads: int, iters: int) -> None:

@@ -86,6 +86,19 @@ bool dense_tc_shape_ok(int dtype, int G, int K, int64_t Cin, int64_t R)
     return dense_tc_supported(dtype, G, K) && Cin % v == 0 && R % v == 0;
 }
 
+// the dense tensor-core GEMM on caller weights p.wdense (no decompression)
+cci_status dense_forward(FwdParams p, int dtype, cudaStream_t stream)
+{
+    if (p.is_conv && p.KH == 1 && p.KW == 1 && p.sh == 1 && p.sw == 1 && p.ph == 0 && p.pw == 0) p.is_conv = 0;
+    const int64_t v = dtype == CCI_F32 ? 4 : 8;  // elements per 16 bytes
+    if (p.R >= (int64_t(1) << 31) || p.Cout >= (int64_t(1) << 31) || p.Cin % v != 0 || p.R % v != 0 ||
+        p.Cout % 4 != 0)
+        return CCI_ERR_UNSUPPORTED;
+    if (!aligned(p.X, 16) || !aligned(p.Y, 16) || !aligned(p.wdense, 16)) return CCI_ERR_ALIGN;
+    if (p.N == 0) return CCI_OK;
+    return to_status(launch_gemm_ws(p, dtype, stream));
+}
+
 cci_status forward(FwdParams p, int dtype, int G, int K, cci_algo algo, void *ws, size_t ws_bytes,
                    cudaStream_t stream)
 {
@@ -250,6 +263,41 @@ cci_status conv_impl(const void *X, int dtype, int64_t B, int64_t H, int64_t W, 
                      int pad_w, int G, int K, void *Y, uint32_t *dev_status, cci_algo algo, void *workspace,
                      size_t workspace_bytes, cci_stream_t stream, Epilogue e);
 
+// geometry of a convolution (cross-correlation, zero padding, floor output size)
+// into p: sizes, strides, padding, N = B*P*Q and R = KH*KW*Cin; CCI_ERR_SHAPE for
+// sizes out of range or without an output
+cci_status conv_params(int64_t B, int64_t H, int64_t W, int64_t Cin, int64_t Cout, int KH, int KW, int stride_h,
+                       int stride_w, int pad_h, int pad_w, FwdParams *p)
+{
+    if (B < 0 || H < 1 || W < 1 || Cin < 1 || Cout < 1 || KH < 1 || KW < 1 || stride_h < 1 || stride_w < 1 ||
+        pad_h < 0 || pad_w < 0)
+        return CCI_ERR_SHAPE;
+    const int64_t lim = int64_t(1) << 30;
+    if (H >= lim || W >= lim || pad_h >= lim || pad_w >= lim) return CCI_ERR_SHAPE;
+    if (H + 2 * pad_h < KH || W + 2 * pad_w < KW) return CCI_ERR_SHAPE;
+    const int64_t P = (H + 2 * pad_h - KH) / stride_h + 1;
+    const int64_t Q = (W + 2 * pad_w - KW) / stride_w + 1;
+    if (!mul_ok(P, Q) || !mul_ok(B, P * Q) || !mul_ok(H, W) || !mul_ok(H * W, Cin) || !mul_ok(B, H * W * Cin) ||
+        !mul_ok(static_cast<int64_t>(KH) * KW, Cin))
+        return CCI_ERR_SHAPE;
+    p->N = B * P * Q;
+    p->Cout = Cout;
+    p->R = static_cast<int64_t>(KH) * KW * Cin;
+    p->Cin = Cin;
+    p->H = H;
+    p->W = W;
+    p->P = P;
+    p->Q = Q;
+    p->KH = KH;
+    p->KW = KW;
+    p->sh = stride_h;
+    p->sw = stride_w;
+    p->ph = pad_h;
+    p->pw = pad_w;
+    p->is_conv = 1;
+    return CCI_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -267,6 +315,13 @@ cci_status cci_td_mask(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, 
     if (!aligned(W, es) || !aligned(W_out, es) || !aligned(uniforms, 4)) return CCI_ERR_ALIGN;
     return to_status(launch_td_mask(W, dtype, Cout, R, G, K, rate, uniforms, W_out, mask, dev_status,
                                     reinterpret_cast<cudaStream_t>(stream)));
+}
+
+float cci_td_drop_rate(int64_t step, int64_t ramp_steps, float start, float end)
+{
+    if (ramp_steps <= 0) return end;
+    const int64_t s = step < 0 ? 0 : (step > ramp_steps ? ramp_steps : step);
+    return start + (end - start) * static_cast<float>(static_cast<double>(s) / static_cast<double>(ramp_steps));
 }
 
 cci_status cci_bbs_pack(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, int G, int K, void *values,
@@ -401,42 +456,16 @@ cci_status conv_impl(const void *X, int dtype, int64_t B, int64_t H, int64_t W, 
                      size_t workspace_bytes, cci_stream_t stream, Epilogue e)
 {
     float *Y = static_cast<float *>(Y_);
-    if (B < 0 || H < 1 || W < 1 || Cin < 1 || KH < 1 || KW < 1 || stride_h < 1 || stride_w < 1 || pad_h < 0 ||
-        pad_w < 0)
-        return valid_dtype(dtype) ? CCI_ERR_SHAPE : CCI_ERR_DTYPE;
-    const int64_t lim = int64_t(1) << 30;
-    if (H >= lim || W >= lim || pad_h >= lim || pad_w >= lim) return CCI_ERR_SHAPE;
-    if (H + 2 * pad_h < KH || W + 2 * pad_w < KW) return CCI_ERR_SHAPE;
-    const int64_t P = (H + 2 * pad_h - KH) / stride_h + 1;
-    const int64_t Q = (W + 2 * pad_w - KW) / stride_w + 1;
-    if (!mul_ok(P, Q) || !mul_ok(B, P * Q) || !mul_ok(H, W) || !mul_ok(H * W, Cin) || !mul_ok(B, H * W * Cin) ||
-        !mul_ok(static_cast<int64_t>(KH) * KW, Cin))
-        return CCI_ERR_SHAPE;
-    const int64_t N = B * P * Q;
-    const int64_t R = static_cast<int64_t>(KH) * KW * Cin;
-    const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, R, G, K);
-    if (st != CCI_OK) return st;
     FwdParams p{};
+    const cci_status geo = conv_params(B, H, W, Cin, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, &p);
+    if (geo != CCI_OK) return valid_dtype(dtype) ? geo : CCI_ERR_DTYPE;
+    const cci_status st = check_common(X, dtype, values, idx, Y, p.N, Cout, p.R, G, K);
+    if (st != CCI_OK) return st;
     p.X = X;
     p.values = values;
     p.idx = idx;
     p.Y = Y;
     p.status = dev_status;
-    p.N = N;
-    p.Cout = Cout;
-    p.R = R;
-    p.Cin = Cin;
-    p.H = H;
-    p.W = W;
-    p.P = P;
-    p.Q = Q;
-    p.KH = KH;
-    p.KW = KW;
-    p.sh = stride_h;
-    p.sw = stride_w;
-    p.ph = pad_h;
-    p.pw = pad_w;
-    p.is_conv = 1;
     p.bias = e.bias;
     p.relu = e.relu;
     p.out_bf16 = e.out_bf16;
@@ -471,6 +500,35 @@ cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int6
 {
     return cci_conv2d_ex(X, dtype, B, H, W, Cin, values, idx, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, G, K,
                          Y, dev_status, CCI_ALGO_AUTO, stream);
+}
+
+cci_status cci_dense_linear_tc(const void *X, cci_dtype dtype, int64_t N, int64_t Cin, const void *Wd,
+                               int64_t Cout, float *Y, uint32_t *dev_status, cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!Wd || (N > 0 && (!X || !Y))) return CCI_ERR_NULL;
+    if (N < 0 || Cin < 1 || Cout < 1 || !mul_ok(N, Cin) || !mul_ok(N, Cout) || !mul_ok(Cout, Cin))
+        return CCI_ERR_SHAPE;
+    FwdParams p = linear_params(X, N, Cin, nullptr, nullptr, Cout, Y, dev_status);
+    p.wdense = Wd;
+    return dense_forward(p, dtype, reinterpret_cast<cudaStream_t>(stream));
+}
+
+cci_status cci_dense_conv2d_tc(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
+                               const void *Wd, int64_t Cout, int KH, int KW, int stride_h, int stride_w, int pad_h,
+                               int pad_w, float *Y, uint32_t *dev_status, cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (!Wd || (B > 0 && (!X || !Y))) return CCI_ERR_NULL;
+    FwdParams p{};
+    const cci_status st = conv_params(B, H, W, Cin, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, &p);
+    if (st != CCI_OK) return st;
+    if (!mul_ok(Cout, p.R)) return CCI_ERR_SHAPE;
+    p.X = X;
+    p.Y = Y;
+    p.status = dev_status;
+    p.wdense = Wd;
+    return dense_forward(p, dtype, reinterpret_cast<cudaStream_t>(stream));
 }
 
 const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K, cci_algo algo)
@@ -575,7 +633,11 @@ extern "C" cci_status cci_linear_dense_tc_static(const void *X, cci_dtype dtype,
     const cci_status st = check_common(X, dtype, values, idx, Y, N, Cout, Cin, G, K);
     if (st != CCI_OK) return st;
     if (dtype != CCI_BF16) return CCI_ERR_UNSUPPORTED;  // the array holds bf16 dense weights
-    if (!mul_ok(N, Cin)) return CCI_ERR_SHAPE;
+    if (!mul_ok(N, Cin) || !mul_ok(Cout, Cin)) return CCI_ERR_SHAPE;
+    // shapes outside the dense kernel's limits are unsupported whatever their size;
+    // only then is the size compared with the array (Cout * Cin cannot wrap here)
+    if (Cin >= (int64_t(1) << 31) || Cout >= (int64_t(1) << 31) || !dense_tc_shape_ok(dtype, G, K, Cin, Cin))
+        return CCI_ERR_UNSUPPORTED;
     if (dense_ws_bytes(dtype, Cout, Cin) > kStaticWsBytes) return CCI_ERR_WORKSPACE;
     if (N == 0) return CCI_OK;
     void *ws = nullptr;

@@ -375,14 +375,10 @@ cudaError_t launch_generic(const FwdParams &p, int dtype, int G, int K, cudaStre
     const int64_t n_col_tiles = (p.N + 127) / 128;
     const int64_t tiles = n_col_tiles * (p.Cout / G);
     const size_t smem = static_cast<size_t>(G) * 128 * sizeof(float);
-    static const bool attr = [] {
-        cudaFuncSetAttribute(generic_kernel<uint32_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             256 * 128 * 4);
-        cudaFuncSetAttribute(generic_kernel<uint16_t>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             256 * 128 * 4);
-        return true;
-    }();
-    (void)attr;
+    static SmemAttrCache attr_f32, attr_bf16;
+    const cudaError_t attr = dtype == CCI_F32 ? smem_attr_once(generic_kernel<uint32_t>, 256 * 128 * 4, attr_f32)
+                                              : smem_attr_once(generic_kernel<uint16_t>, 256 * 128 * 4, attr_bf16);
+    if (attr != cudaSuccess) return attr;
     if (tiles > 0x7fffffffll) return cudaErrorInvalidConfiguration;
     if (dtype == CCI_F32)
         generic_kernel<uint32_t><<<static_cast<unsigned>(tiles), 128, smem, stream>>>(p, G, K, n_col_tiles);

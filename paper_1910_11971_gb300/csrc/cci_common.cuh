@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cstdint>
+#include <mutex>
 #include <cuda_runtime.h>
 
 #include "cci.h"
@@ -26,6 +27,7 @@ struct FwdParams {
     int KH, KW, sh, sw, ph, pw;
     int is_conv;
     const void *wdense;  // dense decompressed weights [Cout][R] (workspace kernels only)
+    int G, K;            // group size and kept weights per group (fused tensor-core kernel)
     // output epilogue (workspace kernels only): y + bias[co], ReLU, bf16 output
     const float *bias;   // nullptr: none
     int relu;
@@ -105,6 +107,32 @@ __device__ __forceinline__ int64_t x_offset(const FwdParams &p, const ColumnSite
     const int w = s.wb + kw;
     if (h < 0 || h >= p.H || w < 0 || w >= p.W) return -1;
     return s.img + (static_cast<int64_t>(h) * p.W + w) * p.Cin + ci;
+}
+
+// Per-device record of a kernel's dynamic shared-memory limit: the CUDA runtime
+// keeps cudaFuncAttributeMaxDynamicSharedMemorySize per device context, so it is
+// set once on every device the kernel is launched on (the first launch there).
+struct SmemAttrCache {
+    static constexpr int kDevices = 64;
+    std::mutex m;
+    bool set[kDevices] = {};
+    cudaError_t err[kDevices] = {};
+};
+
+// cudaFuncSetAttribute(kern, MaxDynamicSharedMemorySize, bytes) on the current
+// device, once per device; later calls return the first call's result
+template <typename Kern>
+cudaError_t smem_attr_once(Kern kern, int bytes, SmemAttrCache &c)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= SmemAttrCache::kDevices)
+        return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(c.m);
+    if (!c.set[dev]) {
+        c.err[dev] = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+        c.set[dev] = true;
+    }
+    return c.err[dev];
 }
 
 }  // namespace cci

@@ -285,8 +285,8 @@ template <int G, int K, bool WS>
 cudaError_t launch(const FwdParams &p, cudaStream_t stream)
 {
     auto kern = dense_tc_kernel<G, K, WS>;
-    static const cudaError_t attr =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kSmemBytes));
+    static SmemAttrCache attr_cache;
+    const cudaError_t attr = smem_attr_once(kern, static_cast<int>(kSmemBytes), attr_cache);
     if (attr != cudaSuccess) return attr;
     const int64_t n_ct = (p.Cout + kN - 1) / kN;
     const int64_t n_nt = (p.N + kM - 1) / kM;

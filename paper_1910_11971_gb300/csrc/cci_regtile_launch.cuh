@@ -20,8 +20,8 @@ cudaError_t launch_regtile_wc(const FwdParams &p, cudaStream_t stream)
     using RT = RegTile<TS, G, K, MG, T, D, WC>;
     static_assert(RT::kTotal <= kMaxSmemPerBlock, "shared-memory layout over the per-block limit");
     auto kern = regtile_kernel<TS, G, K, MG, T, D, WC>;
-    static const cudaError_t attr =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(RT::kTotal));
+    static SmemAttrCache attr_cache;
+    const cudaError_t attr = smem_attr_once(kern, static_cast<int>(RT::kTotal), attr_cache);
     if (attr != cudaSuccess) return attr;
     const int64_t groups = p.Cout / G;
     const int64_t n_ct = (groups + RT::kNGR - 1) / RT::kNGR;

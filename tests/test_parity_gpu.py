@@ -159,13 +159,20 @@ def test_linear_tiny_workload(dev):
     assert_within_tol(f64(Y), Yo, S, case.name)
 
 
-def test_linear_bottleneck_full(dev):
+FULL_FAMILIES = [(cci.ALGO_AUTO, "dense_tc"), (cci.ALGO_REGTILE, "regtile"), (cci.ALGO_EXPAND, "expand")]
+
+
+@pytest.mark.parametrize("algo,prefix", FULL_FAMILIES, ids=["auto", "regtile", "expand"])
+def test_linear_bottleneck_full(dev, algo, prefix):
     """N = 100352 columns, 256 -> 1024, G=8, K=2, fp32: every output written;
-    2048 sampled rows against the oracle."""
+    2048 sampled rows against the oracle.  AUTO through the binding (which
+    passes a workspace) runs the tensor-core family; the two CUDA-core scatter
+    families are selected explicitly."""
     case = wl.BOTTLENECK_1X1
     X, W = wl.linear_inputs(case)
-    assert cci.kernel_name(F32, case.Cin, case.R, case.Cout, case.G, case.K).startswith(("regtile", "expand"))
-    Y = run_linear(dev, X, W, case.G, case.K)
+    named = cci.ALGO_DENSE_TC_WS if algo == cci.ALGO_AUTO else algo
+    assert cci.kernel_name(F32, case.Cin, case.R, case.Cout, case.G, case.K, named).startswith(prefix)
+    Y = run_linear(dev, X, W, case.G, case.K, algo)
     assert torch.isfinite(Y).all()
     rows = sample_rows(case.N, 2048)
     _, _, Wd, mask = oracle_reference(W, case.G, case.K)
@@ -303,39 +310,62 @@ def test_conv_1x1_equals_linear_bitwise(dev):
     assert torch.equal(Yc.reshape(-1, Cout).view(torch.int32), Yl.view(torch.int32))
 
 
-def conv_points(case, k: int, seed: int):
-    """Sampled output positions from the first and last image of the batch."""
+def conv_images(B: int, seed: int):
+    """Images the sampled outputs come from: the first, the last, the middle one
+    and a seeded interior one (4-D copy boxes span several images, so interior
+    images sit inside boxes as well as on their edges)."""
+    rng = np.random.default_rng(seed + 7)
+    imgs = {0, B - 1, B // 2}
+    if B > 3:
+        imgs.add(int(rng.integers(1, B - 1)))
+    return sorted(imgs)
+
+
+def conv_points(case, k: int, seed: int, imgs):
+    """Sampled output positions of the images `imgs` (as rows of the NHWC output):
+    per image its first and last pixels (tile edges, the ragged tail) and random
+    ones."""
     P, Q = case.P, case.Q
     per = P * Q
     rng = np.random.default_rng(seed)
-    first = np.concatenate([np.arange(min(per, k // 4)), rng.choice(per, size=k // 4)])
-    last = (case.B - 1) * per + np.concatenate([np.arange(per - min(per, k // 4), per),
-                                                rng.choice(per, size=k // 4)])
-    return np.unique(np.concatenate([first, last]))
+    each = max(8, k // len(imgs))
+    pts = []
+    for b in imgs:
+        edge = min(per, each // 4)
+        pts.append(b * per + np.concatenate([np.arange(edge), np.arange(per - edge, per),
+                                             rng.choice(per, size=each // 2)]))
+    return np.unique(np.concatenate(pts))
 
 
-def check_conv_case(dev, case, npts=1024, seed=0):
+def check_conv_case(dev, case, npts=1024, seed=0, algo=cci.ALGO_AUTO):
     X, W = wl.conv_inputs(case, device="cpu")
     Y = run_conv(dev, X, W, (case.KH, case.KW, (case.stride,) * 2, (case.pad,) * 2, case.Cout),
-                 case.G, case.K)
+                 case.G, case.K, algo)
     assert torch.isfinite(Y).all()
-    pts = conv_points(case, npts, seed)
-    # oracle on the two images the points come from
-    imgs = [0, case.B - 1] if case.B > 1 else [0]
+    imgs = conv_images(case.B, seed)
+    pts = conv_points(case, npts, seed, imgs)
+    # oracle on the images the points come from, the points renumbered within them
     Xs = f64(X[imgs])
     per = case.P * case.Q
-    local = np.where(pts < per, pts, pts - (case.B - 1) * per + (per if case.B > 1 else 0))
+    pos = {b: j for j, b in enumerate(imgs)}
+    local = np.array([pos[int(p) // per] * per + int(p) % per for p in pts], dtype=np.int64)
     _, _, Wd, mask = oracle_reference(W, case.G, case.K)
     Yo, S = oracle.conv2d(Xs, Wd, mask, case.KH, case.KW, (case.stride,) * 2, (case.pad,) * 2, pts=local)
     Yg = f64(Y.reshape(-1, case.Cout)[torch.from_numpy(pts).to(dev)])
     assert_within_tol(Yg, Yo, S, case.name)
 
 
-def test_conv3x3_full(dev):
-    """Batch 64, 28x28, 128 -> 128, 3x3 s1 p1, G=16, K=4, bf16."""
+@pytest.mark.parametrize("algo,prefix", FULL_FAMILIES, ids=["auto", "regtile", "expand"])
+def test_conv3x3_full(dev, algo, prefix):
+    """Batch 64, 28x28, 128 -> 128, 3x3 s1 p1, G=16, K=4, bf16, through AUTO (the
+    tensor-core family) and the two CUDA-core scatter families explicitly."""
     case = wl.CONV3X3_28
-    assert cci.kernel_name(BF16, case.Cin, case.R, case.Cout, case.G, case.K).startswith(("regtile", "expand"))
-    check_conv_case(dev, case, npts=2048)
+    named = cci.ALGO_DENSE_TC_WS if algo == cci.ALGO_AUTO else algo
+    name = cci.kernel_name(BF16, case.Cin, case.R, case.Cout, case.G, case.K, named)
+    if not name:
+        pytest.skip("no register tile for (G, K) = (16, 4) in bf16")
+    assert name.startswith(prefix)
+    check_conv_case(dev, case, npts=2048, algo=algo)
 
 
 RESNET_PICK = [0, 1, 3, 4, 11, 13, 15, 24, 25, 28, 42, 44, 47, 49, 51]
@@ -407,18 +437,7 @@ def test_dense_tc_conv_small(dev, case, algo):
 
 @pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
 def test_dense_tc_conv3x3_full(dev, algo):
-    case = wl.CONV3X3_28
-    X, W = wl.conv_inputs(case, device="cpu")
-    Y = run_conv(dev, X, W, (case.KH, case.KW, (case.stride,) * 2, (case.pad,) * 2, case.Cout),
-                 case.G, case.K, algo)
-    assert torch.isfinite(Y).all()
-    pts = conv_points(case, 1024, 5)
-    Xs = f64(X[[0, case.B - 1]])
-    per = case.P * case.Q
-    local = np.where(pts < per, pts, pts - (case.B - 1) * per + per)
-    _, _, Wd, mask = oracle_reference(W, case.G, case.K)
-    Yo, S = oracle.conv2d(Xs, Wd, mask, 3, 3, (1, 1), (1, 1), pts=local)
-    assert_within_tol(f64(Y.reshape(-1, case.Cout)[torch.from_numpy(pts).to(dev)]), Yo, S, "conv3x3 dense_tc")
+    check_conv_case(dev, wl.CONV3X3_28, npts=1024, seed=5, algo=algo)
 
 
 @pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
@@ -802,3 +821,43 @@ def test_pack_stats_estimates_eq1(dev, G, Ps):
     # per group the overflow is at most G - K; its variance is bounded by E[over] * (G - K)
     se = np.sqrt(pd * K * (G - K) / groups) / K
     assert abs(est - pd) < 5 * se + 1e-9, (est, pd, se)
+
+
+# ---------------------------------------------------------------------------
+# the same tensor-core GEMM on dense (unpruned) weights: the reference line of
+# what the sparsity buys
+# ---------------------------------------------------------------------------
+def dense_planes(W: torch.Tensor) -> torch.Tensor:
+    """The dense family's weight layout: bf16 as is; fp32 as hi / lo tf32 planes
+    (hi = the low 13 mantissa bits cleared, lo = w - hi, both exact)."""
+    if W.dtype == BF16:
+        return W.contiguous()
+    hi = (W.view(torch.int32) & -8192).view(torch.float32)
+    return torch.stack([hi, W - hi]).contiguous()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("N,Cin,Cout", [(300, 64, 256), (129, 72, 40), (1000, 256, 1024), (2048, 512, 512)])
+def test_dense_linear_tc(dev, dtype, N, Cin, Cout):
+    X, W = wl.random_small(N + Cin + 1, dtype, N, Cin, Cout)
+    Y = torch.full((N, Cout), float("nan"), device=dev)
+    st = cci.new_status(dev)
+    cci.dense_linear_tc(X.to(dev), dense_planes(W).to(dev), Cout, out=Y, status=st)
+    assert cci.read_status(st) == 0
+    Yo, S = oracle.linear(f64(X), f64(W), np.ones((Cout, Cin), dtype=bool))
+    assert_within_tol(f64(Y), Yo, S, f"dense {dtype} {N}x{Cin}->{Cout}")
+
+
+@pytest.mark.parametrize("case", [(2, 14, 14, 64, 128, 3, 3, 1, 1, "bf16"), (3, 9, 9, 32, 64, 3, 3, 2, 1, "bf16"),
+                                  (2, 8, 8, 16, 32, 1, 1, 1, 0, "f32")],
+                         ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_{}".format(*c))
+def test_dense_conv2d_tc(dev, case):
+    B, H, Wi, Cin, Cout, KH, KW, s, p, dtype = case
+    g = torch.Generator().manual_seed(B + Cin)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(_dt(dtype))
+    W = torch.randn((Cout, KH * KW * Cin), generator=g).to(_dt(dtype))
+    st = cci.new_status(dev)
+    Y = cci.dense_conv2d_tc(X.to(dev), dense_planes(W).to(dev), Cout, KH, KW, (s, s), (p, p), status=st)
+    assert cci.read_status(st) == 0
+    Yo, S = oracle.conv2d(f64(X), f64(W), np.ones(W.shape, dtype=bool), KH, KW, (s, s), (p, p))
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))

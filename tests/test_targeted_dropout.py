@@ -60,7 +60,10 @@ def test_drop_frequency():
 
 
 def test_drop_rate_schedule():
-    """50 % at the start, 100 % at the end (Sec. 5.1), non-decreasing between."""
+    """50 % at the start, 100 % at the end (Sec. 5.1), non-decreasing between (the
+    library's host function; no device work)."""
+    from paper_1910_11971_gb300 import build as cci_build
+    cci_build.build()
     rates = [cci.td_drop_rate(s, 1000) for s in range(0, 1201, 50)]
     assert rates[0] == 0.5 and rates[-1] == 1.0 and cci.td_drop_rate(1000, 1000) == 1.0
     assert all(a <= b for a, b in zip(rates, rates[1:]))
