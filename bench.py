@@ -440,8 +440,7 @@ def dense_planes(W: torch.Tensor) -> torch.Tensor:
 def launches_per_product(cci, dtype, case) -> int:
     """Kernels one product launches on the production path (AUTO): the workspace
     family runs a decompression and the GEMM, every other family one kernel."""
-    name = cci.kernel_name(dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
-                           workspace=True)
+    name = cci.kernel_name(dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO)
     return 2 if name.startswith("dense_tc_ws") else 1
 
 
@@ -474,8 +473,7 @@ def run_ours(args, rank, world, local):
         ws = cci.auto_workspace(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K, dev)
     else:
         ws = cci.new_workspace(algo, Xd.dtype, case.Cout, case.R, dev)
-    kname = cci.kernel_name(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
-                            workspace=ws is not None)
+    kname = cci.kernel_name(Xd.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO)
     on_tc = kname.startswith("dense_tc")
     status = cci.new_status(dev)
     flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
@@ -633,7 +631,7 @@ def run_sweep(cci, dev, stream, flush, reps=10):
                     "cublas": sig(dms / ms, 3), "same": sig(dense_same_ms / ms, 3)})
         tu.append({"G": G, "K": K, "tensor_util": case.dense_flops() / (ms * 1e-3) / 1e12 / peak,
                    "cublas_ms": dms, "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, G, K,
-                                                               cci.ALGO_AUTO, workspace=ws is not None)})
+                                                               cci.ALGO_AUTO)})
         del X, W, v, i, Y, Wm, ws
     torch.cuda.empty_cache()
     extra("sweep_4096_details", {"same_kernel_dense_ms": dense_same_ms, "points": tu,
@@ -695,8 +693,7 @@ def run_bottleneck_fp32(cci, dev, stream, flush, reps=10):
     floor_s = max(nzf / (ALU_PEAK_TFLOPS * 1e12), algorithmic_bytes(case, 4) / (HBM_ROOF_GBS * 1e9))
     return {"workload": case.name, "ms": ms, "nz_tflops": nzf / (ms * 1e-3) / 1e12,
             "metric_roofline_frac": floor_s / (ms * 1e-3),
-            "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
-                                      workspace=ws is not None),
+            "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO),
             "cublas_fp32_simt_ms": dms, "speedup_over_cublas_fp32": dms / ms,
             "same_kernel_dense_ms": sms, "sparsity_gain": sms / ms,
             "tensor_vs_simt": dms / sms,
@@ -728,8 +725,7 @@ def run_conv3x3(cci, dev, stream, flush, reps=10):
     return {"workload": case.name, "ms": ms, "nz_tflops": nzf / (ms * 1e-3) / 1e12,
             "metric_roofline_frac": layer_floor_us(case) * 1e-3 / ms,
             "dense_equiv_tflops": case.dense_flops() / (ms * 1e-3) / 1e12,
-            "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO,
-                                      workspace=ws is not None),
+            "kernel": cci.kernel_name(X.dtype, case.Cin, case.R, case.Cout, case.G, case.K, cci.ALGO_AUTO),
             "cudnn_bf16_ms": dms, "speedup_over_cudnn": dms / ms,
             "same_kernel_dense_ms": sms, "sparsity_gain": sms / ms,
             "families": kernel_families(cci, case, X, v, i, Y, True, flush, stream)}
@@ -984,7 +980,7 @@ def run_resnet_stack(cci, dev, stream, flush, reps=5):
                 per_layer.append({"layer": c.name, "ms": round(lm, 5), "floor_ms": round(layer_floor_us(c) * 1e-3, 5),
                                   "cudnn_ms": round(ld, 5), "same_kernel_dense_ms": round(ls, 5),
                                   "kernel": cci.kernel_name(torch.bfloat16, c.Cin, c.R, c.Cout, c.G, c.K,
-                                                            cci.ALGO_AUTO, workspace=kp[8] is not None)})
+                                                            cci.ALGO_AUTO)})
         # the same 52 layers chained through the fused epilogue: each layer reads
         # the bf16 output of the layer before it in its block (the first block its
         # synthetic input), adds a bias, applies ReLU (a and b) and writes bf16

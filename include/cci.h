@@ -83,14 +83,27 @@ typedef enum cci_dtype {
 
 /* Kernel family for cci_linear_ex / cci_conv2d_ex. */
 typedef enum cci_algo {
-    CCI_ALGO_AUTO = 0,      /* the fastest family this build has for (G, K, dtype, shape) */
+    CCI_ALGO_AUTO = 0,      /* the fastest family this build has for (G, K, dtype, shape): the
+                               workspace tensor-core family when a large enough workspace is
+                               given (cci_linear_ws); else the fused tensor-core family
+                               (CCI_ALGO_DENSE_TC) for bf16 layers that have it; else the
+                               CUDA-core families */
     CCI_ALGO_GENERIC = 1,   /* generic kernel: any G <= 256, any K, any alignment */
     CCI_ALGO_REGTILE = 2,   /* register-tiled scatter on CUDA cores: Alg. 2 with the output
                                row chosen per (group, r) by a warp-uniform jump;
                                CCI_ERR_UNSUPPORTED when (G, K, dtype, shape) has no tile */
-    CCI_ALGO_DENSE_TC = 3,  /* comparison only: decompress to bf16 tiles in shared
-                               memory and multiply densely on the tensor cores
-                               (tcgen05); bf16 only */
+    CCI_ALGO_DENSE_TC = 3,  /* fused tensor-core family, no workspace: inside the GEMM the
+                               packed (value, index) runs of each stage are copied by TMA
+                               and expanded by producer warps into the dense bf16 weight
+                               tile in shared memory (each value to row G*i + Idx of its
+                               group, Alg. 2), which tcgen05.mma multiplies with the TMA-
+                               copied activations.  bf16; G in {4, 8, 16, 32}, K in
+                               {1, 2, 4, 8} with K <= G/2; Cin % 8 == 0, R*K % 16 == 0;
+                               16-byte aligned X, Y, values and idx; activations a product
+                               or a convolution with strides <= 2 and Cin % 64 == 0 (else
+                               CCI_ERR_UNSUPPORTED).  Index sets are checked (strictly
+                               increasing, < G; CCI_ERR_INDEX) by the CTAs of the first
+                               column tile of every channel tile */
     CCI_ALGO_EXPAND = 4,    /* register-tiled on CUDA cores without jumps: each (group, r)
                                is expanded to its G weights (pruned ones zero) in shared
                                memory and all G rows are updated; same shape rules as
@@ -165,7 +178,8 @@ cci_status cci_conv2d(const void *X, cci_dtype dtype, int64_t B, int64_t H, int6
                       int K, float *Y, uint32_t *dev_status, cci_stream_t stream);
 
 /* As cci_linear / cci_conv2d, with the kernel family chosen by `algo` and no
- * workspace (CCI_ALGO_DENSE_TC_WS returns CCI_ERR_WORKSPACE; AUTO does not pick it). */
+ * workspace (CCI_ALGO_DENSE_TC_WS returns CCI_ERR_WORKSPACE; AUTO does not pick it,
+ * but does pick the fused tensor-core family, which needs none). */
 cci_status cci_linear_ex(const void *X, cci_dtype dtype, int64_t N, int64_t Cin,
                          const void *values, const uint8_t *idx, int64_t Cout, int G, int K,
                          float *Y, uint32_t *dev_status, cci_algo algo, cci_stream_t stream);
@@ -208,10 +222,11 @@ cci_status cci_conv2d_ws(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
  * X_host[N][Cin] * Wd^T, Wd the dense matrix of the packed weights (which stay
  * on the device).  The columns are processed in chunks of `chunk_cols`; chunk c
  * is copied in on `copy_in_stream`, multiplied on `stream` (the dense
- * tensor-core family, CCI_ALGO_DENSE_TC_WS; the weights are decompressed once,
- * by the first chunk) and copied out on `copy_out_stream`, so that the copies of
- * neighbouring chunks overlap the product.  The result equals cci_linear_ws
- * with CCI_ALGO_DENSE_TC_WS on the same data bit for bit.
+ * tensor-core family AUTO picks: the fused one from the packed weights, else the
+ * workspace one, the weights decompressed once by the first chunk) and copied
+ * out on `copy_out_stream`, so that the copies of neighbouring chunks overlap
+ * the product.  The result equals cci_linear_ws with CCI_ALGO_AUTO and a
+ * workspace on the same data bit for bit.
  *
  *   X_host, Y_host  host memory; page-locked (cudaHostAlloc / registered) for the
  *                   copies to overlap; pageable memory is correct but serialises
@@ -310,7 +325,8 @@ cci_status cci_pack_stats(const void *W, cci_dtype dtype, int64_t Cout, int64_t 
 
 /*
  * cci_linear_fused / cci_conv2d_fused -- the product / convolution of
- * cci_linear_ws / cci_conv2d_ws with CCI_ALGO_DENSE_TC_WS, followed by the usual
+ * cci_linear_ws / cci_conv2d_ws on a tensor-core family (the fused one where AUTO
+ * would pick it or no workspace is given, else CCI_ALGO_DENSE_TC_WS), followed by the usual
  * output stage of a CNN layer, applied in the kernel's epilogue to each fp32
  * accumulator y[n][co] (the sum of Alg. 2, Sec. 3.2):
  *   y += bias[co]          when bias != NULL (fp32, Cout entries, 16-byte aligned);
@@ -319,8 +335,9 @@ cci_status cci_pack_stats(const void *W, cci_dtype dtype, int64_t Cout, int64_t 
  *                          bf16, ties to even (out_dtype CCI_BF16; needs Cout % 8 == 0).
  * The paper defines only the product; bias, ReLU and the bf16 output are the
  * surrounding network's, fused here so that a layer's output is written once at
- * the width the next layer reads.  X and Y must be 16-byte aligned and the
- * workspace as for CCI_ALGO_DENSE_TC_WS (else CCI_ERR_ALIGN / CCI_ERR_WORKSPACE);
+ * the width the next layer reads.  X and Y must be 16-byte aligned and, for
+ * layers without the fused family, the workspace as for CCI_ALGO_DENSE_TC_WS
+ * (else CCI_ERR_ALIGN / CCI_ERR_WORKSPACE; the workspace may be NULL otherwise);
  * layers without that family return CCI_ERR_UNSUPPORTED.  Y is [N][Cout] or NHWC
  * [B][P][Q][Cout] of out_dtype; everything else as for cci_linear_ws /
  * cci_conv2d_ws.  NaN accumulators become 0 under the ReLU.
@@ -396,10 +413,12 @@ cci_status cci_linear_dense_tc_static(const void *X, cci_dtype dtype, int64_t N,
                                       int K, float *Y, uint32_t *dev_status, cci_stream_t stream);
 
 /*
- * cci_kernel_name -- the name of the kernel that cci_linear_ex / cci_conv2d_ex
- * would launch for a layer with these sizes (R = Cin for a product, Cin*KH*KW
- * for a convolution) when every pointer is 16-byte aligned: a static string, ""
- * when the call would be rejected.  No device work; used to label results.
+ * cci_kernel_name -- the name of the kernel family that cci_linear_ws /
+ * cci_conv2d_ws would run for a layer with these sizes (R = Cin for a product,
+ * Cin*KH*KW for a convolution, taken to have strides <= 2) when every pointer is
+ * 16-byte aligned and, for CCI_ALGO_AUTO, the workspace is the one
+ * cci_workspace_size(CCI_ALGO_AUTO) asks for: a static string, "" when the call
+ * would be rejected.  No device work; used to label results.
  */
 const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K,
                             cci_algo algo);

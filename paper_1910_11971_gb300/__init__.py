@@ -276,7 +276,7 @@ def conv2d(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout: int, 
     Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=torch.float32,
                                                 device=X.device)
     if workspace is None and algo == ALGO_AUTO:
-        workspace = auto_workspace(X.dtype, Cin, KH * KW * Cin, Cout, G, K, X.device)
+        workspace = auto_workspace(X.dtype, Cin, KH * KW * Cin, Cout, G, K, X.device, max(stride))
     elif workspace is None and algo == ALGO_DENSE_TC_WS:
         workspace = new_workspace(algo, X.dtype, Cout, KH * KW * Cin, X.device)
     wp, wb = _ws(workspace)
@@ -367,11 +367,12 @@ def linear_fused(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout:
                  out_dtype: torch.dtype = torch.float32, out: Optional[torch.Tensor] = None,
                  status: Optional[torch.Tensor] = None,
                  workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
-    """Y[N][Cout] = relu?(product + bias) in ``out_dtype`` (fp32 or bf16), on the
-    workspace tensor-core family (``cci_linear_fused``)."""
+    """Y[N][Cout] = relu?(product + bias) in ``out_dtype`` (fp32 or bf16), on a
+    tensor-core family (``cci_linear_fused``: the fused one where AUTO takes it,
+    else the workspace one, whose workspace is allocated here when not given)."""
     _cuda_contig(X, "X")
     N, Cin = X.shape
-    if workspace is None:
+    if workspace is None and not kernel_name(X.dtype, Cin, Cin, Cout, G, K).startswith("dense_tc_fused"):
         workspace = new_workspace(ALGO_DENSE_TC_WS, X.dtype, Cout, Cin, X.device)
     Y = out if out is not None else torch.empty((N, Cout), dtype=out_dtype, device=X.device)
     if bias is not None:
@@ -392,13 +393,14 @@ def conv2d_fused(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout:
                  out: Optional[torch.Tensor] = None, status: Optional[torch.Tensor] = None,
                  workspace: Optional[torch.Tensor] = None) -> torch.Tensor:
     """Y NHWC [B][P][Q][Cout] = relu?(convolution + bias) in ``out_dtype`` (fp32 or
-    bf16), on the workspace tensor-core family (``cci_conv2d_fused``)."""
+    bf16), on a tensor-core family (``cci_conv2d_fused``, as ``linear_fused``)."""
     _cuda_contig(X, "X")
     B, H, W, Cin = X.shape
     P, Q = conv_out_hw(H, W, KH, KW, stride, pad)
     Y = out if out is not None else torch.empty((B, max(P, 0), max(Q, 0), Cout), dtype=out_dtype,
                                                 device=X.device)
-    if workspace is None:
+    fused = kernel_name(X.dtype, Cin, KH * KW * Cin, Cout, G, K).startswith("dense_tc_fused") and max(stride) <= 2
+    if workspace is None and not fused:
         workspace = new_workspace(ALGO_DENSE_TC_WS, X.dtype, Cout, KH * KW * Cin, X.device)
     if bias is not None:
         _cuda_contig(bias, "bias")
@@ -446,29 +448,23 @@ def dense_conv2d_tc(X: torch.Tensor, Wd: torch.Tensor, Cout: int, KH: int, KW: i
 
 
 def kernel_name(dtype: torch.dtype, Cin: int, R: int, Cout: int, G: int, K: int,
-                algo: int = ALGO_AUTO, workspace: bool = False) -> str:
-    """The kernel family a call would run (``cci_kernel_name``).  With
-    ``workspace=True`` and AUTO: the family AUTO picks when it is given the
-    workspace it asks for (the workspace tensor-core family where the fused one
-    does not apply)."""
+                algo: int = ALGO_AUTO) -> str:
+    """The kernel family a call would run (``cci_kernel_name``; for AUTO: given the
+    workspace ``auto_workspace`` provides)."""
     code = F32 if dtype == torch.float32 else BF16
-    name = lib().cci_kernel_name(code, Cin, R, Cout, G, K, algo).decode()
-    if algo == ALGO_AUTO and workspace and not name.startswith("dense_tc"):
-        ws_name = lib().cci_kernel_name(code, Cin, R, Cout, G, K, ALGO_DENSE_TC_WS).decode()
-        if ws_name:
-            return ws_name
-    return name
+    return lib().cci_kernel_name(code, Cin, R, Cout, G, K, algo).decode()
 
 
 def auto_workspace(dtype: torch.dtype, Cin: int, R: int, Cout: int, G: int, K: int,
-                   device) -> Optional[torch.Tensor]:
+                   device, stride: int = 1) -> Optional[torch.Tensor]:
     """The workspace AUTO needs to reach its fastest family for a layer (R = Cin
-    for a product, KH*KW*Cin for a convolution), from PyTorch memory: None when
-    that family needs none (the library allocates nothing itself)."""
-    if kernel_name(dtype, Cin, R, Cout, G, K, ALGO_AUTO).startswith("dense_tc"):
+    for a product, KH*KW*Cin for a convolution of the given largest stride), from
+    PyTorch memory: None when that family needs none (the library allocates
+    nothing itself)."""
+    name = kernel_name(dtype, Cin, R, Cout, G, K, ALGO_AUTO)
+    if name.startswith("dense_tc_fused") and stride <= 2:
         return None
-    if not lib().cci_kernel_name(F32 if dtype == torch.float32 else BF16, Cin, R, Cout, G, K,
-                                 ALGO_DENSE_TC_WS):
+    if not lib().cci_kernel_name(F32 if dtype == torch.float32 else BF16, Cin, R, Cout, G, K, ALGO_DENSE_TC_WS):
         return None
     return new_workspace(ALGO_DENSE_TC_WS, dtype, Cout, R, device)
 

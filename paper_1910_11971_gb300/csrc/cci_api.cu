@@ -99,35 +99,93 @@ cci_status dense_forward(FwdParams p, int dtype, cudaStream_t stream)
     return to_status(launch_gemm_ws(p, dtype, stream));
 }
 
+// the fused tensor-core family (packed weights expanded in the GEMM, no
+// workspace) may have this layer: bf16, a dense-kernel shape, 16-byte aligned
+// operands and the expansion's conditions (gemm_pk_shape_ok); whether its
+// activations can be copied by TMA is settled by launch_gemm_pk, which returns
+// cudaErrorNotSupported before launching anything when they cannot
+bool fused_may(const FwdParams &p, int dtype)
+{
+    const bool tc_fits = p.R < (int64_t(1) << 31) && p.Cout < (int64_t(1) << 31);
+    return dtype == CCI_BF16 && tc_fits && p.Cin % 8 == 0 && p.R % 8 == 0 && p.Cout % 4 == 0 && aligned(p.X, 16) &&
+           aligned(p.Y, 16) && gemm_pk_shape_ok(p);
+}
+
+// the entry points with an output epilogue (cci_linear_fused, cci_conv2d_fused):
+// a tensor-core family, whatever the epilogue flags
+constexpr cci_algo kAlgoEpilogue = static_cast<cci_algo>(100);
+
+// AUTO takes the fused family over the workspace family when the caller gives a
+// workspace only where it measured faster on GB300: nowhere yet (the K/G sweep
+// point G = 8, K = 2: 0.57 ms fused against 0.16 ms decompression + GEMM), so
+// with a workspace AUTO runs the workspace family, without one the fused family
+bool auto_prefers_fused(int K)
+{
+    (void)K;
+    return false;
+}
+
+// 1: the fused kernel was launched, 0: the layer does not have it (nothing
+// enqueued), -1: launch error
+int try_fused(const FwdParams &p, int dtype, cudaStream_t stream)
+{
+    if (!fused_may(p, dtype)) return 0;
+    const cudaError_t e = launch_gemm_pk(p, stream);
+    if (e == cudaErrorNotSupported) return 0;
+    return e == cudaSuccess ? 1 : -1;
+}
+
+cci_status fused_status(int r) { return r > 0 ? CCI_OK : CCI_ERR_CUDA; }
+
 cci_status forward(FwdParams p, int dtype, int G, int K, cci_algo algo, void *ws, size_t ws_bytes,
                    cudaStream_t stream)
 {
     // a 1x1 convolution with unit stride and no padding is the product of X[B*H*W][Cin]
     if (p.is_conv && p.KH == 1 && p.KW == 1 && p.sh == 1 && p.sw == 1 && p.ph == 0 && p.pw == 0) p.is_conv = 0;
+    p.G = G;
+    p.K = K;
     const bool tc_fits = p.R < (int64_t(1) << 31) && p.Cout < (int64_t(1) << 31);  // 32-bit copy coordinates
-    if (p.bias || p.relu || p.out_bf16) {
-        // the output epilogue exists on the workspace tensor-core family only
-        if (!tc_fits || !dense_tc_shape_ok(dtype, G, K, p.Cin, p.R)) return CCI_ERR_UNSUPPORTED;
+    const bool ws_ok = ws && ws_bytes >= dense_ws_bytes(dtype, p.Cout, p.R) && aligned(ws, 16);
+    const bool dense_ok = tc_fits && dense_tc_shape_ok(dtype, G, K, p.Cin, p.R);
+    if (algo == kAlgoEpilogue || p.bias || p.relu || p.out_bf16) {
+        // the output epilogue exists on the tensor-core families: the fused one when
+        // the layer has it (preferred as for AUTO, or when no workspace is given),
+        // else the workspace one
+        if (!dense_ok) return CCI_ERR_UNSUPPORTED;
         if (p.out_bf16 && p.Cout % 8 != 0) return CCI_ERR_UNSUPPORTED;  // 16-byte output rows
         if (p.bias && !aligned(p.bias, 16)) return CCI_ERR_ALIGN;
         if (!aligned(p.X, 16) || !aligned(p.Y, 16)) return CCI_ERR_ALIGN;
-        if (!ws || ws_bytes < dense_ws_bytes(dtype, p.Cout, p.R) || !aligned(ws, 16)) return CCI_ERR_WORKSPACE;
+        if (p.N == 0) return CCI_OK;
+        if (auto_prefers_fused(K) || !ws_ok) {
+            const int r = try_fused(p, dtype, stream);
+            if (r != 0) return fused_status(r);
+        }
+        if (!ws_ok) return CCI_ERR_WORKSPACE;
         algo = CCI_ALGO_DENSE_TC_WS;
     }
     if (p.N == 0) return CCI_OK;
-    if (algo == CCI_ALGO_AUTO && tc_fits && dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) && ws &&
-        ws_bytes >= dense_ws_bytes(dtype, p.Cout, p.R) && aligned(ws, 16) && aligned(p.X, 16) && aligned(p.Y, 16))
-        algo = CCI_ALGO_DENSE_TC_WS;
-    if (algo == CCI_ALGO_DENSE_TC || algo == CCI_ALGO_DENSE_TC_WS) {
-        const bool use_ws = algo == CCI_ALGO_DENSE_TC_WS;
+    if (algo == CCI_ALGO_AUTO) {
+        if (auto_prefers_fused(K)) {
+            const int r = try_fused(p, dtype, stream);
+            if (r != 0) return fused_status(r);
+        }
+        if (dense_ok && ws_ok && aligned(p.X, 16) && aligned(p.Y, 16)) {
+            algo = CCI_ALGO_DENSE_TC_WS;
+        } else if (!auto_prefers_fused(K)) {
+            const int r = try_fused(p, dtype, stream);
+            if (r != 0) return fused_status(r);
+        }
+    }
+    if (algo == CCI_ALGO_DENSE_TC) {
+        const int r = try_fused(p, dtype, stream);
+        return r == 0 ? CCI_ERR_UNSUPPORTED : fused_status(r);
+    }
+    if (algo == CCI_ALGO_DENSE_TC_WS) {
         if (!tc_fits || !dense_tc_shape_ok(dtype, G, K, p.Cin, p.R) || !aligned(p.X, 16) || !aligned(p.Y, 16))
             return CCI_ERR_UNSUPPORTED;
-        if (!use_ws && dtype != CCI_BF16) return CCI_ERR_UNSUPPORTED;  // shared-memory decompression: bf16 only
-        if (use_ws) {
-            if (!ws || ws_bytes < dense_ws_bytes(dtype, p.Cout, p.R) || !aligned(ws, 16)) return CCI_ERR_WORKSPACE;
-            p.wdense = ws;
-        }
-        return to_status(launch_dense_tc(p, dtype, G, K, use_ws, stream));
+        if (!ws_ok) return CCI_ERR_WORKSPACE;
+        p.wdense = ws;
+        return to_status(launch_dense_tc_ws(p, dtype, G, K, stream));
     }
     if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
         const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
@@ -407,7 +465,7 @@ cci_status cci_linear_fused(const void *X, cci_dtype dtype, int64_t N, int64_t C
                             size_t workspace_bytes, cci_stream_t stream)
 {
     if (!valid_dtype(out_dtype)) return CCI_ERR_DTYPE;
-    return linear_impl(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, CCI_ALGO_DENSE_TC_WS, workspace,
+    return linear_impl(X, dtype, N, Cin, values, idx, Cout, G, K, Y, dev_status, kAlgoEpilogue, workspace,
                        workspace_bytes, stream, Epilogue{bias, relu != 0, out_dtype == CCI_BF16});
 }
 
@@ -442,7 +500,7 @@ cci_status cci_conv2d_fused(const void *X, cci_dtype dtype, int64_t B, int64_t H
 {
     if (!valid_dtype(out_dtype)) return CCI_ERR_DTYPE;
     return conv_impl(X, dtype, B, H, W, Cin, values, idx, Cout, KH, KW, stride_h, stride_w, pad_h, pad_w, G, K, Y,
-                     dev_status, CCI_ALGO_DENSE_TC_WS, workspace, workspace_bytes, stream,
+                     dev_status, kAlgoEpilogue, workspace, workspace_bytes, stream,
                      Epilogue{bias, relu != 0, out_dtype == CCI_BF16});
 }
 
@@ -531,6 +589,41 @@ cci_status cci_dense_conv2d_tc(const void *X, cci_dtype dtype, int64_t B, int64_
     return dense_forward(p, dtype, reinterpret_cast<cudaStream_t>(stream));
 }
 
+namespace {
+
+// name of the fused tensor-core kernel for a layer, "" when it has none
+// (convolutions: as if the strides were at most 2, the condition of its
+// activation copies)
+const char *fused_name(int dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K)
+{
+    static const char *names[] = {"dense_tc_fused_bf16_G4_K1",  "dense_tc_fused_bf16_G4_K2",
+                                  "dense_tc_fused_bf16_G8_K1",  "dense_tc_fused_bf16_G8_K2",
+                                  "dense_tc_fused_bf16_G8_K4",  "dense_tc_fused_bf16_G16_K1",
+                                  "dense_tc_fused_bf16_G16_K2", "dense_tc_fused_bf16_G16_K4",
+                                  "dense_tc_fused_bf16_G16_K8", "dense_tc_fused_bf16_G32_K1",
+                                  "dense_tc_fused_bf16_G32_K2", "dense_tc_fused_bf16_G32_K4",
+                                  "dense_tc_fused_bf16_G32_K8"};
+    if (dtype != CCI_BF16 || Cin % 8 != 0 || R % 8 != 0 || Cout % 4 != 0 || Cout % G != 0) return "";
+    if (R >= (int64_t(1) << 31) || Cout >= (int64_t(1) << 31)) return "";
+    FwdParams p{};
+    p.values = reinterpret_cast<const void *>(uintptr_t(256));
+    p.idx = reinterpret_cast<const uint8_t *>(uintptr_t(256));
+    p.R = R;
+    p.G = G;
+    p.K = K;
+    if (!gemm_pk_shape_ok(p)) return "";
+    // activations copied by TMA: any product; a convolution (other than 1x1 with
+    // unit stride, which is a product) when Cin is a multiple of the 64-deep stage
+    if (R != Cin && Cin % 64 != 0) return "";
+    int i = 0;
+    for (int g = 4; g <= 32; g *= 2)
+        for (int k = 1; k <= g / 2 && k <= 8; k *= 2, ++i)
+            if (g == G && k == K) return names[i];
+    return "";
+}
+
+}  // namespace
+
 const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cout, int G, int K, cci_algo algo)
 {
     if (!valid_dtype(dtype) || Cin < 1 || R < Cin || check_group(Cout, G, K) != CCI_OK) return "";
@@ -554,19 +647,14 @@ const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cou
                 if (g == G && k == K) return dtype == CCI_F32 ? names_tf[i] : names_ws[i];
         return "";
     }
-    if (algo == CCI_ALGO_DENSE_TC) {
-        if (dtype != CCI_BF16) return "";
-        static const char *names[] = {"dense_tc_bf16_G4_K1", "dense_tc_bf16_G4_K2", "dense_tc_bf16_G8_K1",
-                                      "dense_tc_bf16_G8_K2", "dense_tc_bf16_G8_K4", "dense_tc_bf16_G16_K1",
-                                      "dense_tc_bf16_G16_K2", "dense_tc_bf16_G16_K4", "dense_tc_bf16_G16_K8",
-                                      "dense_tc_bf16_G32_K1", "dense_tc_bf16_G32_K2", "dense_tc_bf16_G32_K4",
-                                      "dense_tc_bf16_G32_K8", "dense_tc_bf16_G32_K16"};
-        if (!dense_tc_shape_ok(dtype, G, K, Cin, R)) return "";
-        int i = 0;
-        for (int g = 4; g <= 32; g *= 2)
-            for (int k = 1; k <= g / 2; k *= 2, ++i)
-                if (g == G && k == K) return names[i];
-        return "";
+    const char *fused = fused_name(dtype, Cin, R, Cout, G, K);
+    if (algo == CCI_ALGO_DENSE_TC) return fused;
+    if (algo == CCI_ALGO_AUTO) {
+        // the family AUTO runs when given the workspace cci_workspace_size asks for
+        if (fused[0] && auto_prefers_fused(K)) return fused;
+        const char *ws = cci_kernel_name(dtype, Cin, R, Cout, G, K, CCI_ALGO_DENSE_TC_WS);
+        if (ws[0]) return ws;
+        if (fused[0]) return fused;
     }
     if (algo == CCI_ALGO_AUTO || algo == CCI_ALGO_REGTILE || algo == CCI_ALGO_EXPAND) {
         const bool expand = algo == CCI_ALGO_EXPAND || (algo == CCI_ALGO_AUTO && auto_prefers_expand(dtype, G, K));
@@ -702,6 +790,14 @@ extern "C" cci_status cci_linear_host(const void *X_host, cci_dtype dtype, int64
     if (N == 0) return CCI_OK;
 
     const cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+    // the fused family multiplies every chunk from the packed weights (no
+    // decompression); otherwise the first chunk decompresses into the workspace
+    // and every chunk runs the workspace GEMM
+    FwdParams probe = linear_params(device_buffer, 1, Cin, values, idx, Cout, static_cast<float *>(device_buffer),
+                                    dev_status);
+    probe.G = G;
+    probe.K = K;
+    const bool fused = auto_prefers_fused(K) && fused_may(probe, dtype) && gemm_pk_supported(probe);
     const cudaStream_t si = copy_in_stream ? reinterpret_cast<cudaStream_t>(copy_in_stream) : cs;
     const cudaStream_t so = copy_out_stream ? reinterpret_cast<cudaStream_t>(copy_out_stream) : cs;
     // events: [0] the call's start on `stream`; per slot k: chunk in (1 + k),
@@ -746,7 +842,11 @@ extern "C" cci_status cci_linear_host(const void *X_host, cci_dtype dtype, int64
         result = to_status(e);
         if (result != CCI_OK) break;
         FwdParams p = linear_params(xd, nc, Cin, values, idx, Cout, yd, dev_status);
-        if (c == 0) {
+        p.G = G;
+        p.K = K;
+        if (fused) {
+            result = to_status(launch_gemm_pk(p, cs));
+        } else if (c == 0) {
             // the first chunk decompresses the weights into the workspace
             result = forward(p, dtype, G, K, CCI_ALGO_DENSE_TC_WS, ws, l.ws, cs);
         } else {

@@ -90,12 +90,120 @@ __global__ void __launch_bounds__(128) pack_reg_kernel(const TB *__restrict__ W,
     }
 }
 
+// Vector form of the register kernel: each thread ranks four consecutive
+// columns r0 .. r0 + 3 of one group, its G rows loaded as one 8-byte (bf16) or
+// 16-byte (fp32) vector each; the group is the block's y index, so no thread
+// divides.  The K kept (value, index) pairs of a column are gathered in 64-bit
+// registers (slot s at bit s * element width) and the four columns' outputs,
+// contiguous in the packed arrays, are written with 16-byte stores.  Needs
+// R % 4 == 0, W, values and idx 16-byte aligned, Cout / G <= 65535 and
+// K * element bits <= 64 with 4 K elements a multiple of 16 bytes (bf16: K in
+// {2, 4}; fp32: K in {1, 2}).
+template <typename TB, int GT, int KT>
+__global__ void __launch_bounds__(128) pack_vec_kernel(const TB *__restrict__ W, int64_t R, TB *__restrict__ values,
+                                                       uint8_t *__restrict__ idx, uint32_t *status)
+{
+    constexpr uint32_t kAbs = sizeof(TB) == 4 ? 0x7fffffffu : 0x7fffu;
+    constexpr uint32_t kInf = sizeof(TB) == 4 ? 0x7f800000u : 0x7f80u;
+    constexpr int kBits = 8 * sizeof(TB);
+    const int64_t gi = blockIdx.y;
+    const int64_t r0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 4;
+    if (r0 >= R) return;
+    const TB *col = W + gi * GT * R + r0;
+    TB w[GT][4];
+#pragma unroll
+    for (int j = 0; j < GT; ++j) {
+        if constexpr (sizeof(TB) == 4) {
+            const uint4 x = __ldg(reinterpret_cast<const uint4 *>(col + static_cast<int64_t>(j) * R));
+            w[j][0] = x.x;
+            w[j][1] = x.y;
+            w[j][2] = x.z;
+            w[j][3] = x.w;
+        } else {
+            const uint2 x = __ldg(reinterpret_cast<const uint2 *>(col + static_cast<int64_t>(j) * R));
+            w[j][0] = static_cast<TB>(x.x);
+            w[j][1] = static_cast<TB>(x.x >> 16);
+            w[j][2] = static_cast<TB>(x.y);
+            w[j][3] = static_cast<TB>(x.y >> 16);
+        }
+    }
+    bool nan = false;
+    uint64_t ov[4], oi[4];  // per column: kept values and indices, slot s at s * width
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+        uint32_t a[GT];
+#pragma unroll
+        for (int j = 0; j < GT; ++j) a[j] = static_cast<uint32_t>(w[j][v]) & kAbs;
+        uint64_t vv = 0, ii = 0;
+        int sh = 0;  // slot * 8 bits
+#pragma unroll
+        for (int j = 0; j < GT; ++j) {
+            nan |= a[j] > kInf;
+            int rank = 0;  // entries ranked ahead of j: larger |w|, or equal |w| at a lower index
+#pragma unroll
+            for (int j2 = 0; j2 < GT; ++j2)
+                rank += j2 < j ? (a[j2] >= a[j]) : (a[j2] > a[j]);
+            if (rank < KT) {
+                vv |= static_cast<uint64_t>(w[j][v]) << (sh * (kBits / 8));
+                ii |= static_cast<uint64_t>(j) << sh;
+                sh += 8;
+            }
+        }
+        ov[v] = vv;
+        oi[v] = ii;
+    }
+    // values of the four columns: 4 K elements from (gi * R + r0) * K on
+    const int64_t t0 = (gi * R + r0) * KT;
+    constexpr int kVB = KT * kBits;  // bits of one column's values (32 or 64)
+    uint4 *pv = reinterpret_cast<uint4 *>(values + t0);
+    if constexpr (kVB == 32) {
+        pv[0] = make_uint4(static_cast<uint32_t>(ov[0]), static_cast<uint32_t>(ov[1]), static_cast<uint32_t>(ov[2]),
+                           static_cast<uint32_t>(ov[3]));
+    } else {
+        pv[0] = make_uint4(static_cast<uint32_t>(ov[0]), static_cast<uint32_t>(ov[0] >> 32),
+                           static_cast<uint32_t>(ov[1]), static_cast<uint32_t>(ov[1] >> 32));
+        pv[1] = make_uint4(static_cast<uint32_t>(ov[2]), static_cast<uint32_t>(ov[2] >> 32),
+                           static_cast<uint32_t>(ov[3]), static_cast<uint32_t>(ov[3] >> 32));
+    }
+    // indices: 4 K bytes
+    if constexpr (KT == 1) {
+        *reinterpret_cast<uint32_t *>(idx + t0) = static_cast<uint32_t>(oi[0] | (oi[1] << 8) | (oi[2] << 16) | (oi[3] << 24));
+    } else if constexpr (KT == 2) {
+        *reinterpret_cast<uint2 *>(idx + t0) = make_uint2(static_cast<uint32_t>(oi[0] | (oi[1] << 16)),
+                                                          static_cast<uint32_t>(oi[2] | (oi[3] << 16)));
+    } else {
+        *reinterpret_cast<uint4 *>(idx + t0) = make_uint4(static_cast<uint32_t>(oi[0]), static_cast<uint32_t>(oi[1]),
+                                                          static_cast<uint32_t>(oi[2]), static_cast<uint32_t>(oi[3]));
+    }
+    if (nan) report(status, CCI_ERR_VALUE);
+}
+
 template <typename TB>
 cudaError_t launch_pack_t(const TB *W, int64_t Cout, int64_t R, int G, int K, TB *values, uint8_t *idx,
                           uint32_t *status, cudaStream_t stream)
 {
     const int64_t total = (Cout / G) * R;
     const bool reg = G == 2 || G == 4 || G == 8 || G == 16 || G == 32;
+    const bool vec_k = sizeof(TB) == 2 ? (K == 2 || K == 4) : (K == 1 || K == 2);
+    const bool vec_g = (G == 4 && K <= 2) || (G == 8 && K <= 4) || (G == 16 && K <= 4) || (G == 32 && K <= 4);
+    if (vec_k && vec_g && R % 4 == 0 && Cout / G <= 65535 && reinterpret_cast<uintptr_t>(W) % 16 == 0 &&
+        reinterpret_cast<uintptr_t>(values) % 16 == 0 && reinterpret_cast<uintptr_t>(idx) % 16 == 0 &&
+        (R / 4 + 127) / 128 <= 0x7fffffff) {
+        const dim3 grid(static_cast<unsigned>((R / 4 + 127) / 128), static_cast<unsigned>(Cout / G));
+#define CCI_PACK_VEC(g, k)                                                                          \
+    if (G == g && K == k) {                                                                         \
+        pack_vec_kernel<TB, g, k><<<grid, 128, 0, stream>>>(W, R, values, idx, status);            \
+        return cudaGetLastError();                                                                  \
+    }
+        if constexpr (sizeof(TB) == 2) {
+            CCI_PACK_VEC(4, 2) CCI_PACK_VEC(8, 2) CCI_PACK_VEC(8, 4) CCI_PACK_VEC(16, 2) CCI_PACK_VEC(16, 4)
+            CCI_PACK_VEC(32, 2) CCI_PACK_VEC(32, 4)
+        } else {
+            CCI_PACK_VEC(4, 1) CCI_PACK_VEC(4, 2) CCI_PACK_VEC(8, 1) CCI_PACK_VEC(8, 2) CCI_PACK_VEC(16, 1)
+            CCI_PACK_VEC(16, 2) CCI_PACK_VEC(32, 1) CCI_PACK_VEC(32, 2)
+        }
+#undef CCI_PACK_VEC
+    }
     const int threads = reg ? 128 : 256;
     const int64_t blocks = (total + threads - 1) / threads;
     const int grid = static_cast<int>(blocks < 65536 * 16 ? blocks : 65536 * 16);

@@ -32,11 +32,20 @@
 //   split each row into hi and lo and store both in tensor memory (per stage 64
 //   columns after the accumulators), from where the MMAs read A: the three
 //   passes then read only B from shared memory.
+// Weights (the template's PK):
+//   PK = false  the dense workspace planes written by the one-pass decompression;
+//   PK = true   the packed (value, index) pairs themselves (bf16 only, no
+//               workspace): the producer warps load the K-slot runs of their
+//               groups from global memory two stages ahead (into registers),
+//               expand them into rows (Alg. 2's index: each pair goes to row
+//               G*i + Idx of its group), 8 rows x 8 indices per thread, and once
+//               the stage is free store the rows into its swizzled B tile.
 // Output: fp32 Y written by TMA stores from a swizzled staging buffer (two
 // alternating 16 KB buffers of [128 rows][32 columns]), 2-D over Y[N][Cout] or,
 // for kA4d, 4-D over Y[B][P][Q][Cout] with the tile's pixel box.
 // Roles: warps 0-3 epilogue (TMEM lanes), warps 4-7 producers of the activation
-// planes that are not copied by TMA, warp 8 allocates TMEM and issues the MMAs,
+// planes that are not copied by TMA (PK: of the weight tiles), warp 8
+// allocates TMEM and issues the MMAs,
 // warps 9.. issue the TMA copies as soon as a stage is free (so copy latency
 // overlaps the producers' work), stage by stage in turn: the copies one thread
 // issues are processed one box after another (measured on GB300: about 0.5 us
@@ -48,6 +57,8 @@
 
 #include <cuda.h>
 #include <cudaTypedefs.h>
+
+#include <type_traits>
 
 #include "cci_tc_common.cuh"
 
@@ -82,10 +93,12 @@ struct AMaps {
 // EPI = 2: a second epilogue group (warps 4-7, idle when bf16 activations are
 // copied by TMA) and two staging buffers per group, for layers whose tiles have
 // few stages (the output write dominates); EPI = 1: one group, more stages
-template <bool TF32, int ASRC, int BN, int CG, int EPI>
+template <bool TF32, int ASRC, int BN, int CG, int EPI, bool PK = false>
 struct Cfg {
     static constexpr int kM = 128, kN = BN;
     static_assert(CG == 1 || (CG == 2 && !TF32 && ASRC != kAGather), "pair mode: bf16 with TMA activations");
+    static_assert(!PK || (!TF32 && ASRC != kAGather && EPI == 1 && (BN / CG) <= 128),
+                  "packed weights: bf16, TMA activations, producers busy, one item per producer");
     static constexpr int kBRows = kN / CG;  // B rows held by one CTA
     static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
@@ -99,6 +112,7 @@ struct Cfg {
     static constexpr int kBPlane = kBRows * 128;
     static constexpr int kBOff = kHalo ? 0 : kAPlanes * kAPlane;  // B planes within a stage
     static constexpr int kStage = kBOff + kBPlanes * kBPlane;
+    static_assert(kStage % 1024 == 0, "stages must keep the 1024-byte swizzle alignment");
     // halo copies: fewer weight stages, the rest of shared memory for a ring of
     // halo buffers whose size and count the host sets per layer (ConvBox)
     static constexpr int kHaloStages = kBPlane <= 8192 ? 6 : (kBPlane <= 16384 ? 4 : 3);
@@ -334,6 +348,204 @@ __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
 }
 
 
+// ---- expansion of packed weights into a B tile (PK) ----
+// One producer thread builds an item: 8 consecutive B rows (output channels
+// co0 + m0 .. + 7) x 8 consecutive reduction indices (one 16-byte chunk of each
+// row).  Its inputs are the K-slot runs of the item's group(s) over those 8
+// indices, loaded from the packed arrays ([r][slot]: values bf16, indices
+// uint8) into registers.  Rows are built two indices (one 32-bit word: a bf16 pair) at
+// a time: for r-pair p and slot s, the pair's two values are ANDed with a mask
+// that is 0xffff in each half whose index names the row, and ORed into the row's
+// word.  The masks come from one byte permute per row: the permute's selector
+// nibbles are the two indices (each twice), its 8 source bytes the row table
+// (byte jj = 0xff for row jj, else 0), so byte k of the result is 0xff exactly
+// when the index of half k / 2 equals the row.
+namespace pk {
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
+{
+    uint32_t r;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+    return r;
+}
+
+// row table of row jj of the 8-row item: source bytes 0-3 (lo) and 4-7 (hi)
+__device__ __forceinline__ constexpr uint32_t row_lo(int jj) { return jj < 4 ? 0xffu << (8 * jj) : 0u; }
+__device__ __forceinline__ constexpr uint32_t row_hi(int jj) { return jj >= 4 ? 0xffu << (8 * (jj - 4)) : 0u; }
+
+// values of slot s at r = 2p (low half) and 2p + 1 (high half); vw holds the
+// item's K-slot runs, v[r][s] at bf16 position r * K + s
+template <int K>
+__device__ __forceinline__ uint32_t val_pair(const uint32_t *vw, int p, int s)
+{
+    if constexpr (K == 1) {
+        return vw[p];
+    } else {
+        const int e0 = 2 * p * K + s, e1 = (2 * p + 1) * K + s;  // bf16 positions
+        return prmt(vw[e0 >> 1], vw[e1 >> 1], (e0 & 1 ? 0x32u : 0x10u) | (e1 & 1 ? 0x7600u : 0x5400u));
+    }
+}
+
+// indices of slot s at r = 2p (byte 0) and 2p + 1 (byte 1); bytes 2 and 3 are
+// not used by the callers
+template <int K>
+__device__ __forceinline__ uint32_t idx_pair(const uint32_t *iw, int p, int s)
+{
+    const int b0 = 2 * p * K + s, b1 = (2 * p + 1) * K + s;
+    if ((b0 >> 2) == (b1 >> 2)) return prmt(iw[b0 >> 2], 0u, static_cast<uint32_t>((b0 & 3) | ((b1 & 3) << 4)) | 0x4400u);
+    return prmt(iw[b0 >> 2], iw[b1 >> 2], static_cast<uint32_t>((b0 & 3) | ((4 + (b1 & 3)) << 4)) | 0x4400u);
+}
+
+// adds one group's K slots to the item's rows.  MODE 0: indices are rows (G = 8,
+// or the first group of a G = 4 item); MODE 1: rows are index + 4 (the second
+// group of a G = 4 item); MODE 2: G >= 16, the item covers rows j0 .. j0 + 7 of
+// its group (J = j0 * 0x0101) and slots whose index lies outside add nothing.
+// INIT: the first group of the item (rows start from its contributions).
+template <int K, int MODE, bool INIT>
+__device__ __forceinline__ void expand_group(uint32_t (&out)[8][4], const uint32_t *vw, const uint32_t *iw, uint32_t J)
+{
+#pragma unroll
+    for (int pr = 0; pr < 4; ++pr) {
+#pragma unroll
+        for (int s = 0; s < K; ++s) {
+            uint32_t v = val_pair<K>(vw, pr, s);
+            const uint32_t u = idx_pair<K>(iw, pr, s);
+            uint32_t sel;
+            if constexpr (MODE == 2) {
+                const uint32_t x = u ^ J;  // in the block: x < 8 (j0 is a multiple of 8, index < 32)
+                sel = (x & 0x0707u) * 0x11u;
+                // halves outside the block: 0xffff (sign of byte + 0x7f), value cleared
+                v &= ~prmt((x & 0x1818u) + 0x7f7fu, 0u, 0x9988u);
+            } else {
+                sel = (MODE == 1 ? u + 0x0404u : u) * 0x11u;  // nibbles (i0, i0, i1, i1)
+            }
+#pragma unroll
+            for (int jj = 0; jj < 8; ++jj) {
+                const uint32_t m = prmt(row_lo(jj), row_hi(jj), sel);
+                if (INIT && s == 0)
+                    out[jj][pr] = v & m;
+                else
+                    out[jj][pr] |= v & m;
+            }
+        }
+    }
+}
+
+// true if an index set of the group at one of the item's first nr reduction
+// indices is not strictly increasing or has an index >= G (cci_pack never
+// writes such sets)
+template <int K>
+__device__ __forceinline__ bool bad_sets(const uint32_t *iw, int G, int nr)
+{
+    bool bad = false;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+        if (r >= nr) break;
+        int prev = -1;
+#pragma unroll
+        for (int s = 0; s < K; ++s) {
+            const int b = r * K + s;
+            const int j = static_cast<int>((iw[b >> 2] >> (8 * (b & 3))) & 0xffu);
+            bad |= j >= G || j <= prev;
+            prev = j;
+        }
+    }
+    return bad;
+}
+
+// the K-slot runs of an item's group(s) at its 8 reduction indices, in
+// registers: NG groups (2 for G = 4, whose items span two groups), per group
+// 4K words of values (v[r][s] at bf16 position r*K + s) and 2K words of indices
+template <int K>
+struct Runs {
+    static constexpr int NG = K <= 2 ? 2 : 1;
+    uint32_t v[NG][4 * K];
+    uint32_t i[NG][2 * K];
+};
+
+// global loads of one group's runs at reduction indices r .. r + 7: 16 K bytes
+// of values and 8 K bytes of indices from offset (g*R + r)*K of the packed
+// arrays (16-byte aligned: R % 8 == 0, r % 8 == 0); zeros for a group past the
+// last one or indices past R (R % 8 == 0, so a chunk is wholly inside or out)
+template <int K>
+__device__ __forceinline__ void load_group(uint32_t (&v)[4 * K], uint32_t (&iw)[2 * K], const uint16_t *V,
+                                           const uint8_t *I, int64_t g, int64_t groups, int64_t r, int64_t R)
+{
+    if (g < groups && r < R) {
+        const int64_t off = (g * R + r) * K;
+        const uint4 *pv = reinterpret_cast<const uint4 *>(V + off);
+#pragma unroll
+        for (int q = 0; q < K; ++q) {
+            const uint4 x = __ldg(pv + q);
+            v[4 * q] = x.x;
+            v[4 * q + 1] = x.y;
+            v[4 * q + 2] = x.z;
+            v[4 * q + 3] = x.w;
+        }
+        if constexpr (K == 1) {
+            const uint2 x = __ldg(reinterpret_cast<const uint2 *>(I + off));
+            iw[0] = x.x;
+            iw[1] = x.y;
+        } else {
+            const uint4 *pi = reinterpret_cast<const uint4 *>(I + off);
+#pragma unroll
+            for (int q = 0; q < K / 2; ++q) {
+                const uint4 x = __ldg(pi + q);
+                iw[4 * q] = x.x;
+                iw[4 * q + 1] = x.y;
+                iw[4 * q + 2] = x.z;
+                iw[4 * q + 3] = x.w;
+            }
+        }
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4 * K; ++q) v[q] = 0u;
+#pragma unroll
+        for (int q = 0; q < 2 * K; ++q) iw[q] = 0u;  // index 0 with value 0: adds nothing
+    }
+}
+
+// the runs of the item whose first row is in group g (rows of groups g and g + 1
+// for G = 4) at reduction indices r .. r + 7
+template <int K>
+__device__ __forceinline__ void load_item(Runs<K> &run, const FwdParams &p, int64_t g, int64_t r, int64_t groups)
+{
+    const uint16_t *V = static_cast<const uint16_t *>(p.values);
+    if constexpr (Runs<K>::NG == 2) {
+        if (p.G == 4) {
+            load_group<K>(run.v[0], run.i[0], V, p.idx, g, groups, r, p.R);
+            load_group<K>(run.v[1], run.i[1], V, p.idx, g + 1, groups, r, p.R);
+            return;
+        }
+    }
+    load_group<K>(run.v[0], run.i[0], V, p.idx, g, groups, r, p.R);
+}
+
+// the item's 8 rows of 8 bf16 (4 words each) from its runs (group g, first row
+// j0 of the group); chk: check the index sets of its group(s) at the first nr
+// indices (bad set on a bad one)
+template <int K>
+__device__ __forceinline__ void expand_item(uint32_t (&out)[8][4], const Runs<K> &run, int G, int64_t g, int j0,
+                                            int64_t groups, int nr, bool chk, bool &bad)
+{
+    if constexpr (Runs<K>::NG == 2) {
+        if (G == 4) {
+            if (chk && g < groups) bad |= bad_sets<K>(run.i[0], G, nr);
+            if (chk && g + 1 < groups) bad |= bad_sets<K>(run.i[1], G, nr);
+            expand_group<K, 0, true>(out, run.v[0], run.i[0], 0u);
+            expand_group<K, 1, false>(out, run.v[1], run.i[1], 0u);
+            return;
+        }
+    }
+    if (chk && j0 == 0 && g < groups) bad |= bad_sets<K>(run.i[0], G, nr);
+    if (G == 8)
+        expand_group<K, 0, true>(out, run.v[0], run.i[0], 0u);
+    else
+        expand_group<K, 2, true>(out, run.v[0], run.i[0], static_cast<uint32_t>(j0) * 0x0101u);
+}
+
+}  // namespace pk
+
 // (box along q, box along p, batch box) of M tile mt
 struct BoxIdx {
     int qb, pb;
@@ -349,13 +561,15 @@ __device__ __forceinline__ BoxIdx box_of(int64_t mt, const ConvBox &box)
     return i;
 }
 
-template <bool TF32, int ASRC, int BN, int CG, int EPI>
-__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
+// PK: tmB0 / tmB1 are the maps of the packed values and indices (2-D over
+// [Cout/G][R*K]); otherwise the maps of the workspace planes
+template <bool TF32, int ASRC, int BN, int CG, int EPI, bool PK = false>
+__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
     gemm_ws_kernel(FwdParams p, const __grid_constant__ AMaps tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmY, ConvBox box,
                    int64_t n_ct, int64_t n_tiles)
 {
-    using C = Cfg<TF32, ASRC, BN, CG, EPI>;
+    using C = Cfg<TF32, ASRC, BN, CG, EPI, PK>;
     constexpr int kM = C::kM, kN = C::kN, kKS = C::kKS, kStages = C::kStages;
     constexpr int kLag = 2;  // bf16 gather: stages in flight before a producer's arrive
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -384,8 +598,12 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
     };
 
     if (tid == 0) {
+        // full[s]: the copy issuer's expect_tx arrival (none for PK halo stages) and
+        // PK: one arrival per producer group of the pair (elected after their
+        // writes), else 128 producer arrivals when the producers fill the stage
+        const uint32_t full_count = PK ? (C::kHalo ? 0u : 1u) + CG : (C::kATma ? 1u : 129u);
         for (int s = 0; s < kStages; ++s) {
-            tc::mbar_init(&S->full[s], C::kATma ? 1 : 129);
+            tc::mbar_init(&S->full[s], full_count);
             tc::mbar_init(&S->empty[s], 1);
             tc::mbar_init(&S->aux[s], 1);
         }
@@ -428,7 +646,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
         if constexpr (ASRC == kA4d)
             for (int i = 0; i < p.sh * p.sw; ++i) tc::tma_prefetch_desc(&tmA.m[i]);
         if constexpr (ASRC == kAHalo) tc::tma_prefetch_desc(&tmA.m[0]);
-        tc::tma_prefetch_desc(&tmB0);
+        if constexpr (!PK) tc::tma_prefetch_desc(&tmB0);
         if constexpr (C::kBPlanes > 1) tc::tma_prefetch_desc(&tmB1);
         tc::tma_prefetch_desc(&tmY);
     }
@@ -476,7 +694,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                     __syncwarp();
                 }
             }
-        } else
+        } else if (!(PK && C::kHalo))  // PK halo stages hold only the producers' weight tiles
         for (int64_t u = u0; u < n_tiles && ok; u += ustep) {
             int64_t mt, ct;
             split_unit(u, mt, ct);
@@ -500,12 +718,17 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                 }
                 if (lane == 0 && CG == 2) {
                     // both CTAs' copies complete on the even CTA's full barrier, which
-                    // expects the bytes of the pair
+                    // expects the bytes of the pair (PK: the activations only; each
+                    // CTA's packed runs land on its own aux barrier)
                     const uint32_t st = base + s * C::kStage;
                     const uint32_t bst = st + C::kAPlane;
                     const uint32_t fb = map_to_rank(tc::smem_u32(&S->full[s]), 0);
-                    if (crank == 0) tc::mbar_arrive_expect_tx(&S->full[s], 2 * (C::kBBytes + a_bytes));
-                    tma_load_2d_pair(bst, &tmB0, ks * kKS, static_cast<int>(co0), fb);
+                    if constexpr (PK) {
+                        if (crank == 0) tc::mbar_arrive_expect_tx(&S->full[s], 2 * a_bytes);
+                    } else {
+                        if (crank == 0) tc::mbar_arrive_expect_tx(&S->full[s], 2 * (C::kBBytes + a_bytes));
+                        tma_load_2d_pair(bst, &tmB0, ks * kKS, static_cast<int>(co0), fb);
+                    }
                     if constexpr (ASRC == kA2d) {
                         tma_load_2d_pair(st, &tmA.m[0], ks * kKS, static_cast<int>(mt * kM), fb);
                     } else {
@@ -524,10 +747,14 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                     // the activation copy completes on aux (raw fp32, split afterwards) or full
                     uint64_t *abar = C::kARaw ? &S->aux[s] : &S->full[s];
                     if constexpr (C::kARaw) tc::mbar_arrive_expect_tx(abar, a_bytes);
-                    tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes + (C::kATma ? a_bytes : 0u));
-                    tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
-                    if constexpr (C::kBPlanes > 1)
-                        tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                    if constexpr (PK) {
+                        tc::mbar_arrive_expect_tx(&S->full[s], a_bytes);
+                    } else {
+                        tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes + (C::kATma ? a_bytes : 0u));
+                        tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                        if constexpr (C::kBPlanes > 1)
+                            tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                    }
                     if constexpr (ASRC == kA2d) {
                         tc::tma_load_2d(st, &tmA.m[0], ks * kKS, static_cast<int>(mt * kM), abar);
                     } else if constexpr (ASRC == kA4d) {
@@ -545,6 +772,120 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
                 __syncwarp();
             }
         }
+    } else if (PK && warp >= 4 && warp < 8) {
+        // ------------------------------------------------------------ weight producers (PK)
+        // thread pt builds item pt of every stage: rows 8 (pt / 8) .. + 7 of this
+        // CTA's B tile, reduction indices 8 (pt % 8) .. + 7 of the stage.  Its runs
+        // are loaded NB stages ahead into a ring of NB register sets (a set is
+        // refilled right after it is expanded), expanded into rows while the stage
+        // may still be in use, and stored once the stage's MMAs released it.
+        const int pt = tid - 128;
+        const int m0 = (pt >> 3) * 8, c = pt & 7;
+        const bool active = m0 < C::kBRows;
+        const int64_t groups = p.Cout / p.G;
+        const int lg = 31 - __clz(p.G);  // G is a power of two
+        const uint32_t full_remote = CG == 2 ? map_to_rank(tc::smem_u32(&S->full[0]), 0) : 0u;
+        bool bad = false;
+        // a stage of this CTA, in the MMAs' order, and the item's place in it: the
+        // output channel of its first row, its group, the reduction index of its
+        // first column, whether its tile checks index sets (the first M tile, or
+        // pair, of each N tile).  Advanced stage by stage without division (one
+        // per tile).
+        struct Cursor {
+            int64_t u, co, g, r;
+            int ks, t, ch, j0;
+            bool chk;
+        };
+        auto tile_start = [&](Cursor &q) {
+            if (q.u >= n_tiles) return;
+            int64_t mt, ct;
+            split_unit(q.u, mt, ct);
+            q.co = ct * kN + crank * C::kBRows + m0;
+            q.g = q.co >> lg;
+            q.j0 = static_cast<int>(q.co & (p.G - 1));
+            q.chk = mt < CG;
+            q.ks = q.t = q.ch = 0;
+            q.r = 8 * c;
+        };
+        auto advance = [&](Cursor &q) {
+            if (++q.ks == nks) {
+                q.u += ustep;
+                tile_start(q);
+                return;
+            }
+            if constexpr (ASRC == kAHalo) {  // stages chunk by chunk, the taps of a chunk in turn
+                if (++q.t == taps) {
+                    q.t = 0;
+                    ++q.ch;
+                }
+                q.r = static_cast<int64_t>(q.t) * p.Cin + q.ch * 64 + 8 * c;
+            } else {
+                q.r += 64;
+            }
+        };
+        auto run_k = [&](auto kc) {
+            constexpr int K = decltype(kc)::value;
+            constexpr int NB = K <= 4 ? 2 : 1;
+            pk::Runs<K> ring[NB];
+            Cursor cur{u0, 0, 0, 0, 0, 0, 0, 0, false};  // the stage being built
+            tile_start(cur);
+            Cursor pre = cur;  // the stage whose runs are loaded next (NB ahead)
+            auto load = [&](pk::Runs<K> &rg) {
+                if (active && pre.u < n_tiles) pk::load_item<K>(rg, p, pre.g, pre.r, groups);
+                advance(pre);
+            };
+#pragma unroll
+            for (int q = 0; q < NB; ++q) load(ring[q]);
+            bool ok = true;
+            int s = 0;               // stage of the ring
+            uint32_t eph = 0;        // parity of the empty-barrier phase to wait for
+            bool wrapped = false;    // every stage used once already
+            while (ok && cur.u < n_tiles) {
+#pragma unroll
+                for (int q = 0; q < NB; ++q) {
+                    if (!ok || cur.u >= n_tiles) break;
+                    uint32_t out[8][4];
+                    if (active) {
+                        const int64_t left = p.R - cur.r;
+                        const int nr = left <= 0 ? 0 : (left >= 8 ? 8 : static_cast<int>(left));
+                        pk::expand_item<K>(out, ring[q], p.G, cur.g, cur.j0, groups, nr, cur.chk, bad);
+                    }
+                    load(ring[q]);
+                    if (wrapped) ok = tc::mbar_wait(&S->empty[s], eph, abort, p.status);
+                    if (ok && active) {
+                        const uint32_t bst = base + s * C::kStage + C::kBOff;
+#pragma unroll
+                        for (int jj = 0; jj < 8; ++jj)
+                            st_shared_v4(bst + sw_chunk(m0 + jj, c), out[jj][0], out[jj][1], out[jj][2], out[jj][3]);
+                    }
+                    // the tile's writes are visible to the MMAs (async proxy) once one
+                    // thread of the group arrives after all of them (pair: on the even
+                    // CTA's barrier, released at cluster scope)
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    ok = tc::named_and(3, 128, ok);
+                    if (!ok) break;
+                    if (pt == 0) {
+                        if (CG == 2 && crank != 0)
+                            mbar_arrive_remote(full_remote + static_cast<uint32_t>(s * sizeof(uint64_t)));
+                        else
+                            tc::mbar_arrive(&S->full[s]);
+                    }
+                    advance(cur);
+                    if (++s == kStages) {
+                        s = 0;
+                        eph ^= wrapped ? 1u : 0u;
+                        wrapped = true;
+                    }
+                }
+            }
+        };
+        switch (p.K) {
+            case 1: run_k(std::integral_constant<int, 1>{}); break;
+            case 2: run_k(std::integral_constant<int, 2>{}); break;
+            case 4: run_k(std::integral_constant<int, 4>{}); break;
+            default: run_k(std::integral_constant<int, 8>{}); break;
+        }
+        if (bad) report(p.status, CCI_ERR_INDEX);
     } else if (warp >= 4 && warp < 8 && C::kEG == 1) {
         // ------------------------------------------------------------ producers
         const int pt = tid - 128;
@@ -812,7 +1153,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI>::kThreads, 1)
             } else
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
                 const int s = it % kStages;
-                ok = tc::mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
+                // PK pairs: the phase includes the odd CTA's producers (released at cluster scope)
+                ok = tc::mbar_wait<PK && CG == 2>(&S->full[s], (it / kStages) & 1, abort, p.status);
                 if (!ok) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 if (lane == 0) {
@@ -975,9 +1317,10 @@ inline PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
 
 // map over `rank` dims (dims[0] innermost, element counts) with byte strides
 // strides[i] of dims 1.., box[] elements per dim, 128-byte swizzle (box[0] * elem
-// must be 128); false if the driver rejects it
+// must be 128) unless `swizzle` is false (box[0] * elem a multiple of 16); false
+// if the driver rejects it
 inline bool make_map_strided(CUtensorMap *m, const void *ptr, CUtensorMapDataType dt, int rank,
-                             const int64_t *dims, const int64_t *strides, const int *box)
+                             const int64_t *dims, const int64_t *strides, const int *box, bool swizzle = true)
 {
     auto fn = encode_fn();
     if (!fn || rank < 1 || rank > 5) return false;
@@ -991,8 +1334,8 @@ inline bool make_map_strided(CUtensorMap *m, const void *ptr, CUtensorMapDataTyp
         if (i > 0) gs[i - 1] = static_cast<cuuint64_t>(strides[i - 1]);
     }
     return fn(m, dt, static_cast<cuuint32_t>(rank), const_cast<void *>(ptr), gd, gs, bx, es,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // the same over a packed row-major array
@@ -1105,11 +1448,11 @@ inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn, int cg = 1)
     return best;
 }
 
-template <bool TF32, int ASRC, int BN, int CG, int EPI = 1>
+template <bool TF32, int ASRC, int BN, int CG, int EPI = 1, bool PK = false>
 cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &tmA, cudaStream_t stream)
 {
-    using C = Cfg<TF32, ASRC, BN, CG, EPI>;
-    auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG, EPI>;
+    using C = Cfg<TF32, ASRC, BN, CG, EPI, PK>;
+    auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG, EPI, PK>;
     ConvBox box = box_in;
     size_t smem = C::kSmem;
     if constexpr (C::kHalo) {
@@ -1120,17 +1463,17 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &t
         if (box.nh < 2) return cudaErrorInvalidValue;
         smem += static_cast<size_t>(box.nh) * hb;
     }
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-        static_cast<int>(C::kHalo ? static_cast<size_t>(kMaxSmemPerBlock) : C::kSmem));
+    static SmemAttrCache attr_cache;
+    const cudaError_t attr = smem_attr_once(
+        kern, static_cast<int>(C::kHalo ? static_cast<size_t>(kMaxSmemPerBlock) : C::kSmem), attr_cache);
     if (attr != cudaSuccess) return attr;
     CUtensorMap tmB0{}, tmB1{}, tmY{};
     const CUtensorMapDataType dt = TF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     const int elem = TF32 ? 4 : 2;
     const int64_t wdims[2] = {p.R, p.Cout};
     const int wbox[2] = {C::kKS, C::kBRows};
-    if (!make_map(&tmB0, p.wdense, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
-    if (C::kBPlanes > 1) {
+    if (!PK && !make_map(&tmB0, p.wdense, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
+    if (!PK && C::kBPlanes > 1) {
         const char *lo = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
         if (!make_map(&tmB1, lo, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
     }

@@ -21,18 +21,27 @@ cudaError_t launch_fma_probe(float *out, int blocks, int threads, int iters, cud
 // bounded-wait diagnostic (cci_dense_tc.cu): arrive = 0 lets the wait expire
 cudaError_t launch_wait_probe(uint32_t *status, int arrive, cudaStream_t stream);
 
-// dense tensor-core comparison kernel (tcgen05, bf16 only)
+// (G, K) pairs of the workspace tensor-core family
 bool dense_tc_supported(int dtype, int G, int K);
-// ws = true: decompress once into p.wdense and copy B tiles from it (bf16: dense
-// [Cout][R]; fp32: hi and lo tf32 planes [2][Cout][R], three-pass tf32 product);
-// ws = false (bf16 only): decompress each B tile in shared memory
-cudaError_t launch_dense_tc(const FwdParams &p, int dtype, int G, int K, bool ws, cudaStream_t stream);
+// decompress once into p.wdense and copy B tiles from it (bf16: dense [Cout][R];
+// fp32: hi and lo tf32 planes [2][Cout][R], three-pass tf32 product)
+cudaError_t launch_dense_tc_ws(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);
 
 // dense product on the tensor cores from the decompressed workspace p.wdense
 // (cci_gemm_ws_*.cu): bf16 dense [Cout][R], or fp32 hi / lo tf32 planes [2][Cout][R]
 cudaError_t launch_gemm_ws(const FwdParams &p, int dtype, cudaStream_t stream);
 cudaError_t launch_gemm_ws_bf16(const FwdParams &p, cudaStream_t stream);
 cudaError_t launch_gemm_ws_tf32(const FwdParams &p, cudaStream_t stream);
+
+// fused tensor-core product (cci_gemm_pk*.cu): the GEMM of the workspace family
+// with the packed weights (p.values, p.idx, p.G, p.K) expanded into each B tile
+// in shared memory; bf16 only.  gemm_pk_shape_ok: (G, K), packed-array shape and
+// alignment allow it; gemm_pk_supported: also the activations are copied by
+// TMA; launch_gemm_pk returns cudaErrorNotSupported, before any launch, for a
+// layer without it.
+bool gemm_pk_shape_ok(const FwdParams &p);
+bool gemm_pk_supported(const FwdParams &p);
+cudaError_t launch_gemm_pk(const FwdParams &p, cudaStream_t stream);
 
 // One register-tiled instantiation: (dtype, G, K) -> tile shape and launcher.
 struct RegtileEntry {

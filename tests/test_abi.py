@@ -117,10 +117,20 @@ def test_pack_rejects(lib):
 def test_algo_dense_tc_names(lib):
     import torch
     assert cci.kernel_name(torch.float32, 16, 16, 16, 8, 2, cci.ALGO_DENSE_TC) == ""  # bf16 only
-    assert cci.kernel_name(torch.bfloat16, 16, 16, 16, 8, 2, cci.ALGO_DENSE_TC) == "dense_tc_bf16_G8_K2"
-    assert cci.kernel_name(torch.bfloat16, 16, 16, 64, 32, 16, cci.ALGO_DENSE_TC) == "dense_tc_bf16_G32_K16"
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 16, 8, 2, cci.ALGO_DENSE_TC) == "dense_tc_fused_bf16_G8_K2"
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 64, 32, 8, cci.ALGO_DENSE_TC) == "dense_tc_fused_bf16_G32_K8"
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 64, 32, 16, cci.ALGO_DENSE_TC) == ""  # K = 16: no expansion
     assert cci.kernel_name(torch.bfloat16, 12, 12, 16, 8, 2, cci.ALGO_DENSE_TC) == ""  # Cin % 8
     assert cci.kernel_name(torch.bfloat16, 16, 16, 24, 8, 3, cci.ALGO_DENSE_TC) == ""  # K not a power of 2
+    assert cci.kernel_name(torch.bfloat16, 24, 24, 16, 8, 1, cci.ALGO_DENSE_TC) == ""  # R * K % 16
+    assert cci.kernel_name(torch.bfloat16, 64, 576, 64, 8, 2, cci.ALGO_DENSE_TC) == "dense_tc_fused_bf16_G8_K2"
+    assert cci.kernel_name(torch.bfloat16, 32, 288, 64, 8, 2, cci.ALGO_DENSE_TC) == ""  # conv, Cin % 64
+    # AUTO (given the workspace it asks for): a tensor-core family for these layers;
+    # the workspace one for K = 8
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 16, 8, 2) in ("dense_tc_fused_bf16_G8_K2", "dense_tc_ws_bf16_G8_K2")
+    assert cci.kernel_name(torch.bfloat16, 16, 16, 64, 32, 8) == "dense_tc_ws_bf16_G32_K8"
+    # fp32: the workspace family (three-pass tf32) with a workspace; CUDA-core kernels without one
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2) == "dense_tc_ws_tf32x3_G8_K2"
 
 
 def test_kernel_names(lib):

@@ -100,7 +100,7 @@ def test_host_product_matches_device_product(dtype, N, Cin, Cout, G, K, chunk, m
         cci.linear_host(Xh, v, i, Cout, G, K, out=Yh, status=st, chunk=chunk)
     torch.cuda.current_stream(dev).synchronize()
     assert cci.read_status(st) == 0
-    Yd = cci.linear(X.to(dev), v, i, Cout, G, K, algo=cci.ALGO_DENSE_TC_WS).cpu()
+    Yd = cci.linear(X.to(dev), v, i, Cout, G, K, algo=cci.ALGO_AUTO).cpu()
     same = Yh.view(torch.int32) == Yd.view(torch.int32)
     assert bool(same.all()), f"{int((~same).sum())} outputs differ from the device-resident product"
     _, _, Wo, mask = oracle_reference(W, G, K)
@@ -144,7 +144,7 @@ def test_host_product_bottleneck_full():
     Yh = cci.linear_host(X.pin_memory(), v, i, case.Cout, case.G, case.K, status=st, chunk=chunk)
     torch.cuda.current_stream(dev).synchronize()
     assert cci.read_status(st) == 0
-    Yd = cci.linear(X.to(dev), v, i, case.Cout, case.G, case.K, algo=cci.ALGO_DENSE_TC_WS).cpu()
+    Yd = cci.linear(X.to(dev), v, i, case.Cout, case.G, case.K, algo=cci.ALGO_AUTO).cpu()
     assert bool((Yh.view(torch.int32) == Yd.view(torch.int32)).all())
     edges = np.concatenate([np.arange(c * chunk - 2, c * chunk + 2) for c in range(1, case.N // chunk)])
     rows = np.unique(np.concatenate([sample_rows(case.N, 1024, seed=5), edges]))

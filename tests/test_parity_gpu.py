@@ -40,20 +40,24 @@ PACK_GK = [(1, 1), (2, 1), (3, 2), (4, 1), (4, 2), (4, 4), (5, 3), (8, 1), (8, 2
            (16, 4), (16, 8), (32, 4), (32, 16), (64, 5), (256, 7), (256, 256)]
 
 
+@pytest.mark.parametrize("R", [37, 40], ids=["R37", "R40_vec"])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("G,K", PACK_GK)
-def test_pack_random(dev, dtype, G, K):
-    Cout, R = 2 * G, 37
+def test_pack_random(dev, dtype, G, K, R):
+    """R = 37: the one-column-per-thread kernels; R = 40: four columns per thread
+    (vector loads) for the power-of-two G up to 32."""
+    Cout = 2 * G
     W = wl.draw_w(Cout, R, 1.0, dtype, seed=G * 100 + K).to(dev)
     v, i = cci.pack(W, G, K)
     vo, io, _, _ = oracle_reference(W, G, K)
     assert_pack_equal(v, i, vo, io)
 
 
+@pytest.mark.parametrize("R", [29, 32])
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-@pytest.mark.parametrize("G,K", [(4, 2), (8, 3), (16, 5), (3, 1)])
-def test_pack_ties_signed_zero_inf(dev, dtype, G, K):
-    Cout, R = 4 * G, 29
+@pytest.mark.parametrize("G,K", [(4, 2), (8, 3), (16, 5), (3, 1), (32, 7)])
+def test_pack_ties_signed_zero_inf(dev, dtype, G, K, R):
+    Cout = 4 * G
     W = wl.integer_valued((Cout, R), -3, 3, seed=G + K)  # many equal magnitudes
     W[0, :5] = -0.0
     W[1, 5] = float("inf")
@@ -66,8 +70,9 @@ def test_pack_ties_signed_zero_inf(dev, dtype, G, K):
     assert_pack_equal(v, i, vo, io)
 
 
-def test_pack_nan_reported(dev):
-    W = torch.randn(16, 9, device=dev)
+@pytest.mark.parametrize("R", [9, 12])
+def test_pack_nan_reported(dev, R):
+    W = torch.randn(16, R, device=dev)
     W[5, 3] = float("nan")
     with pytest.raises(cci.CCIError) as e:
         cci.pack(W, 8, 2)
@@ -392,7 +397,14 @@ DENSE_SMALL = [
 
 
 DENSE_ALGOS = [cci.ALGO_DENSE_TC, cci.ALGO_DENSE_TC_WS]
-DENSE_IDS = ["smem", "ws"]
+DENSE_IDS = ["fused", "ws"]
+
+
+def skip_without(dtype, Cin, R, Cout, G, K, algo):
+    name = cci.kernel_name(dtype, Cin, R, Cout, G, K, algo)
+    if not name:
+        pytest.skip("the family does not have this layer")
+    assert name.startswith("dense_tc")
 
 
 @pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
@@ -400,7 +412,7 @@ DENSE_IDS = ["smem", "ws"]
 def test_dense_tc_small(dev, case, algo):
     N, Cin, Cout, G, K = case
     X, W = wl.random_small(N * 3 + Cin, "bf16", N, Cin, Cout)
-    assert cci.kernel_name(BF16, Cin, Cin, Cout, G, K, algo).startswith("dense_tc")
+    skip_without(BF16, Cin, Cin, Cout, G, K, algo)
     Y = run_linear(dev, X, W, G, K, algo)
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.linear(f64(X), Wd, mask)
@@ -411,6 +423,7 @@ def test_dense_tc_small(dev, case, algo):
 @pytest.mark.parametrize("G,K", wl.SWEEP_POINTS)
 def test_dense_tc_sweep_full(dev, G, K, algo):
     case = wl.sweep_case(G, K)
+    skip_without(BF16, case.Cin, case.R, case.Cout, G, K, algo)
     X, W = wl.linear_inputs(case, device="cpu")
     Y = run_linear(dev, X, W, G, K, algo)
     assert torch.isfinite(Y).all()
@@ -426,6 +439,8 @@ def test_dense_tc_sweep_full(dev, G, K, algo):
 @pytest.mark.parametrize("algo", DENSE_ALGOS, ids=DENSE_IDS)
 def test_dense_tc_conv_small(dev, case, algo):
     B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
+    if algo == cci.ALGO_DENSE_TC and not (Cin % 64 == 0 or (KH == KW == 1 and stride == (1, 1) and pad == (0, 0))):
+        pytest.skip("fused family: activations by TMA need Cin % 64 == 0")
     g = torch.Generator().manual_seed(B * 11 + Cin)
     X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(BF16)
     W = torch.randn((Cout, KH * KW * Cin), generator=g).to(BF16)
@@ -455,9 +470,97 @@ def test_dense_tc_rejects_repeated_indices(dev, algo):
     assert cci.read_status(st) == 10
 
 
+# ---------------------------------------------------------------------------
+# the fused tensor-core family: packed weights expanded inside the GEMM
+# ---------------------------------------------------------------------------
+# (N, Cin, Cout, G, K): ragged N, Cout below a tile (64-wide N tiles, idle
+# producers), two-group items (G = 4), row blocks of larger groups (G = 16, 32),
+# K = 8, a reduction not a multiple of the 64-deep stage (R = 80, 200, 136),
+# long reductions (R up to 2048), groups past Cout in the last channel tile
+# (Cout = 320, 96); the CTA-pair tiles are covered by the sweep tests
+FUSED_SMALL = [
+    (1, 64, 64, 8, 2), (129, 80, 96, 8, 1), (300, 200, 320, 4, 2), (257, 128, 128, 4, 1),
+    (515, 192, 384, 16, 8), (100, 256, 320, 32, 4), (77, 64, 64, 32, 8), (640, 1024, 512, 8, 2),
+    (1000, 2048, 1024, 16, 4), (333, 1088, 768, 32, 1), (4096, 512, 2048, 8, 4), (130, 136, 96, 16, 2),
+]
+
+
+@pytest.mark.parametrize("case", FUSED_SMALL, ids=lambda c: "N{}_C{}x{}_G{}K{}".format(*c))
+def test_fused_small(dev, case):
+    N, Cin, Cout, G, K = case
+    skip_without(BF16, Cin, Cin, Cout, G, K, cci.ALGO_DENSE_TC)
+    X, W = wl.random_small(N * 7 + Cin + G, "bf16", N, Cin, Cout)
+    Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, "fused " + str(case))
+    Yw = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC_WS)
+    assert_within_tol(f64(Y), f64(Yw), S, "fused vs workspace " + str(case))
+
+
+# (B, H, W, Cin, Cout, KH, KW, stride, pad, G, K): 4-D copies at stride 1 and 2,
+# a 1x1 stride-2 downsample, halo copies (3x3, Cin >= 256) with K = 8, a 5x5
+# window, CTA pairs on a long reduction
+FUSED_CONV = [
+    (2, 14, 14, 64, 128, 3, 3, 1, 1, 8, 2), (3, 15, 15, 64, 64, 3, 3, 2, 1, 16, 4),
+    (2, 14, 14, 128, 256, 1, 1, 2, 0, 8, 1), (1, 14, 14, 256, 256, 3, 3, 1, 1, 8, 4),
+    (2, 7, 7, 512, 512, 3, 3, 1, 1, 32, 8), (2, 12, 12, 64, 64, 5, 5, 1, 2, 4, 2),
+    (16, 14, 14, 256, 512, 3, 3, 2, 1, 8, 2), (8, 28, 28, 128, 128, 3, 3, 1, 1, 16, 4),
+]
+
+
+@pytest.mark.parametrize("case", FUSED_CONV, ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}".format(*c))
+def test_fused_conv(dev, case):
+    B, H, Wi, Cin, Cout, KH, KW, s_, p_, G, K = case
+    skip_without(BF16, Cin, KH * KW * Cin, Cout, G, K, cci.ALGO_DENSE_TC)
+    g = torch.Generator().manual_seed(B * 13 + Cin + KH)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, KH * KW * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (KH, KW, (s_, s_), (p_, p_), Cout), G, K, cci.ALGO_DENSE_TC)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, KH, KW, (s_, s_), (p_, p_))
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, "fused conv " + str(case))
+
+
+def test_fused_checks_index_sets_of_every_tile(dev):
+    """Many column tiles: the CTAs of the first column tile check every group's
+    index sets, so a bad set anywhere is reported (an index >= G here, in the
+    last group and the last reduction index)."""
+    G, K, Cout, Cin, N = 8, 2, 512, 128, 2000
+    W = torch.randn((Cout, Cin), device=dev).to(BF16)
+    v, i = cci.pack(W, G, K)
+    X = torch.randn(N, Cin, device=dev).to(BF16)
+    st = cci.new_status(dev)
+    cci.linear(X, v, i, Cout, G, K, status=st, algo=cci.ALGO_DENSE_TC)
+    assert cci.read_status(st) == 0
+    i[-1, -1, 1] = G
+    st = cci.new_status(dev)
+    cci.linear(X, v, i, Cout, G, K, status=st, algo=cci.ALGO_DENSE_TC)
+    assert cci.read_status(st) == 10
+
+
+def test_auto_without_workspace_uses_fused(dev):
+    """Plain cci_linear (AUTO, no workspace) reaches the tensor cores through the
+    fused family, with the workspace family's result."""
+    N, Cin, Cout, G, K = 700, 256, 512, 8, 2
+    X, W = wl.random_small(41, "bf16", N, Cin, Cout)
+    Xd = X.to(dev)
+    v, i = cci.pack(W.to(dev), G, K)
+    assert cci.kernel_name(BF16, Cin, Cin, Cout, G, K, cci.ALGO_DENSE_TC).startswith("dense_tc_fused")
+    Y = torch.empty((N, Cout), device=dev)
+    st = cci.new_status(dev)
+    code = cci.lib().cci_linear(Xd.data_ptr(), cci.BF16, N, Cin, v.data_ptr(), i.data_ptr(), Cout, G, K,
+                                Y.data_ptr(), st.data_ptr(), torch.cuda.current_stream(dev).cuda_stream)
+    assert code == 0 and cci.read_status(st) == 0
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.linear(f64(X), Wd, mask)
+    assert_within_tol(f64(Y), Yo, S, "plain cci_linear")
+
+
 def test_auto_with_workspace_uses_dense_tc_ws(dev):
-    """AUTO picks the dense tensor-core family for bf16 when given a workspace."""
-    N, Cin, Cout, G, K = 300, 64, 256, 8, 2
+    """AUTO picks the workspace tensor-core family for a bf16 layer the fused
+    family does not take (K = 8) when given a workspace."""
+    N, Cin, Cout, G, K = 300, 64, 256, 16, 8
     X, W = wl.random_small(4, "bf16", N, Cin, Cout)
     Xd = X.to(dev)
     v, i = cci.pack(W.to(dev), G, K)
@@ -774,13 +877,25 @@ def test_fused_pair_tiles(dev):
 
 
 def test_fused_identity_equals_plain_product(dev):
-    """No bias, no ReLU, fp32 output: bit for bit the plain workspace product."""
-    N, Cin, Cout, G, K = 700, 128, 256, 8, 2
-    X, W = wl.random_small(5, "bf16", N, Cin, Cout)
-    Xd = X.to(dev)
+    """No bias, no ReLU, fp32 output: bit for bit the plain product of the family
+    AUTO picks (the binding passes both calls the workspace AUTO asks for), and,
+    with no workspace, of the fused family."""
+    for G, K in ((8, 2), (16, 8)):
+        N, Cin, Cout = 700, 128, 256
+        X, W = wl.random_small(5, "bf16", N, Cin, Cout)
+        Xd = X.to(dev)
+        v, i = cci.pack(W.to(dev), G, K)
+        Yf = cci.linear_fused(Xd, v, i, Cout, G, K)
+        Yp = cci.linear(Xd, v, i, Cout, G, K)
+        assert torch.equal(Yf.view(torch.int32), Yp.view(torch.int32))
+    G, K = 8, 2
     v, i = cci.pack(W.to(dev), G, K)
-    Yf = cci.linear_fused(Xd, v, i, Cout, G, K)
-    Yp = cci.linear(Xd, v, i, Cout, G, K, algo=cci.ALGO_DENSE_TC_WS)
+    Yf = torch.empty((N, Cout), device=dev)
+    code = cci.lib().cci_linear_fused(Xd.data_ptr(), cci.BF16, N, Cin, v.data_ptr(), i.data_ptr(), Cout, G, K,
+                                      None, 0, cci.F32, Yf.data_ptr(), None, None, 0,
+                                      torch.cuda.current_stream(dev).cuda_stream)
+    assert code == 0
+    Yp = cci.linear(Xd, v, i, Cout, G, K, algo=cci.ALGO_DENSE_TC)
     assert torch.equal(Yf.view(torch.int32), Yp.view(torch.int32))
 
 
