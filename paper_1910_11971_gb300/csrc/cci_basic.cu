@@ -1,5 +1,7 @@
 // cci_basic.cu -- the pack kernel, the targeted-dropout mask, the allocation
 // statistics of packing, the generic product kernel and the FMA probe.
+#include <type_traits>
+
 #include "cci_kernels.h"
 
 namespace cci {
@@ -129,21 +131,33 @@ __global__ void __launch_bounds__(128) pack_vec_kernel(const TB *__restrict__ W,
     }
     bool nan = false;
     uint64_t ov[4], oi[4];  // per column: kept values and indices, slot s at s * width
+    // ranking keys: the magnitude bits above the inverted index, so that keys are
+    // distinct and a larger key is a larger |w|, or an equal |w| at a lower index
+    // (the tie rule); the K kept entries are those whose key is at least the K-th
+    // largest, found by K passes of a maximum over the keys below the last one
+    using Key = typename std::conditional<sizeof(TB) == 4, uint64_t, uint32_t>::type;
 #pragma unroll
     for (int v = 0; v < 4; ++v) {
-        uint32_t a[GT];
+        Key key[GT];
 #pragma unroll
-        for (int j = 0; j < GT; ++j) a[j] = static_cast<uint32_t>(w[j][v]) & kAbs;
+        for (int j = 0; j < GT; ++j) {
+            const uint32_t a = static_cast<uint32_t>(w[j][v]) & kAbs;
+            nan |= a > kInf;
+            key[j] = (static_cast<Key>(a) << 8) | static_cast<Key>(255 - j);
+        }
+        Key t = ~static_cast<Key>(0);  // the previous maximum (none yet)
+#pragma unroll
+        for (int k = 0; k < KT; ++k) {
+            Key m = 0;
+#pragma unroll
+            for (int j = 0; j < GT; ++j) m = key[j] < t && key[j] > m ? key[j] : m;
+            t = m;
+        }
         uint64_t vv = 0, ii = 0;
         int sh = 0;  // slot * 8 bits
 #pragma unroll
         for (int j = 0; j < GT; ++j) {
-            nan |= a[j] > kInf;
-            int rank = 0;  // entries ranked ahead of j: larger |w|, or equal |w| at a lower index
-#pragma unroll
-            for (int j2 = 0; j2 < GT; ++j2)
-                rank += j2 < j ? (a[j2] >= a[j]) : (a[j2] > a[j]);
-            if (rank < KT) {
+            if (key[j] >= t) {
                 vv |= static_cast<uint64_t>(w[j][v]) << (sh * (kBits / 8));
                 ii |= static_cast<uint64_t>(j) << sh;
                 sh += 8;

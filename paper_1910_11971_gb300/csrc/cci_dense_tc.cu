@@ -1,7 +1,7 @@
 // cci_dense_tc.cu -- the one-pass decompression of the packed weights into the
 // workspace of CCI_ALGO_DENSE_TC_WS (namespace dc), which precedes the
 // workspace GEMM, and the diagnostic of the kernels' bounded waits.
-#include "cci_tc_common.cuh"
+#include "cci_gemm_ws.cuh"
 
 namespace cci {
 namespace tc {
@@ -105,9 +105,59 @@ __global__ void __launch_bounds__(kSlab) decompress_kernel(const T *__restrict__
     }
 }
 
+// bf16 form without shared memory: each thread expands an item of 8 output
+// channels x 8 reduction indices from its group's packed runs in registers (the
+// expansion of the fused GEMM's producers) and writes the 8 rows with 16-byte
+// stores; blocks run along r (coalesced rows), the block's y index is the row
+// block, so no thread divides.  Index sets are checked everywhere.  Needs
+// G in {4, 8, 16, 32}, K in {1, 2, 4, 8}, K <= G / 2, R % 8 == 0, 16-byte
+// aligned packed arrays and workspace, Cout / 8 <= 65535.
+template <int K>
+__global__ void __launch_bounds__(128) decompress_rows_kernel(FwdParams p, uint16_t *__restrict__ w0)
+{
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 8;
+    if (r >= p.R) return;
+    const int64_t co = static_cast<int64_t>(blockIdx.y) * 8;
+    const int lg = 31 - __clz(p.G);
+    const int64_t groups = p.Cout / p.G;
+    const int64_t g = co >> lg;
+    const int j0 = static_cast<int>(co & (p.G - 1));
+    ws::pk::Runs<K> run;
+    ws::pk::load_item<K>(run, p, g, r, groups);
+    uint32_t out[8][4];
+    bool bad = false;
+    ws::pk::expand_item<K>(out, run, p.G, g, j0, groups, 8, true, bad);
+    if (bad) report(p.status, CCI_ERR_INDEX);
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj)
+        if (co + jj < p.Cout)
+            __stcg(reinterpret_cast<uint4 *>(w0 + (co + jj) * p.R + r),
+                   make_uint4(out[jj][0], out[jj][1], out[jj][2], out[jj][3]));
+}
+
+bool rows_ok(const FwdParams &p, int G, int K)
+{
+    return (G == 4 || G == 8 || G == 16 || G == 32) && (K == 1 || K == 2 || K == 4 || K == 8) && 2 * K <= G &&
+           p.R % 8 == 0 && (p.Cout + 7) / 8 <= 65535 && (p.R / 8 + 127) / 128 <= 0x7fffffff &&
+           reinterpret_cast<uintptr_t>(p.values) % 16 == 0 && reinterpret_cast<uintptr_t>(p.idx) % 16 == 0 &&
+           reinterpret_cast<uintptr_t>(p.wdense) % 16 == 0;
+}
+
 template <typename T, int G, int K, bool SPLIT>
 cudaError_t launch(const FwdParams &p, cudaStream_t stream)
 {
+    if constexpr (!SPLIT) {
+        if (rows_ok(p, G, K) && K <= 8) {
+            FwdParams q = p;
+            q.G = G;
+            q.K = K;
+            const dim3 grid(static_cast<unsigned>((p.R / 8 + 127) / 128), static_cast<unsigned>((p.Cout + 7) / 8));
+            decompress_rows_kernel<(K <= 8 ? K : 8)><<<grid, 128, 0, stream>>>(
+                q, static_cast<uint16_t *>(const_cast<void *>(p.wdense)));
+            return cudaGetLastError();
+        }
+    }
     const int64_t slabs = (p.R + kSlab - 1) / kSlab;
     const int64_t blocks = (p.Cout / G) * slabs;
     if (blocks > 0x7fffffff) return cudaErrorInvalidValue;
