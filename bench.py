@@ -340,13 +340,18 @@ def extra(name: str, payload) -> None:
 # ---------------------------------------------------------------------------
 # our arm
 # ---------------------------------------------------------------------------
+# the sources of the tensor-core product (decompression and GEMM): a DRAM-traffic
+# record in profiles/traffic.txt holds for the sources it was taken on
+PRODUCT_SOURCES = ("cci_common.cuh", "cci_kernels.h", "cci_tc_common.cuh", "cci_gemm_ws.cuh",
+                   "cci_gemm_ws_bf16.cu", "cci_gemm_ws_tf32.cu", "cci_dense_tc.cu")
+
+
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_1910_11971_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + f.read())
+    for name in PRODUCT_SOURCES:
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
     return h.hexdigest()[:16]
 
 

@@ -131,37 +131,55 @@ __global__ void __launch_bounds__(128) pack_vec_kernel(const TB *__restrict__ W,
     }
     bool nan = false;
     uint64_t ov[4], oi[4];  // per column: kept values and indices, slot s at s * width
-    // ranking keys: the magnitude bits above the inverted index, so that keys are
-    // distinct and a larger key is a larger |w|, or an equal |w| at a lower index
-    // (the tie rule); the K kept entries are those whose key is at least the K-th
-    // largest, found by K passes of a maximum over the keys below the last one
+    // ranking keys: the magnitude bits, then the inverted index, then the sign:
+    // keys are distinct, a larger key is a larger |w| or an equal |w| at a lower
+    // index (the tie rule; the sign ranks nothing), and a key gives back its entry
+    // (value = sign and magnitude, index = 255 - the index field).  The K kept
+    // entries are the K largest keys, found by K passes of a maximum over the
+    // keys below the previous one, then put in increasing index.
     using Key = typename std::conditional<sizeof(TB) == 4, uint64_t, uint32_t>::type;
 #pragma unroll
     for (int v = 0; v < 4; ++v) {
         Key key[GT];
 #pragma unroll
         for (int j = 0; j < GT; ++j) {
-            const uint32_t a = static_cast<uint32_t>(w[j][v]) & kAbs;
+            const uint32_t b = static_cast<uint32_t>(w[j][v]);
+            const uint32_t a = b & kAbs;
             nan |= a > kInf;
-            key[j] = (static_cast<Key>(a) << 8) | static_cast<Key>(255 - j);
+            // the fields do not overlap: a multiply-add builds the key (FMA pipe)
+            key[j] = static_cast<Key>(a) * 512u + static_cast<Key>(((255 - j) << 1) + (b >> (kBits - 1)));
         }
-        Key t = ~static_cast<Key>(0);  // the previous maximum (none yet)
+        Key sel[KT];
+        Key t = key[0];
 #pragma unroll
-        for (int k = 0; k < KT; ++k) {
+        for (int j = 1; j < GT; ++j) t = key[j] > t ? key[j] : t;
+        sel[0] = t;
+#pragma unroll
+        for (int k = 1; k < KT; ++k) {
             Key m = 0;
 #pragma unroll
-            for (int j = 0; j < GT; ++j) m = key[j] < t && key[j] > m ? key[j] : m;
-            t = m;
-        }
-        uint64_t vv = 0, ii = 0;
-        int sh = 0;  // slot * 8 bits
-#pragma unroll
-        for (int j = 0; j < GT; ++j) {
-            if (key[j] >= t) {
-                vv |= static_cast<uint64_t>(w[j][v]) << (sh * (kBits / 8));
-                ii |= static_cast<uint64_t>(j) << sh;
-                sh += 8;
+            for (int j = 0; j < GT; ++j) {
+                const Key c = key[j] < t ? key[j] : 0;
+                m = c > m ? c : m;
             }
+            sel[k] = t = m;
+        }
+        // increasing index = decreasing inverted-index field
+#pragma unroll
+        for (int a = 0; a < KT; ++a)
+#pragma unroll
+            for (int b = 0; b + 1 < KT - a; ++b) {
+                const Key x = sel[b], y = sel[b + 1];
+                const bool swap = ((x >> 1) & 255) < ((y >> 1) & 255);
+                sel[b] = swap ? y : x;
+                sel[b + 1] = swap ? x : y;
+            }
+        uint64_t vv = 0, ii = 0;
+#pragma unroll
+        for (int k = 0; k < KT; ++k) {
+            const uint64_t value = static_cast<uint64_t>((sel[k] >> 9) | (static_cast<Key>(sel[k] & 1) << (kBits - 1)));
+            vv |= value << (k * kBits);
+            ii |= static_cast<uint64_t>(255 - ((sel[k] >> 1) & 255)) << (8 * k);
         }
         ov[v] = vv;
         oi[v] = ii;

@@ -237,6 +237,32 @@ __device__ __forceinline__ void stage_f16(uint32_t d, uint64_t adesc, uint64_t b
         : "memory");
 }
 
+// ---- one pipeline stage of bf16 MMAs over a CTA pair ----
+// The four 16-deep cta_group::2 MMAs of a 64-wide stage (issued by the even CTA;
+// descriptors advance by 32 bytes per MMA) and the commit that releases the
+// stage in both CTAs (arrival multicast to the barrier at this offset in each),
+// from one block executed by the issuing thread alone.  The separate per-MMA
+// form took ~360 cycles per stage to issue on GB300 (clock stamps), against 512
+// cycles of MMA work: the issue, not the tensor pipe, set the stage period.
+template <uint32_t kIdesc>
+__device__ __forceinline__ void stage_f16_pair(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t acc0,
+                                               uint32_t bar)
+{
+    asm volatile(
+        "{\n.reg .pred pa, pt;\n.reg .b64 ad, bd;\n"
+        "setp.ne.b32 pa, %3, 0;\nsetp.eq.b32 pt, 0, 0;\n"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %4, pa;\n"
+        "add.s64 ad, %1, 2;\nadd.s64 bd, %2, 2;\n"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, %1, 4;\nadd.s64 bd, %2, 4;\n"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, %1, 6;\nadd.s64 bd, %2, 6;\n"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%5], %6;\n}\n" ::"r"(d),
+        "l"(adesc), "l"(bdesc), "r"(acc0), "n"(kIdesc), "r"(bar), "h"(static_cast<uint16_t>(3))
+        : "memory");
+}
+
 // ---- cluster-pair helpers (CG = 2) ----
 __device__ __forceinline__ uint32_t cluster_rank()
 {
@@ -1105,6 +1131,41 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                             d, tmem + static_cast<uint32_t>(C::kAColBase + s * 64),
                             bdesc0 + static_cast<uint64_t>(s) * (C::kStage >> 4) + (C::kBOff >> 4), ks > 0 ? 1u : 0u,
                             1u, empty0 + 8u * s);
+                    }
+                    if (ok) commit(&S->tmem_full[acc]);
+                }
+            }
+            ok = false;  // the generic loop below is not entered
+        }
+        if constexpr (!TF32 && ASRC != kAHalo) {
+            // bf16 stages of one A and one B plane: one thread runs the issue loop,
+            // each stage's MMAs and its commit issued from one block (pairs: from the
+            // even CTA, which alone enters with ok set)
+            if (lane == 0 && ok) {
+                int s = 0;
+                uint32_t ph = 0u;  // parity of the full-barrier phase to wait for
+                const uint64_t sunits = C::kStage >> 4, bunits = C::kBOff >> 4;
+                for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
+                    const int acc = t & 1;
+                    // CG = 2: the phase includes arrivals of the odd CTA's epilogue
+                    if (t >= 2) ok = tc::mbar_wait<CG == 2>(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
+                    if (!ok) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
+                    for (int ks = 0; ks < nks; ++ks) {
+                        // PK pairs: the phase includes the odd CTA's producers (released at cluster scope)
+                        ok = tc::mbar_wait<PK && CG == 2>(&S->full[s], ph, abort, p.status);
+                        if (!ok) break;
+                        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                        const uint64_t ad = bdesc0 + static_cast<uint64_t>(s) * sunits;
+                        if constexpr (CG == 2)
+                            stage_f16_pair<C::kIdesc>(d, ad, ad + bunits, ks > 0 ? 1u : 0u, empty0 + 8u * s);
+                        else
+                            stage_f16<C::kIdesc>(d, ad, ad + bunits, ks > 0 ? 1u : 0u, 1u, empty0 + 8u * s);
+                        if (++s == kStages) {
+                            s = 0;
+                            ph ^= 1u;
+                        }
                     }
                     if (ok) commit(&S->tmem_full[acc]);
                 }
