@@ -35,24 +35,25 @@
 // Weights (the template's PK):
 //   PK = false  the dense workspace planes written by the one-pass decompression;
 //   PK = true   the packed (value, index) pairs themselves (bf16 only, no
-//               workspace): the producer warps load the K-slot runs of their
-//               groups from global memory two stages ahead (into registers),
-//               expand them into rows (Alg. 2's index: each pair goes to row
-//               G*i + Idx of its group), 8 rows x 8 indices per thread, and once
-//               the stage is free store the rows into its swizzled B tile.
+//               workspace): two groups of four producer warps take the stages
+//               in turn; each thread loads the K-slot runs of its groups from
+//               global memory two of its stages ahead (into registers), expands
+//               them into rows (Alg. 2's index: each pair goes to row G*i + Idx
+//               of its group), 8 rows x 8 indices per thread, and once the stage
+//               is free stores the rows into its swizzled B tile.
 // Output: fp32 Y written by TMA stores from a swizzled staging buffer (two
 // alternating 16 KB buffers of [128 rows][32 columns]), 2-D over Y[N][Cout] or,
 // for kA4d, 4-D over Y[B][P][Q][Cout] with the tile's pixel box.
 // Roles: warps 0-3 epilogue (TMEM lanes), warps 4-7 producers of the activation
-// planes that are not copied by TMA (PK: of the weight tiles), warp 8
-// allocates TMEM and issues the MMAs,
-// warps 9.. issue the TMA copies as soon as a stage is free (so copy latency
-// overlaps the producers' work), stage by stage in turn: the copies one thread
-// issues are processed one box after another (measured on GB300: about 0.5 us
-// per box of 16-64 KB from one issuer; copy throughput grows with the number of
-// issuing warps), so up to six warps issue (one per stage in flight).  Every
-// mbarrier wait is bounded
-// (CCI_ERR_TIMEOUT, abort flag, drain, TMEM freed).
+// planes that are not copied by TMA (PK: of the weight tiles, with warps
+// 9 + kIssuers .. + 3 as the second producer group), warp 8 allocates TMEM and
+// issues the MMAs, warps 9 .. 8 + kIssuers issue the TMA copies as soon as a
+// stage is free (so copy latency overlaps the producers' work), stage by stage in
+// turn: the copies one thread issues are processed one box after another
+// (measured on GB300: about 0.5 us per box of 16-64 KB from one issuer; copy
+// throughput grows with the number of issuing warps), so up to six warps issue
+// (one per stage in flight; PK: three, one activation box per stage).  Every
+// mbarrier wait is bounded (CCI_ERR_TIMEOUT, abort flag, drain, TMEM freed).
 #pragma once
 
 #include <cuda.h>
@@ -144,8 +145,13 @@ struct Cfg {
     // more boxes moving.  kIssuers <= kStages keeps every empty-barrier wait
     // within one phase of the barrier (no parity aliasing).
     // (kAHalo: one more warp, which copies the halos)
-    static constexpr int kIssuers = ASRC == kAGather ? 1 : (kStages < 6 ? kStages : 6) + (kHalo ? 1 : 0);
-    static constexpr int kThreads = 32 * (9 + kIssuers);
+    // PK: three issuers (one activation box per stage) and a second group of four
+    // producer warps after them
+    static constexpr int kStageIssuers = PK ? (kHalo ? 1 : 3) : 6;  // PK halo stages: the producers' tiles only
+    static constexpr int kIssuers =
+        ASRC == kAGather ? 1 : (kStages < kStageIssuers ? kStages : kStageIssuers) + (kHalo ? 1 : 0);
+    static constexpr int kProdGroups = PK ? 2 : 1;
+    static constexpr int kThreads = 32 * (9 + kIssuers + 4 * (kProdGroups - 1));
     static_assert(kIssuers - (kHalo ? 1 : 0) >= 1 && kIssuers - (kHalo ? 1 : 0) <= kStages,
                   "stage issuers must not outnumber the stages");
 };
@@ -289,6 +295,17 @@ __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr)
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
+// arrival on the even CTA's barrier that releases this thread's (and, through a
+// preceding warp or CTA barrier, its peers') shared-memory writes: a release
+// fence restricted to shared::cta accesses, then a relaxed arrive.  Measured on
+// GB300 in the fused family's producer loop: ~950 cycles per stage for the
+// cluster-scope release arrive above, a few hundred for this form.
+__device__ __forceinline__ void mbar_arrive_remote_smem(uint32_t cluster_addr)
+{
+    asm volatile("fence.release.sync_restrict::shared::cta.cluster;" ::: "memory");
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
 // tcgen05.commit of the pair's MMAs, arriving on the barrier at this offset in both CTAs
 __device__ __forceinline__ void mma_commit_pair(uint64_t *bar)
 {
@@ -379,13 +396,13 @@ __device__ __forceinline__ uint32_t lo_bits(uint32_t x)
 // co0 + m0 .. + 7) x 8 consecutive reduction indices (one 16-byte chunk of each
 // row).  Its inputs are the K-slot runs of the item's group(s) over those 8
 // indices, loaded from the packed arrays ([r][slot]: values bf16, indices
-// uint8) into registers.  Rows are built two indices (one 32-bit word: a bf16 pair) at
-// a time: for r-pair p and slot s, the pair's two values are ANDed with a mask
-// that is 0xffff in each half whose index names the row, and ORed into the row's
-// word.  The masks come from one byte permute per row: the permute's selector
-// nibbles are the two indices (each twice), its 8 source bytes the row table
-// (byte jj = 0xff for row jj, else 0), so byte k of the result is 0xff exactly
-// when the index of half k / 2 equals the row.
+// uint8) into registers.  Rows are built two indices (one 32-bit word: a bf16
+// pair) at a time: for r-pair p and slot s, the pair's two values are ANDed with
+// a mask that is 0xffff in each half whose index names the row, and ORed into
+// the row's word.  The masks come from one packed f16x2 equality test per row:
+// each index i of the pair becomes the f16 number with bits 0x3c00 | i (a key
+// in [1, 2), distinct per index, exact), compared with the row's key; the test
+// yields 0xffff per equal half.
 namespace pk {
 
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
@@ -395,9 +412,16 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel)
     return r;
 }
 
-// row table of row jj of the 8-row item: source bytes 0-3 (lo) and 4-7 (hi)
-__device__ __forceinline__ constexpr uint32_t row_lo(int jj) { return jj < 4 ? 0xffu << (8 * jj) : 0u; }
-__device__ __forceinline__ constexpr uint32_t row_hi(int jj) { return jj >= 4 ? 0xffu << (8 * (jj - 4)) : 0u; }
+// 0xffff in each half of a where it equals the same half of b (both f16x2)
+__device__ __forceinline__ uint32_t eq_mask(uint32_t a, uint32_t b)
+{
+    uint32_t r;
+    asm("set.eq.u32.f16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+    return r;
+}
+
+// key of row jj in both halves
+__device__ __forceinline__ constexpr uint32_t row_key(int jj) { return (0x3c00u | static_cast<uint32_t>(jj)) * 0x00010001u; }
 
 // values of slot s at r = 2p (low half) and 2p + 1 (high half); vw holds the
 // item's K-slot runs, v[r][s] at bf16 position r * K + s
@@ -412,42 +436,36 @@ __device__ __forceinline__ uint32_t val_pair(const uint32_t *vw, int p, int s)
     }
 }
 
-// indices of slot s at r = 2p (byte 0) and 2p + 1 (byte 1); bytes 2 and 3 are
-// not used by the callers
+// keys of the indices of slot s at r = 2p (low half) and 2p + 1 (high half):
+// bytes (index, 0x3c, index, 0x3c)
 template <int K>
-__device__ __forceinline__ uint32_t idx_pair(const uint32_t *iw, int p, int s)
+__device__ __forceinline__ uint32_t key_pair(const uint32_t *iw, int p, int s)
 {
     const int b0 = 2 * p * K + s, b1 = (2 * p + 1) * K + s;
-    if ((b0 >> 2) == (b1 >> 2)) return prmt(iw[b0 >> 2], 0u, static_cast<uint32_t>((b0 & 3) | ((b1 & 3) << 4)) | 0x4400u);
-    return prmt(iw[b0 >> 2], iw[b1 >> 2], static_cast<uint32_t>((b0 & 3) | ((4 + (b1 & 3)) << 4)) | 0x4400u);
+    if ((b0 >> 2) == (b1 >> 2))
+        return prmt(iw[b0 >> 2], 0x3c3c3c3cu, static_cast<uint32_t>((b0 & 3) | 0x40 | ((b1 & 3) << 8) | 0x4000));
+    return (prmt(iw[b0 >> 2], iw[b1 >> 2], static_cast<uint32_t>((b0 & 3) | ((4 + (b1 & 3)) << 8))) & 0x00ff00ffu) |
+           0x3c003c00u;
 }
 
-// adds one group's K slots to the item's rows.  MODE 0: indices are rows (G = 8,
-// or the first group of a G = 4 item); MODE 1: rows are index + 4 (the second
-// group of a G = 4 item); MODE 2: G >= 16, the item covers rows j0 .. j0 + 7 of
-// its group (J = j0 * 0x0101) and slots whose index lies outside add nothing.
-// INIT: the first group of the item (rows start from its contributions).
-template <int K, int MODE, bool INIT>
-__device__ __forceinline__ void expand_group(uint32_t (&out)[8][4], const uint32_t *vw, const uint32_t *iw, uint32_t J)
+// adds one group's K slots to rows J0 .. J1 - 1 of the item: a slot of index i
+// goes to row i + off (off: 4 for the second group of a G = 4 item, -j0 for
+// G >= 16, whose items cover rows j0 .. j0 + 7 of their group; slots whose row
+// lies outside add nothing).  INIT: these rows start from this group's
+// contributions.
+template <int K, int J0, int J1, bool INIT>
+__device__ __forceinline__ void expand_group(uint32_t (&out)[8][4], const uint32_t *vw, const uint32_t *iw, int off)
 {
+    const uint32_t kadd = static_cast<uint32_t>(off) * 0x00010001u;  // off + 0x3c00 >= 0 in each half: no borrow
 #pragma unroll
     for (int pr = 0; pr < 4; ++pr) {
 #pragma unroll
         for (int s = 0; s < K; ++s) {
-            uint32_t v = val_pair<K>(vw, pr, s);
-            const uint32_t u = idx_pair<K>(iw, pr, s);
-            uint32_t sel;
-            if constexpr (MODE == 2) {
-                const uint32_t x = u ^ J;  // in the block: x < 8 (j0 is a multiple of 8, index < 32)
-                sel = (x & 0x0707u) * 0x11u;
-                // halves outside the block: 0xffff (sign of byte + 0x7f), value cleared
-                v &= ~prmt((x & 0x1818u) + 0x7f7fu, 0u, 0x9988u);
-            } else {
-                sel = (MODE == 1 ? u + 0x0404u : u) * 0x11u;  // nibbles (i0, i0, i1, i1)
-            }
+            const uint32_t v = val_pair<K>(vw, pr, s);
+            const uint32_t key = key_pair<K>(iw, pr, s) + kadd;
 #pragma unroll
-            for (int jj = 0; jj < 8; ++jj) {
-                const uint32_t m = prmt(row_lo(jj), row_hi(jj), sel);
+            for (int jj = J0; jj < J1; ++jj) {
+                const uint32_t m = eq_mask(key, row_key(jj));
                 if (INIT && s == 0)
                     out[jj][pr] = v & m;
                 else
@@ -558,16 +576,13 @@ __device__ __forceinline__ void expand_item(uint32_t (&out)[8][4], const Runs<K>
         if (G == 4) {
             if (chk && g < groups) bad |= bad_sets<K>(run.i[0], G, nr);
             if (chk && g + 1 < groups) bad |= bad_sets<K>(run.i[1], G, nr);
-            expand_group<K, 0, true>(out, run.v[0], run.i[0], 0u);
-            expand_group<K, 1, false>(out, run.v[1], run.i[1], 0u);
+            expand_group<K, 0, 4, true>(out, run.v[0], run.i[0], 0);
+            expand_group<K, 4, 8, true>(out, run.v[1], run.i[1], 4);
             return;
         }
     }
     if (chk && j0 == 0 && g < groups) bad |= bad_sets<K>(run.i[0], G, nr);
-    if (G == 8)
-        expand_group<K, 0, true>(out, run.v[0], run.i[0], 0u);
-    else
-        expand_group<K, 2, true>(out, run.v[0], run.i[0], static_cast<uint32_t>(j0) * 0x0101u);
+    expand_group<K, 0, 8, true>(out, run.v[0], run.i[0], -j0);  // G = 8: j0 = 0
 }
 
 }  // namespace pk
@@ -625,9 +640,10 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
 
     if (tid == 0) {
         // full[s]: the copy issuer's expect_tx arrival (none for PK halo stages) and
-        // PK: one arrival per producer group of the pair (elected after their
-        // writes), else 128 producer arrivals when the producers fill the stage
-        const uint32_t full_count = PK ? (C::kHalo ? 0u : 1u) + CG : (C::kATma ? 1u : 129u);
+        // PK: one arrival per producer warp of the stage's group in each CTA of the
+        // pair (after the warp's writes), else 128 producer arrivals when the
+        // producers fill the stage
+        const uint32_t full_count = PK ? (C::kHalo ? 0u : 1u) + 4 * CG : (C::kATma ? 1u : 129u);
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(&S->full[s], full_count);
             tc::mbar_init(&S->empty[s], 1);
@@ -687,7 +703,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
     // after that grid has completed and its writes are visible
     asm volatile("griddepcontrol.wait;" ::: "memory");
 
-    if (warp >= 9) {
+    if (warp >= 9 && warp < 9 + C::kIssuers) {
         // ------------------------------------------------------------ TMA issuers
         const uint32_t a_bytes = ASRC == kA4d ? static_cast<uint32_t>(box.rows) * 128u : C::kAPlane;
         const int cpt = static_cast<int>(p.Cin / kKS);  // stages per tap (kA4d)
@@ -798,14 +814,20 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                 __syncwarp();
             }
         }
-    } else if (PK && warp >= 4 && warp < 8) {
+    } else if (PK && ((warp >= 4 && warp < 8) || warp >= 9 + C::kIssuers)) {
         // ------------------------------------------------------------ weight producers (PK)
-        // thread pt builds item pt of every stage: rows 8 (pt / 8) .. + 7 of this
-        // CTA's B tile, reduction indices 8 (pt % 8) .. + 7 of the stage.  Its runs
-        // are loaded NB stages ahead into a ring of NB register sets (a set is
-        // refilled right after it is expanded), expanded into rows while the stage
-        // may still be in use, and stored once the stage's MMAs released it.
-        const int pt = tid - 128;
+        // two groups of four warps (4-7 and the four after the issuers) take the
+        // stages in turn: group q builds the stages it with it % 2 == q, so each
+        // group has two MMA stages of time per tile it builds.  Thread pt of a
+        // group builds item pt of each of its stages: rows 8 (pt / 8) .. + 7 of
+        // this CTA's B tile, reduction indices 8 (pt % 8) .. + 7 of the stage.  Its
+        // runs are loaded NB of its stages ahead into a ring of NB register sets (a
+        // set is refilled right after it is expanded), expanded into rows while the
+        // stage may still be in use, and stored once the stage's MMAs released it;
+        // then each warp releases its writes to the stage's full barrier (pair: the
+        // even CTA's).
+        const int q = warp >= 8 ? 1 : 0;
+        const int pt = tid - (q ? 32 * (9 + C::kIssuers) : 128);
         const int m0 = (pt >> 3) * 8, c = pt & 7;
         const bool active = m0 < C::kBRows;
         const int64_t groups = p.Cout / p.G;
@@ -822,31 +844,31 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
             int ks, t, ch, j0;
             bool chk;
         };
-        auto tile_start = [&](Cursor &q) {
-            if (q.u >= n_tiles) return;
+        auto tile_start = [&](Cursor &cu) {
+            if (cu.u >= n_tiles) return;
             int64_t mt, ct;
-            split_unit(q.u, mt, ct);
-            q.co = ct * kN + crank * C::kBRows + m0;
-            q.g = q.co >> lg;
-            q.j0 = static_cast<int>(q.co & (p.G - 1));
-            q.chk = mt < CG;
-            q.ks = q.t = q.ch = 0;
-            q.r = 8 * c;
+            split_unit(cu.u, mt, ct);
+            cu.co = ct * kN + crank * C::kBRows + m0;
+            cu.g = cu.co >> lg;
+            cu.j0 = static_cast<int>(cu.co & (p.G - 1));
+            cu.chk = mt < CG;
+            cu.ks = cu.t = cu.ch = 0;
+            cu.r = 8 * c;
         };
-        auto advance = [&](Cursor &q) {
-            if (++q.ks == nks) {
-                q.u += ustep;
-                tile_start(q);
+        auto advance = [&](Cursor &cu) {
+            if (++cu.ks == nks) {
+                cu.u += ustep;
+                tile_start(cu);
                 return;
             }
             if constexpr (ASRC == kAHalo) {  // stages chunk by chunk, the taps of a chunk in turn
-                if (++q.t == taps) {
-                    q.t = 0;
-                    ++q.ch;
+                if (++cu.t == taps) {
+                    cu.t = 0;
+                    ++cu.ch;
                 }
-                q.r = static_cast<int64_t>(q.t) * p.Cin + q.ch * 64 + 8 * c;
+                cu.r = static_cast<int64_t>(cu.t) * p.Cin + cu.ch * 64 + 8 * c;
             } else {
-                q.r += 64;
+                cu.r += 64;
             }
         };
         auto run_k = [&](auto kc) {
@@ -855,52 +877,54 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
             pk::Runs<K> ring[NB];
             Cursor cur{u0, 0, 0, 0, 0, 0, 0, 0, false};  // the stage being built
             tile_start(cur);
-            Cursor pre = cur;  // the stage whose runs are loaded next (NB ahead)
+            if (q) advance(cur);  // group 1 starts at the second stage
+            Cursor pre = cur;     // the stage whose runs are loaded next (NB of this group's ahead)
             auto load = [&](pk::Runs<K> &rg) {
                 if (active && pre.u < n_tiles) pk::load_item<K>(rg, p, pre.g, pre.r, groups);
                 advance(pre);
+                advance(pre);
             };
 #pragma unroll
-            for (int q = 0; q < NB; ++q) load(ring[q]);
+            for (int b = 0; b < NB; ++b) load(ring[b]);
             bool ok = true;
-            int s = 0;               // stage of the ring
-            uint32_t eph = 0;        // parity of the empty-barrier phase to wait for
-            bool wrapped = false;    // every stage used once already
+            int s = q;     // stage of the ring
+            int pass = 0;  // passes over the ring completed before this stage
             while (ok && cur.u < n_tiles) {
 #pragma unroll
-                for (int q = 0; q < NB; ++q) {
+                for (int b = 0; b < NB; ++b) {
                     if (!ok || cur.u >= n_tiles) break;
                     uint32_t out[8][4];
                     if (active) {
                         const int64_t left = p.R - cur.r;
                         const int nr = left <= 0 ? 0 : (left >= 8 ? 8 : static_cast<int>(left));
-                        pk::expand_item<K>(out, ring[q], p.G, cur.g, cur.j0, groups, nr, cur.chk, bad);
+                        pk::expand_item<K>(out, ring[b], p.G, cur.g, cur.j0, groups, nr, cur.chk, bad);
                     }
-                    load(ring[q]);
-                    if (wrapped) ok = tc::mbar_wait(&S->empty[s], eph, abort, p.status);
+                    load(ring[b]);
+                    if (pass > 0) ok = tc::mbar_wait(&S->empty[s], (pass - 1) & 1, abort, p.status);
                     if (ok && active) {
                         const uint32_t bst = base + s * C::kStage + C::kBOff;
 #pragma unroll
                         for (int jj = 0; jj < 8; ++jj)
                             st_shared_v4(bst + sw_chunk(m0 + jj, c), out[jj][0], out[jj][1], out[jj][2], out[jj][3]);
                     }
-                    // the tile's writes are visible to the MMAs (async proxy) once one
-                    // thread of the group arrives after all of them (pair: on the even
-                    // CTA's barrier, released at cluster scope)
+                    // the warp's writes are visible to the MMAs (async proxy) once its
+                    // lane 0 arrives after all of them (pair: on the even CTA's barrier)
                     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                    ok = tc::named_and(3, 128, ok);
+                    __syncwarp();
+                    ok = __all_sync(0xffffffffu, ok);
                     if (!ok) break;
-                    if (pt == 0) {
+                    if (lane == 0) {
                         if (CG == 2 && crank != 0)
-                            mbar_arrive_remote(full_remote + static_cast<uint32_t>(s * sizeof(uint64_t)));
+                            mbar_arrive_remote_smem(full_remote + static_cast<uint32_t>(s * sizeof(uint64_t)));
                         else
                             tc::mbar_arrive(&S->full[s]);
                     }
                     advance(cur);
-                    if (++s == kStages) {
-                        s = 0;
-                        eph ^= wrapped ? 1u : 0u;
-                        wrapped = true;
+                    advance(cur);
+                    s += 2;
+                    if (s >= kStages) {
+                        s -= kStages;
+                        ++pass;
                     }
                 }
             }
