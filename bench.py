@@ -432,16 +432,6 @@ def profile_conv(cci, case, args, dev, stream):
     return 0
 
 
-def dense_planes(W: torch.Tensor) -> torch.Tensor:
-    """Unpruned weights in the dense family's layout, for the same-kernel dense
-    line: bf16 as is; fp32 as the hi / lo tf32 planes (hi = low 13 mantissa bits
-    cleared, lo = w - hi)."""
-    if W.dtype == torch.bfloat16:
-        return W.contiguous()
-    hi = (W.view(torch.int32) & -8192).view(torch.float32)
-    return torch.stack([hi, W - hi]).contiguous()
-
-
 def launches_per_product(cci, dtype, case) -> int:
     """Kernels one product launches on the production path (AUTO): the workspace
     family runs a decompression and the GEMM, every other family one kernel."""
@@ -624,7 +614,7 @@ def run_sweep(cci, dev, stream, flush, reps=10):
         Wm.view(case.Cout // G, G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
         dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), reps, flush, stream))
         if dense_same_ms is None:  # one shape for every point: the unpruned W of the first
-            Wp = dense_planes(W)
+            Wp = cci.dense_planes(W)
             fd = lambda: cci.dense_linear_tc(X, Wp, case.Cout, out=Y)  # noqa: E731
             fd()
             dense_same_ms = statistics.median(time_device(fd, reps, flush, stream))
@@ -690,7 +680,7 @@ def run_bottleneck_fp32(cci, dev, stream, flush, reps=10):
     Wm = torch.zeros_like(W)
     Wm.view(case.Cout // case.G, case.G, case.R).scatter_(1, i.permute(0, 2, 1).long(), v.permute(0, 2, 1))
     dms = statistics.median(time_device(lambda: torch.matmul(X, Wm.t()), reps, flush, stream))
-    Wp = dense_planes(W)
+    Wp = cci.dense_planes(W)
     fd = lambda: cci.dense_linear_tc(X, Wp, case.Cout, out=Y)  # noqa: E731
     fd()
     sms = statistics.median(time_device(fd, reps, flush, stream))

@@ -111,10 +111,15 @@ typedef enum cci_algo {
     CCI_ALGO_DENSE_TC_WS = 5  /* decompress the packed weights once per call into a caller
                                workspace and multiply densely on the tensor cores (tcgen05),
                                operands copied by TMA (cp.async.bulk.tensor).  bf16: dense bf16 [Cout][R],
-                               Cin % 8 == 0, R % 8 == 0.  fp32: hi and lo tf32 planes
-                               [2][Cout][R] and a three-pass tf32 product (hi*hi + hi*lo +
-                               lo*hi, |error| below 2^-21 of sum |w||x|), Cin % 4 == 0,
-                               R % 4 == 0.  Needs cci_workspace_size() bytes */
+                               Cin % 8 == 0, R % 8 == 0.  fp32: every operand split as
+                               hi + lo (hi a tf32 value) and, per 32 indices, the product
+                               hi(x) hi(w) on tf32 MMAs plus bf16(x) bf16(lo(w)) +
+                               bf16(lo(x)) bf16(hi(w)) on bf16 MMAs (8 MMAs; per term
+                               |error| <= 5.7e-6 |w||x| before the fp32 accumulation);
+                               workspace: plane 0 [Cout][R] fp32 hi, then plane 1
+                               [Cout][ceil(R/32)*64] bf16 (per 32-wide chunk of r, 32
+                               bf16(hi(w)) then 32 bf16(lo(w))).  Cin % 4 == 0, R % 4 == 0.
+                               Needs cci_workspace_size() bytes */
 } cci_algo;
 
 /*
@@ -193,7 +198,8 @@ cci_status cci_conv2d_ex(const void *X, cci_dtype dtype, int64_t B, int64_t H, i
  * cci_workspace_size -- bytes of device workspace that cci_linear_ws /
  * cci_conv2d_ws need for this kernel family and layer (R = Cin for a product,
  * Cin*KH*KW for a convolution): for CCI_ALGO_DENSE_TC_WS Cout*R*2 (bf16) or
- * Cout*R*8 (fp32), 0 for the families that need none.  For CCI_ALGO_AUTO: the
+ * Cout*(R*4 + ceil(R/32)*128) (fp32: Cout*R*8 when R % 32 == 0), 0 for the
+ * families that need none.  For CCI_ALGO_AUTO: the
  * bytes that let AUTO pick its fastest family (the dense tensor-core one).
  */
 size_t cci_workspace_size(cci_algo algo, cci_dtype dtype, int64_t Cout, int64_t R);
@@ -363,9 +369,9 @@ cci_status cci_conv2d_fused(const void *X, cci_dtype dtype, int64_t B, int64_t H
  * work of the product by G/K; timing the same kernel on the unpruned weights
  * shows how much of that a dense tensor-core product keeps.
  *
- *   Wd   device, 16-byte aligned, in the workspace layout of the dense family:
- *        bf16 dense [Cout][R]; fp32 the hi and lo tf32 planes [2][Cout][R]
- *        (hi = w with the low 13 mantissa bits cleared, lo = w - hi)
+ *   Wd   device, 16-byte aligned, in the workspace layout of the dense family
+ *        (CCI_ALGO_DENSE_TC_WS): bf16 dense [Cout][R]; fp32 the two operand
+ *        planes, as cci_dense_planes writes them
  *   X, Y as cci_linear / cci_conv2d, 16-byte aligned; Cin % 8 == 0 (bf16) or
  *        % 4 == 0 (fp32); Cout % 4 == 0
  * Errors: CCI_ERR_NULL, CCI_ERR_SHAPE, CCI_ERR_DTYPE, CCI_ERR_ALIGN,
@@ -377,6 +383,20 @@ cci_status cci_dense_conv2d_tc(const void *X, cci_dtype dtype, int64_t B, int64_
                                int64_t Cin, const void *Wd, int64_t Cout, int KH, int KW,
                                int stride_h, int stride_w, int pad_h, int pad_w, float *Y,
                                uint32_t *dev_status, cci_stream_t stream);
+
+/*
+ * cci_dense_planes -- writes a dense weight matrix W[Cout][R] (device, 16-byte
+ * aligned, OHWI order for a convolution) in the workspace layout that
+ * cci_dense_linear_tc / cci_dense_conv2d_tc read: bf16 copied as is; fp32 split
+ * into the two operand planes of CCI_ALGO_DENSE_TC_WS (hi the nearest tf32 value
+ * of w, lo = w - hi).  Wd: device, 16-byte aligned, bytes >=
+ * cci_workspace_size(CCI_ALGO_DENSE_TC_WS, dtype, Cout, R).  Asynchronous on
+ * stream.  Errors: CCI_ERR_DTYPE, CCI_ERR_SHAPE, CCI_ERR_NULL, CCI_ERR_WORKSPACE
+ * (bytes too small), CCI_ERR_ALIGN (pointers, or R % 4 (fp32) / % 8 (bf16)),
+ * CCI_ERR_CUDA.
+ */
+cci_status cci_dense_planes(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, void *Wd, size_t bytes,
+                            cci_stream_t stream);
 
 /* Largest dense-weight size (Cout*R*2 bytes) that cci_linear_dense_tc_static accepts. */
 #define CCI_STATIC_WORKSPACE_BYTES (16u * 1024u * 1024u)

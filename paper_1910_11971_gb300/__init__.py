@@ -64,6 +64,7 @@ SIGNATURES = {
     "cci_linear_dense_tc_static": (_I32, [_P, _I32, _I64, _I64, _P, _P, _I64, _I32, _I32, _P, _U32P,
                                           _P]),
     "cci_dense_linear_tc": (_I32, [_P, _I32, _I64, _I64, _P, _I64, _P, _U32P, _P]),
+    "cci_dense_planes": (_I32, [_P, _I32, _I64, _I64, _P, ctypes.c_size_t, _P]),
     "cci_dense_conv2d_tc": (_I32, [_P, _I32, _I64, _I64, _I64, _I64, _P, _I64, _I32, _I32, _I32, _I32,
                                    _I32, _I32, _P, _U32P, _P]),
     "cci_kernel_name": (ctypes.c_char_p, [_I32, _I64, _I64, _I64, _I32, _I32, _I32]),
@@ -415,11 +416,25 @@ def conv2d_fused(X: torch.Tensor, values: torch.Tensor, idx: torch.Tensor, Cout:
     return Y
 
 
+def dense_planes(W: torch.Tensor) -> torch.Tensor:
+    """Dense weights W[Cout][R] (OHWI rows for a convolution) in the workspace
+    layout of the dense tensor-core family (``cci_dense_planes``), for
+    ``dense_linear_tc`` / ``dense_conv2d_tc``: bf16 as is, fp32 as its two
+    operand planes (a byte tensor)."""
+    _cuda_contig(W, "W")
+    Cout = W.shape[0]
+    R = W.numel() // Cout
+    Wd = new_workspace(ALGO_DENSE_TC_WS, W.dtype, Cout, R, W.device)
+    _check(lib().cci_dense_planes(W.data_ptr(), _dtype_code(W), Cout, R, Wd.data_ptr(), Wd.numel(),
+                                  _stream(W.device)), "cci_dense_planes")
+    return Wd
+
+
 def dense_linear_tc(X: torch.Tensor, Wd: torch.Tensor, Cout: int, *, out: Optional[torch.Tensor] = None,
                     status: Optional[torch.Tensor] = None) -> torch.Tensor:
     """Y[N][Cout] = X Wd^T on the library's tensor-core GEMM with dense weights and
     no decompression (``cci_dense_linear_tc``).  Wd is the dense family's workspace
-    layout: bf16 [Cout][Cin]; fp32 the hi / lo tf32 planes [2][Cout][Cin]."""
+    layout, as ``dense_planes`` writes it."""
     _cuda_contig(X, "X")
     _cuda_contig(Wd, "Wd")
     N, Cin = X.shape

@@ -74,10 +74,13 @@ bool regtile_ptr_ok(const FwdParams &p)
 cci_status to_status(cudaError_t e) { return e == cudaSuccess ? CCI_OK : CCI_ERR_CUDA; }
 
 // workspace of the dense tensor-core family: bf16 dense weights [Cout][R], or
-// for fp32 the hi and lo tf32 planes [2][Cout][R] of 4-byte elements
+// for fp32 the two operand planes of the split (cci_common.cuh): plane 0
+// [Cout][R] of 4-byte elements, plane 1 [Cout][ceil(R / 32) * 64] of 2-byte ones
 size_t dense_ws_bytes(int dtype, int64_t Cout, int64_t R)
 {
-    return static_cast<size_t>(Cout) * static_cast<size_t>(R) * (dtype == CCI_F32 ? 8 : 2);
+    if (dtype == CCI_F32)
+        return static_cast<size_t>(Cout) * (static_cast<size_t>(R) * 4 + static_cast<size_t>((R + 31) / 32) * 128);
+    return static_cast<size_t>(Cout) * static_cast<size_t>(R) * 2;
 }
 
 bool dense_tc_shape_ok(int dtype, int G, int K, int64_t Cin, int64_t R)
@@ -572,6 +575,20 @@ cci_status cci_dense_linear_tc(const void *X, cci_dtype dtype, int64_t N, int64_
     return dense_forward(p, dtype, reinterpret_cast<cudaStream_t>(stream));
 }
 
+cci_status cci_dense_planes(const void *W, cci_dtype dtype, int64_t Cout, int64_t R, void *Wd, size_t bytes,
+                            cci_stream_t stream)
+{
+    if (!valid_dtype(dtype)) return CCI_ERR_DTYPE;
+    if (Cout < 1 || R < 1 || !mul_ok(Cout, R)) return CCI_ERR_SHAPE;
+    if (!W || !Wd) return CCI_ERR_NULL;
+    if (bytes < dense_ws_bytes(dtype, Cout, R)) return CCI_ERR_WORKSPACE;
+    if (!aligned(W, 16) || !aligned(Wd, 16) || R % (dtype == CCI_F32 ? 4 : 8) != 0) return CCI_ERR_ALIGN;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (dtype == CCI_BF16)
+        return to_status(cudaMemcpyAsync(Wd, W, static_cast<size_t>(Cout) * R * 2, cudaMemcpyDeviceToDevice, st));
+    return to_status(launch_dense_split(static_cast<const uint32_t *>(W), Cout, R, Wd, st));
+}
+
 cci_status cci_dense_conv2d_tc(const void *X, cci_dtype dtype, int64_t B, int64_t H, int64_t W, int64_t Cin,
                                const void *Wd, int64_t Cout, int KH, int KW, int stride_h, int stride_w, int pad_h,
                                int pad_w, float *Y, uint32_t *dev_status, cci_stream_t stream)
@@ -633,13 +650,13 @@ const char *cci_kernel_name(cci_dtype dtype, int64_t Cin, int64_t R, int64_t Cou
                                          "dense_tc_ws_bf16_G16_K2", "dense_tc_ws_bf16_G16_K4", "dense_tc_ws_bf16_G16_K8",
                                          "dense_tc_ws_bf16_G32_K1", "dense_tc_ws_bf16_G32_K2", "dense_tc_ws_bf16_G32_K4",
                                          "dense_tc_ws_bf16_G32_K8", "dense_tc_ws_bf16_G32_K16"};
-        static const char *names_tf[] = {"dense_tc_ws_tf32x3_G4_K1", "dense_tc_ws_tf32x3_G4_K2",
-                                         "dense_tc_ws_tf32x3_G8_K1", "dense_tc_ws_tf32x3_G8_K2",
-                                         "dense_tc_ws_tf32x3_G8_K4", "dense_tc_ws_tf32x3_G16_K1",
-                                         "dense_tc_ws_tf32x3_G16_K2", "dense_tc_ws_tf32x3_G16_K4",
-                                         "dense_tc_ws_tf32x3_G16_K8", "dense_tc_ws_tf32x3_G32_K1",
-                                         "dense_tc_ws_tf32x3_G32_K2", "dense_tc_ws_tf32x3_G32_K4",
-                                         "dense_tc_ws_tf32x3_G32_K8", "dense_tc_ws_tf32x3_G32_K16"};
+        static const char *names_tf[] = {"dense_tc_ws_f32split_G4_K1", "dense_tc_ws_f32split_G4_K2",
+                                         "dense_tc_ws_f32split_G8_K1", "dense_tc_ws_f32split_G8_K2",
+                                         "dense_tc_ws_f32split_G8_K4", "dense_tc_ws_f32split_G16_K1",
+                                         "dense_tc_ws_f32split_G16_K2", "dense_tc_ws_f32split_G16_K4",
+                                         "dense_tc_ws_f32split_G16_K8", "dense_tc_ws_f32split_G32_K1",
+                                         "dense_tc_ws_f32split_G32_K2", "dense_tc_ws_f32split_G32_K4",
+                                         "dense_tc_ws_f32split_G32_K8", "dense_tc_ws_f32split_G32_K16"};
         if (!dense_tc_shape_ok(dtype, G, K, Cin, R)) return "";
         int i = 0;
         for (int g = 4; g <= 32; g *= 2)

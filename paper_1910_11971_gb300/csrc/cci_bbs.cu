@@ -6,8 +6,8 @@
 //   bbs_pack_kernel        per (co, g): the K of largest |w|, ties to the lower
 //                          index, in increasing index (CCI's selection rule)
 //   bbs_decompress_kernel  per (co, g): the G dense weights of the group into the
-//                          workspace of the tensor-core product (bf16, or fp32 hi /
-//                          lo tf32 planes), which then runs the CCI GEMM unchanged
+//                          workspace of the tensor-core product (bf16, or the fp32
+//                          operand planes), which then runs the CCI GEMM unchanged
 //   bbs_gather_kernel      the product on CUDA cores (G dividing 32): X staged
 //                          transposed in shared memory, each (value, index) pair
 //                          reads one staged row (a warp-uniform address: no
@@ -50,13 +50,8 @@ __global__ void bbs_pack_kernel(const TB *__restrict__ W, int64_t Cout, int64_t 
     }
 }
 
-__device__ __forceinline__ uint32_t hi_bits(uint32_t x) { return x & 0xffffe000u; }
-__device__ __forceinline__ uint32_t lo_bits(uint32_t x)
-{
-    return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
-}
 
-// SPLIT: fp32 hi plane to w0, lo plane to w1; else the weights to w0.  Indices
+// SPLIT: the two fp32 operand planes (store_w_split4) at w0 and w1; else the weights to w0.  Indices
 // must be strictly increasing inside a group and < G (else CCI_ERR_INDEX).
 // GC > 0: G == GC known at compile time, the group assembled in registers and
 // written with 16-byte stores (G * element size a multiple of 16); GC == 0: any
@@ -70,7 +65,8 @@ __global__ void bbs_decompress_kernel(const TB *__restrict__ values, const uint8
     const int64_t total = Cout * ng;
     for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
          t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const int64_t base = (t / ng) * R + (t % ng) * G;
+        const int64_t row = t / ng, c0 = (t % ng) * G;  // output channel, first index of the group
+        const int64_t base = row * R + c0;
         int s = 0, prev = -1;
         bool bad = false;
         if constexpr (GC > 0) {
@@ -92,20 +88,20 @@ __global__ void bbs_decompress_kernel(const TB *__restrict__ values, const uint8
             constexpr int kV = 16 / static_cast<int>(sizeof(TB));  // elements per 16-byte store
 #pragma unroll
             for (int q = 0; q < GC / kV; ++q) {
-                uint32_t h[4], l[4];
+                uint32_t h[4];
 #pragma unroll
                 for (int e = 0; e < 4; ++e) {
-                    uint32_t word;
                     if constexpr (sizeof(TB) == 4)
-                        word = static_cast<uint32_t>(g[q * kV + e]);
+                        h[e] = static_cast<uint32_t>(g[q * kV + e]);
                     else
-                        word = static_cast<uint32_t>(g[q * kV + 2 * e]) |
+                        h[e] = static_cast<uint32_t>(g[q * kV + 2 * e]) |
                                (static_cast<uint32_t>(g[q * kV + 2 * e + 1]) << 16);
-                    h[e] = SPLIT ? hi_bits(word) : word;
-                    l[e] = SPLIT ? lo_bits(word) : 0u;
                 }
-                reinterpret_cast<uint4 *>(w0 + base)[q] = make_uint4(h[0], h[1], h[2], h[3]);
-                if constexpr (SPLIT) reinterpret_cast<uint4 *>(w1 + base)[q] = make_uint4(l[0], l[1], l[2], l[3]);
+                if constexpr (SPLIT)
+                    store_w_split4(reinterpret_cast<uint32_t *>(w0), reinterpret_cast<uint16_t *>(w1), R, row,
+                                   c0 + q * kV, h);
+                else
+                    reinterpret_cast<uint4 *>(w0 + base)[q] = make_uint4(h[0], h[1], h[2], h[3]);
             }
         } else {
             for (int j = 0; j < G; ++j) {
@@ -120,8 +116,8 @@ __global__ void bbs_decompress_kernel(const TB *__restrict__ values, const uint8
                     }
                 }
                 if constexpr (SPLIT) {
-                    w0[base + j] = hi_bits(v);
-                    w1[base + j] = lo_bits(v);
+                    store_w_split1(reinterpret_cast<uint32_t *>(w0), reinterpret_cast<uint16_t *>(w1), R, row, c0 + j,
+                                   static_cast<uint32_t>(v));
                 } else {
                     w0[base + j] = v;
                 }

@@ -45,6 +45,89 @@ __device__ __forceinline__ float bf16_bits_to_f32(uint32_t b16)
     return __uint_as_float(b16 << 16);
 }
 
+// ---- fp32 operands of the tensor-core product ----
+// An fp32 value v is split as v = hi + lo: hi is a tf32 value (fp32 bits whose
+// low 13 mantissa bits are zero), lo = v - hi exactly.  Per 32 reduction indices
+// the product takes three terms, 8 MMAs in all (x: activation, w: weight):
+//   hi(x) * hi(w)                 tf32, 4 MMAs of 8 indices (exact products)
+//   bf16(x) * bf16(lo(w))         bf16, 2 MMAs of 16 indices
+//   bf16(lo(x)) * bf16(hi(w))     bf16, 2 MMAs of 16 indices
+// The first cross term takes the whole x, so lo(x) * lo(w) is included.  Weight
+// hi is the nearest tf32 (|lo| <= 2^-11 |w|); activation hi is truncated (|lo| <
+// 2^-10 |x|, one logic op in the producers); bf16 conversions round to nearest
+// and saturate to the largest finite bf16.  Per term of the reduction the error
+// is at most |x||w| (2^-8 * 2^-11 + 2^-8 * 2^-10 (1 + 2^-11)), about
+// 5.7e-6 |x||w|, under the 1e-5 sum |x||w| tolerance before the fp32 accumulation.
+// Operand planes (weights in the workspace; activations in shared or tensor
+// memory): plane 0 holds hi as fp32 bits, [rows][R]; plane 1 holds bf16 pairs
+// [rows][ceil(R / 32) * 64]: for chunk c of 32 indices, element c * 64 + t is the
+// first bf16 operand of index c * 32 + t (t < 32) and element c * 64 + 32 + t
+// the second (bf16(hi(w)) and bf16(lo(w)) for weights, bf16(x) and bf16(lo(x))
+// for activations); indices past R hold zeros.
+__device__ __forceinline__ uint32_t tf32_trunc(uint32_t v) { return v & 0xffffe000u; }
+
+// nearest tf32 (ties to even); a finite value that would round up into the
+// exponent of inf keeps its truncation, inf and NaN are truncated
+__device__ __forceinline__ uint32_t tf32_rn(uint32_t v)
+{
+    const uint32_t r = (v + 0x0fffu + ((v >> 13) & 1u)) & 0xffffe000u;
+    return (r & 0x7f800000u) == 0x7f800000u ? (v & 0xffffe000u) : r;
+}
+
+// bf16 pair (e0 in the low half), round to nearest, saturating at the largest
+// finite bf16
+__device__ __forceinline__ uint32_t bf16x2_rn_sat(float e0, float e1)
+{
+    uint32_t r;
+    asm("cvt.rn.satfinite.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(e1), "f"(e0));
+    return r;
+}
+
+// 16-bit elements of plane 1 per row for R reduction indices
+__device__ __forceinline__ int64_t split_plane1_row(int64_t R) { return (R + 31) / 32 * 64; }
+
+// writes weights w[0..3] of row `row` at indices r0 .. r0 + 3 (r0 % 4 == 0) into
+// the two weight planes; the writer of the last indices (r0 + 4 == R) also
+// zeroes the rest of plane 1's last chunk
+__device__ __forceinline__ void store_w_split4(uint32_t *plane0, uint16_t *plane1, int64_t R, int64_t row,
+                                               int64_t r0, const uint32_t (&w)[4])
+{
+    uint32_t h[4];
+    float l[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        h[e] = tf32_rn(w[e]);
+        l[e] = __uint_as_float(w[e]) - __uint_as_float(h[e]);
+    }
+    __stcg(reinterpret_cast<uint4 *>(plane0 + row * R + r0), make_uint4(h[0], h[1], h[2], h[3]));
+    uint16_t *q = plane1 + row * split_plane1_row(R) + (r0 >> 5) * 64 + (r0 & 31);
+    __stcg(reinterpret_cast<uint2 *>(q), make_uint2(bf16x2_rn_sat(__uint_as_float(h[0]), __uint_as_float(h[1])),
+                                                    bf16x2_rn_sat(__uint_as_float(h[2]), __uint_as_float(h[3]))));
+    __stcg(reinterpret_cast<uint2 *>(q + 32), make_uint2(bf16x2_rn_sat(l[0], l[1]), bf16x2_rn_sat(l[2], l[3])));
+    if (r0 + 4 == R && (R & 31) != 0) {
+        for (int t = static_cast<int>(R & 31); t < 32; t += 4) {
+            uint16_t *z = plane1 + row * split_plane1_row(R) + (r0 >> 5) * 64 + t;
+            __stcg(reinterpret_cast<uint2 *>(z), make_uint2(0u, 0u));
+            __stcg(reinterpret_cast<uint2 *>(z + 32), make_uint2(0u, 0u));
+        }
+    }
+}
+
+// the same for one weight at any index r (2-byte plane-1 stores); the writer of
+// index R - 1 zeroes the rest of the last chunk
+__device__ __forceinline__ void store_w_split1(uint32_t *plane0, uint16_t *plane1, int64_t R, int64_t row,
+                                               int64_t r, uint32_t w)
+{
+    const uint32_t h = tf32_rn(w);
+    const float l = __uint_as_float(w) - __uint_as_float(h);
+    plane0[row * R + r] = h;
+    uint16_t *q = plane1 + row * split_plane1_row(R) + (r >> 5) * 64;
+    q[r & 31] = static_cast<uint16_t>(bf16x2_rn_sat(__uint_as_float(h), 0.0f));
+    q[32 + (r & 31)] = static_cast<uint16_t>(bf16x2_rn_sat(l, 0.0f));
+    if (r == R - 1)
+        for (int t = static_cast<int>((r & 31) + 1); t < 32; ++t) q[t] = q[32 + t] = 0;
+}
+
 // Packed fp32 FMA on two lanes: d = a * b + d, element-wise on (lo, hi) pairs,
 // each element an IEEE binary32 fused multiply-add with one rounding.
 __device__ __forceinline__ void ffma2(unsigned long long &d, unsigned long long a,

@@ -35,9 +35,9 @@ cudaError_t launch_wait_probe(uint32_t *status, int arrive, cudaStream_t stream)
 // ===========================================================================
 // One-pass decompression of the packed weights into the workspace of
 // CCI_ALGO_DENSE_TC_WS: the dense W[Cout][R] (bf16, bit for bit), or for fp32
-// layers its hi and lo tf32 planes [2][Cout][R] (hi = w with the low 13 mantissa
-// bits cleared, exactly a tf32 value; lo = w - hi, exact in fp32) for the
-// three-pass product hi*hi + hi*lo + lo*hi.
+// layers its two operand planes (store_w_split4: hi as a tf32 value, then the
+// bf16 pairs of hi and lo per 32-wide chunk) for the product
+// hi(x) hi(w) + bf16(x) bf16(lo(w)) + bf16(lo(x)) bf16(hi(w)).
 // One block per (group gi, slab of kSlab columns r): each thread scatters the K
 // kept weights of one column into a zeroed [G][kSlab] tile in shared memory,
 // then the block writes the G rows of the slab with 16-byte stores.  Index sets
@@ -48,15 +48,9 @@ namespace dc {
 
 constexpr int kSlab = 256;  // columns r per block (= threads per block)
 
-__device__ __forceinline__ uint32_t hi_bits(uint32_t x) { return x & 0xffffe000u; }
-__device__ __forceinline__ uint32_t lo_bits(uint32_t x)
-{
-    return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
-}
-
-// T = uint16_t (bf16 bits) or uint32_t (fp32 bits); SPLIT: write hi to w0 and
-// lo to w1 (fp32 only), else the weights to w0.  R must be a multiple of the
-// elements per 16 bytes.
+// T = uint16_t (bf16 bits) or uint32_t (fp32 bits); SPLIT: write the two operand
+// planes (fp32 only: plane 0 at w0, plane 1 at w1), else the weights to w0.  R
+// must be a multiple of the elements per 16 bytes.
 template <typename T, int G, int K, bool SPLIT>
 __global__ void __launch_bounds__(kSlab) decompress_kernel(const T *__restrict__ values,
                                                            const uint8_t *__restrict__ idx, int64_t R,
@@ -97,8 +91,8 @@ __global__ void __launch_bounds__(kSlab) decompress_kernel(const T *__restrict__
         const uint4 x = *reinterpret_cast<const uint4 *>(&tile[j][c * V]);
         const int64_t off = (gi * G + j) * R + rr;
         if constexpr (SPLIT) {
-            __stcg(reinterpret_cast<uint4 *>(w0 + off), make_uint4(hi_bits(x.x), hi_bits(x.y), hi_bits(x.z), hi_bits(x.w)));
-            __stcg(reinterpret_cast<uint4 *>(w1 + off), make_uint4(lo_bits(x.x), lo_bits(x.y), lo_bits(x.z), lo_bits(x.w)));
+            const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+            store_w_split4(reinterpret_cast<uint32_t *>(w0), reinterpret_cast<uint16_t *>(w1), R, gi * G + j, rr, w);
         } else {
             __stcg(reinterpret_cast<uint4 *>(w0 + off), x);
         }
@@ -186,6 +180,35 @@ cudaError_t launch_dense_tc_ws(const FwdParams &p, int dtype, int G, int K, cuda
     CCI_TC_CASE(32, 1) CCI_TC_CASE(32, 2) CCI_TC_CASE(32, 4) CCI_TC_CASE(32, 8) CCI_TC_CASE(32, 16)
 #undef CCI_TC_CASE
     return cudaErrorNotSupported;
+}
+
+namespace dc {
+
+// one thread per 4 consecutive r of one row: the dense weights into the planes
+__global__ void __launch_bounds__(256) dense_split_kernel(const uint32_t *__restrict__ W, int64_t Cout, int64_t R,
+                                                          uint32_t *plane0, uint16_t *plane1)
+{
+    const int64_t q = R / 4;
+    for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < Cout * q;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t row = t / q, r0 = (t - row * q) * 4;
+        const uint4 x = __ldg(reinterpret_cast<const uint4 *>(W + row * R + r0));
+        const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+        store_w_split4(plane0, plane1, R, row, r0, w);
+    }
+}
+
+}  // namespace dc
+
+cudaError_t launch_dense_split(const uint32_t *W, int64_t Cout, int64_t R, void *planes, cudaStream_t stream)
+{
+    uint32_t *p0 = static_cast<uint32_t *>(planes);
+    uint16_t *p1 = reinterpret_cast<uint16_t *>(p0 + Cout * R);
+    const int64_t work = Cout * (R / 4);
+    const int64_t blocks = (work + 255) / 256;
+    dc::dense_split_kernel<<<static_cast<unsigned>(blocks < 65536 ? blocks : 65536), 256, 0, stream>>>(W, Cout, R, p0,
+                                                                                                      p1);
+    return cudaGetLastError();
 }
 
 bool dense_tc_supported(int dtype, int G, int K)

@@ -5,12 +5,15 @@
 // tile [128 n][BN co], BN in {64, 128, 256}, two BN-column accumulators:
 //   bf16:  A = activation tile [128 n][64 r], B = weight tile [BN co][64 r], one
 //          kind::f16 MMA per 16 r.
-//   tf32x3 (fp32 layers): every operand split as hi + lo (hi: the low 13 mantissa
-//          bits cleared, exactly a tf32 value; lo = x - hi exactly); per 8 r three
-//          kind::tf32 MMAs lo*hi + hi*lo + hi*hi; 32 r per stage, planes A hi,
-//          A lo, B hi, B lo.
+//   fp32 layers: every operand split as hi + lo (hi a tf32 value, lo = v - hi
+//          exactly; cci_common.cuh), 32 r per stage and 8 MMAs: hi(x) hi(w) as
+//          four kind::tf32 MMAs, bf16(x) bf16(lo(w)) and bf16(lo(x)) bf16(hi(w))
+//          as two kind::f16 MMAs each; operand plane 0 holds hi, plane 1 the
+//          bf16 pairs (a 128-byte row per stage: 32 bf16 of one term, then 32 of
+//          the other).
 // Operands (all K-major, 128-byte swizzle, 1024-byte aligned stage buffers):
-//   weights      TMA from the workspace planes (tensor maps over [Cout][R]);
+//   weights      TMA from the workspace planes (tensor maps over [Cout][R], fp32
+//                plane 1 over [Cout][ceil(R / 32) * 64] bf16);
 //   activations  one of (the template's ASRC):
 //     kA2d      products: TMA over X[N][Cin];
 //     kA4d      stride-1 convolutions with Cin a multiple of the stage depth:
@@ -29,9 +32,10 @@
 //     kAGather  other convolutions: the producer warps gather rows (cp.async for
 //               bf16; registers, two stages ahead, then the hi/lo split, for fp32).
 //   fp32 activations copied by TMA land raw in shared memory; the producer warps
-//   split each row into hi and lo and store both in tensor memory (per stage 64
-//   columns after the accumulators), from where the MMAs read A: the three
-//   passes then read only B from shared memory.
+//   split each row and store its two planes in tensor memory (per stage 64
+//   columns after the accumulators: 32 of tf32 hi, 16 of bf16 pairs of x, 16 of
+//   lo(x)), from where the MMAs read A: the eight MMAs then read only B from
+//   shared memory.
 // Weights (the template's PK):
 //   PK = false  the dense workspace planes written by the one-pass decompression;
 //   PK = true   the packed (value, index) pairs themselves (bf16 only, no
@@ -105,7 +109,7 @@ struct Cfg {
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
     static constexpr bool kHalo = ASRC == kAHalo;  // A: per-chunk halo buffers, stages hold B only
     static_assert(!kHalo || (!TF32 && CG == 1), "halo copies: bf16 single-CTA tiles");
-    // raw fp32 A by TMA; the producers split it into hi / lo and write both to
+    // raw fp32 A by TMA; the producers split it into its two planes and write both to
     // tensor memory, where the MMAs read A (no A planes in shared memory)
     static constexpr bool kARaw = TF32 && ASRC != kAGather;
     static constexpr int kAPlanes = (TF32 && !kARaw) ? 2 : 1, kBPlanes = TF32 ? 2 : 1;
@@ -126,7 +130,7 @@ struct Cfg {
     static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - kYBufs * kYBuf - 1024;
     static constexpr int kStagesFit = (kBudget / kStage) < tc::kMaxStages ? (kBudget / kStage) : tc::kMaxStages;
     static constexpr int kStages = kHalo ? kHaloStages : kStagesFit;
-    // accumulators: 2 x kN columns; kARaw adds per stage A hi and A lo (32 columns each)
+    // accumulators: 2 x kN columns; kARaw adds per stage the A planes (32 + 32 columns)
     static constexpr int kAColBase = 2 * kN;
     static constexpr int kTmemCols = kARaw ? 512 : 2 * kN;
     static constexpr size_t kSmem =
@@ -136,6 +140,9 @@ struct Cfg {
                                        | (TF32 ? (2u << 7) | (2u << 10) : (1u << 7) | (1u << 10))  // tf32 / bf16
                                        | (static_cast<uint32_t>(kN >> 3) << 17) |
                                        (static_cast<uint32_t>((kM * CG) >> 4) << 24);
+    // fp32 layers: the bf16 MMAs of the split's cross terms
+    static constexpr uint32_t kIdescB = (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(kN >> 3) << 17) |
+                                        (static_cast<uint32_t>((kM * CG) >> 4) << 24);
     static_assert(kSmem <= kMaxSmemPerBlock, "stage buffers over the per-block limit");
     static_assert(kStages >= 3, "too few pipeline stages");
     static_assert(kTmemCols == 128 || kTmemCols == 256 || kTmemCols == 512, "TMEM allocation not a power of 2");
@@ -180,40 +187,43 @@ __device__ __forceinline__ void mma(uint32_t d, uint64_t a, uint64_t b, uint32_t
     }
 }
 
-// ---- one pipeline stage of three-pass tf32 MMAs, A in tensor memory ----
-// Per 8 r (k = 0..3 of a 32-wide stage): lo(A) * hi(B) + hi(A) * lo(B) + hi(A) * hi(B),
-// A hi at TMEM column a0 + 8k and A lo 32 columns on, B hi at descriptor bh + 2k
-// (32 bytes per step) and B lo one plane (kBLo 16-byte units) further.  Every
-// lane of the MMA warp executes the block; the lane with `issue` set issues the
-// twelve MMAs and commits the stage to `bar`.  One block with the addresses
+// ---- one pipeline stage of the fp32 product (8 MMAs), A in tensor memory ----
+// The three terms of the split (cci_common.cuh) over a 32-wide stage:
+//   hi(x) hi(w)           4 kind::tf32 MMAs: A at TMEM columns a0 + 8k, B plane 0
+//                         at descriptor b0 + 2k (32 bytes per 8 indices);
+//   bf16(x) bf16(lo(w))   2 kind::f16 MMAs: A at a0 + 32 + 8k (two bf16 per
+//                         column), B plane 1 (kB1 16-byte units on) at + 4 + 2k;
+//   bf16(lo(x)) bf16(hi(w)) 2 kind::f16 MMAs: A at a0 + 48 + 8k, B plane 1 at + 2k.
+// Every lane of the MMA warp executes the block; the lane with `issue` set issues
+// the eight MMAs and commits the stage to `bar`.  One block with the addresses
 // formed by adds: the MMA warp's instruction stream per stage bounds this
-// product (measured on GB300 with clock stamps: the MMAs waited ~130 cycles per
-// stage for their operands while the issue of a stage took ~850).
-template <uint32_t kIdesc, uint32_t kBLo>
-__device__ __forceinline__ void stage_tf32x3(uint32_t d, uint32_t a0, uint64_t bh, uint32_t acc0, uint32_t issue,
-                                             uint32_t bar)
+// product (measured on GB300 with clock stamps for the three-pass form of twelve
+// MMAs: operands waited for ~130 cycles per stage, the issue of a stage took ~850).
+template <uint32_t kIdescT, uint32_t kIdescB, uint32_t kB1>
+__device__ __forceinline__ void stage_tf32_split(uint32_t d, uint32_t a0, uint64_t b0, uint32_t acc0, uint32_t issue,
+                                                 uint32_t bar)
 {
     asm volatile(
-        "{\n.reg .pred pe, pa, pt;\n.reg .b32 ah, al;\n.reg .b64 bh, bl;\n"
+        "{\n.reg .pred pe, pa, pt;\n.reg .b32 a;\n.reg .b64 b;\n"
         "setp.ne.b32 pe, %4, 0;\nsetp.ne.b32 pa, %3, 0;\nsetp.eq.b32 pt, 0, 0;\n"
-        "add.u32 al, %1, 32;\nadd.s64 bl, %2, %6;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], %2, %5, pa;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], bl, %5, pt;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %5, pt;\n"
-        "add.u32 ah, %1, 8;\nadd.u32 al, %1, 40;\nadd.s64 bh, %2, 2;\nadd.s64 bl, bl, 2;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], bh, %5, pt;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bl, %5, pt;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bh, %5, pt;\n"
-        "add.u32 ah, %1, 16;\nadd.u32 al, %1, 48;\nadd.s64 bh, %2, 4;\nadd.s64 bl, bl, 2;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], bh, %5, pt;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bl, %5, pt;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bh, %5, pt;\n"
-        "add.u32 ah, %1, 24;\nadd.u32 al, %1, 56;\nadd.s64 bh, %2, 6;\nadd.s64 bl, bl, 2;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [al], bh, %5, pt;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bl, %5, pt;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [ah], bh, %5, pt;\n"
-        "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%7];\n}\n" ::"r"(d),
-        "r"(a0), "l"(bh), "r"(acc0), "r"(issue), "n"(kIdesc), "n"(static_cast<uint64_t>(kBLo)), "r"(bar)
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [%1], %2, %5, pa;\n"
+        "add.u32 a, %1, 8;\nadd.s64 b, %2, 2;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [a], b, %5, pt;\n"
+        "add.u32 a, %1, 16;\nadd.s64 b, %2, 4;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [a], b, %5, pt;\n"
+        "add.u32 a, %1, 24;\nadd.s64 b, %2, 6;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::tf32 [%0], [a], b, %5, pt;\n"
+        "add.u32 a, %1, 32;\nadd.s64 b, %2, %7;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %6, pt;\n"
+        "add.u32 a, %1, 40;\nadd.s64 b, b, 2;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %6, pt;\n"
+        "add.u32 a, %1, 48;\nadd.s64 b, %2, %8;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %6, pt;\n"
+        "add.u32 a, %1, 56;\nadd.s64 b, b, 2;\n"
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %6, pt;\n"
+        "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%9];\n}\n" ::"r"(d),
+        "r"(a0), "l"(b0), "r"(acc0), "r"(issue), "n"(kIdescT), "n"(kIdescB),
+        "n"(static_cast<uint64_t>(kB1 + 4)), "n"(static_cast<uint64_t>(kB1)), "r"(bar)
         : "memory");
 }
 
@@ -384,10 +394,31 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 {
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
 }
-__device__ __forceinline__ uint32_t hi_bits(uint32_t x) { return x & 0xffffe000u; }
-__device__ __forceinline__ uint32_t lo_bits(uint32_t x)
+__device__ __forceinline__ void st_shared_v2(uint32_t addr, uint32_t a, uint32_t b)
 {
-    return __float_as_uint(__uint_as_float(x) - __uint_as_float(hi_bits(x)));
+    asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(a), "r"(b) : "memory");
+}
+
+// the gathered fp32 activations x[0..3] of one 16-byte chunk of an A row, split
+// into the operand planes (cci_common.cuh): the tf32 hi into plane 0 (at
+// plane0), the bf16 pairs of x and lo(x) into plane 1 (at plane1), 8 bytes each
+// at their places of the 128-byte-swizzled row
+__device__ __forceinline__ void st_shared_x_split(uint32_t plane0, uint32_t plane1, int row, int chunk, uint4 v)
+{
+    const uint32_t x[4] = {v.x, v.y, v.z, v.w};
+    uint32_t h[4];
+    float l[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        h[e] = tf32_trunc(x[e]);
+        l[e] = __uint_as_float(x[e]) - __uint_as_float(h[e]);
+    }
+    st_shared_v4(plane0 + sw_chunk(row, chunk), h[0], h[1], h[2], h[3]);
+    const uint32_t half = static_cast<uint32_t>(chunk & 1) * 8;
+    st_shared_v2(plane1 + sw_chunk(row, chunk >> 1) + half,
+                 bf16x2_rn_sat(__uint_as_float(x[0]), __uint_as_float(x[1])),
+                 bf16x2_rn_sat(__uint_as_float(x[2]), __uint_as_float(x[3])));
+    st_shared_v2(plane1 + sw_chunk(row, 4 + (chunk >> 1)) + half, bf16x2_rn_sat(l[0], l[1]), bf16x2_rn_sat(l[2], l[3]));
 }
 
 
@@ -795,7 +826,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                         tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes + (C::kATma ? a_bytes : 0u));
                         tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
                         if constexpr (C::kBPlanes > 1)
-                            tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                            tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * 64, static_cast<int>(co0), &S->full[s]);  // plane 1: 64 bf16 per stage
                     }
                     if constexpr (ASRC == kA2d) {
                         tc::tma_load_2d(st, &tmA.m[0], ks * kKS, static_cast<int>(mt * kM), abar);
@@ -1060,13 +1091,14 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                             tc::mbar_arrive(&S->full[(it - kLag) % kStages]);
                         }
                     } else if constexpr (C::kARaw) {
-                        // the raw fp32 tile landed: row m = pt, split into hi and lo in
-                        // registers and written to this stage's A columns of tensor
-                        // memory (lane m; warp 4 + q owns lanes 32q..32q+31)
+                        // the raw fp32 tile landed: row m = pt, split in registers (the
+                        // operand planes of cci_common.cuh: hi(x) as tf32, then the bf16
+                        // pairs of x and lo(x)) and written to this stage's 64 A columns
+                        // of tensor memory (lane m; warp 4 + q owns lanes 32q..32q+31)
                         ok = tc::mbar_wait(&S->aux[s], (it / kStages) & 1, abort, p.status);
                         ok = __all_sync(0xffffffffu, ok);
                         if (!ok) break;
-                        uint32_t hv[32], lv[32];
+                        uint32_t hv[32], bv[32];
 #pragma unroll
                         for (int q = 0; q < 8; ++q) {
                             uint4 v;
@@ -1074,31 +1106,28 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                                          : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                                          : "r"(st + sw_chunk(pt, q))
                                          : "memory");
-                            hv[4 * q] = hi_bits(v.x);
-                            hv[4 * q + 1] = hi_bits(v.y);
-                            hv[4 * q + 2] = hi_bits(v.z);
-                            hv[4 * q + 3] = hi_bits(v.w);
-                            lv[4 * q] = lo_bits(v.x);
-                            lv[4 * q + 1] = lo_bits(v.y);
-                            lv[4 * q + 2] = lo_bits(v.z);
-                            lv[4 * q + 3] = lo_bits(v.w);
+                            const uint32_t x[4] = {v.x, v.y, v.z, v.w};
+                            float l[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) {
+                                hv[4 * q + e] = tf32_trunc(x[e]);
+                                l[e] = __uint_as_float(x[e]) - __uint_as_float(hv[4 * q + e]);
+                            }
+                            bv[2 * q] = bf16x2_rn_sat(__uint_as_float(x[0]), __uint_as_float(x[1]));
+                            bv[2 * q + 1] = bf16x2_rn_sat(__uint_as_float(x[2]), __uint_as_float(x[3]));
+                            bv[16 + 2 * q] = bf16x2_rn_sat(l[0], l[1]);
+                            bv[16 + 2 * q + 1] = bf16x2_rn_sat(l[2], l[3]);
                         }
                         const uint32_t ta = tmem + (static_cast<uint32_t>((warp - 4) * 32) << 16) +
                                             static_cast<uint32_t>(C::kAColBase + s * 64);
                         tc::tmem_st32(ta, hv);
-                        tc::tmem_st32(ta + 32, lv);
+                        tc::tmem_st32(ta + 32, bv);
                         asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
                         asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
                         tc::mbar_arrive(&S->full[s]);
                     } else {
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            const uint32_t o = sw_chunk(rowb + 16 * i, chunk);
-                            st_shared_v4(st + o, hi_bits(xa[i].x), hi_bits(xa[i].y), hi_bits(xa[i].z),
-                                         hi_bits(xa[i].w));
-                            st_shared_v4(st + C::kAPlane + o, lo_bits(xa[i].x), lo_bits(xa[i].y), lo_bits(xa[i].z),
-                                         lo_bits(xa[i].w));
-                        }
+                        for (int i = 0; i < 8; ++i) st_shared_x_split(st, st + C::kAPlane, rowb + 16 * i, chunk, xa[i]);
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                         tc::mbar_arrive(&S->full[s]);
 #pragma unroll
@@ -1151,7 +1180,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                         ok = tc::mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
                         if (!ok) break;
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                        stage_tf32x3<C::kIdesc, (C::kBPlane >> 4)>(
+                        stage_tf32_split<C::kIdesc, C::kIdescB, (C::kBPlane >> 4)>(
                             d, tmem + static_cast<uint32_t>(C::kAColBase + s * 64),
                             bdesc0 + static_cast<uint64_t>(s) * (C::kStage >> 4) + (C::kBOff >> 4), ks > 0 ? 1u : 0u,
                             1u, empty0 + 8u * s);
@@ -1246,15 +1275,16 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                     const uint32_t st = base + s * C::kStage;
                     const uint32_t bst = st + C::kBOff;
                     if constexpr (TF32) {
+                        // the split's three terms (stage_tf32_split), A planes in shared memory
 #pragma unroll
-                        for (int k = 0; k < kKS / 8; ++k) {
-                            const uint64_t ah = tc::sw128_desc(st + k * 32);
-                            const uint64_t al = tc::sw128_desc(st + C::kAPlane + k * 32);
-                            const uint64_t bh = tc::sw128_desc(bst + k * 32);
-                            const uint64_t bl = tc::sw128_desc(bst + C::kBPlane + k * 32);
-                            mma<TF32, CG>(d, al, bh, C::kIdesc, (ks > 0 || k > 0) ? 1u : 0u);
-                            mma<TF32, CG>(d, ah, bl, C::kIdesc, 1u);
-                            mma<TF32, CG>(d, ah, bh, C::kIdesc, 1u);
+                        for (int k = 0; k < 4; ++k)
+                            mma<true, 1>(d, tc::sw128_desc(st + k * 32), tc::sw128_desc(bst + k * 32), C::kIdesc,
+                                         (ks > 0 || k > 0) ? 1u : 0u);
+#pragma unroll
+                        for (int k = 0; k < 2; ++k) {
+                            const uint32_t a1 = st + C::kAPlane + k * 32, b1 = bst + C::kBPlane + k * 32;
+                            mma<false, 1>(d, tc::sw128_desc(a1), tc::sw128_desc(b1 + 64), C::kIdescB, 1u);
+                            mma<false, 1>(d, tc::sw128_desc(a1 + 64), tc::sw128_desc(b1), C::kIdescB, 1u);
                         }
                     } else if constexpr (CG == 2) {
 #pragma unroll
@@ -1559,8 +1589,11 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &t
     const int wbox[2] = {C::kKS, C::kBRows};
     if (!PK && !make_map(&tmB0, p.wdense, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
     if (!PK && C::kBPlanes > 1) {
-        const char *lo = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
-        if (!make_map(&tmB1, lo, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
+        // fp32: plane 1 of the split, bf16 [Cout][ceil(R / 32) * 64], one 128-byte row per stage
+        const char *pl1 = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
+        const int64_t dims1[2] = {(p.R + 31) / 32 * 64, p.Cout};
+        const int box1[2] = {64, C::kBRows};
+        if (!make_map(&tmB1, pl1, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, 2, dims1, box1)) return cudaErrorInvalidValue;
     }
     // output rows of 128 bytes: 32 fp32 or 64 bf16 channels
     const CUtensorMapDataType ydt = p.out_bf16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;

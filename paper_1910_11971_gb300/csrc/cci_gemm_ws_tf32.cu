@@ -1,5 +1,6 @@
-// cci_gemm_ws_tf32.cu -- fp32 layers of the workspace family (three-pass tf32
-// products): the kernel configurations and the choice among them.
+// cci_gemm_ws_tf32.cu -- fp32 layers of the workspace family (the split product:
+// tf32 hi*hi plus bf16 cross terms): the kernel configurations and the choice
+// among them.
 #include "cci_gemm_ws.cuh"
 
 namespace cci {

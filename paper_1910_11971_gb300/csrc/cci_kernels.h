@@ -24,11 +24,13 @@ cudaError_t launch_wait_probe(uint32_t *status, int arrive, cudaStream_t stream)
 // (G, K) pairs of the workspace tensor-core family
 bool dense_tc_supported(int dtype, int G, int K);
 // decompress once into p.wdense and copy B tiles from it (bf16: dense [Cout][R];
-// fp32: hi and lo tf32 planes [2][Cout][R], three-pass tf32 product)
+// fp32: the two operand planes of the split, cci_common.cuh)
 cudaError_t launch_dense_tc_ws(const FwdParams &p, int dtype, int G, int K, cudaStream_t stream);
+// dense fp32 W[Cout][R] (R % 4 == 0, 16-byte aligned) into the operand planes at planes
+cudaError_t launch_dense_split(const uint32_t *W, int64_t Cout, int64_t R, void *planes, cudaStream_t stream);
 
 // dense product on the tensor cores from the decompressed workspace p.wdense
-// (cci_gemm_ws_*.cu): bf16 dense [Cout][R], or fp32 hi / lo tf32 planes [2][Cout][R]
+// (cci_gemm_ws_*.cu): bf16 dense [Cout][R], or the fp32 operand planes
 cudaError_t launch_gemm_ws(const FwdParams &p, int dtype, cudaStream_t stream);
 cudaError_t launch_gemm_ws_bf16(const FwdParams &p, cudaStream_t stream);
 cudaError_t launch_gemm_ws_tf32(const FwdParams &p, cudaStream_t stream);

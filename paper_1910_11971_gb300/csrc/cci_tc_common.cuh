@@ -17,7 +17,7 @@ constexpr int kMaxHalo = 4;  // halo buffers of a 3x3 convolution tile ring
 struct Smem {
     uint64_t full[kMaxStages];
     uint64_t empty[kMaxStages];
-    uint64_t aux[kMaxStages];  // per-stage barrier of a second copy (tf32x3: raw activation tile landed)
+    uint64_t aux[kMaxStages];  // per-stage barrier of a second copy (fp32: raw activation tile landed)
     uint64_t tmem_full[2];
     uint64_t tmem_empty[2];
     uint64_t drain;

@@ -129,8 +129,8 @@ def test_algo_dense_tc_names(lib):
     # the workspace one for K = 8
     assert cci.kernel_name(torch.bfloat16, 16, 16, 16, 8, 2) in ("dense_tc_fused_bf16_G8_K2", "dense_tc_ws_bf16_G8_K2")
     assert cci.kernel_name(torch.bfloat16, 16, 16, 64, 32, 8) == "dense_tc_ws_bf16_G32_K8"
-    # fp32: the workspace family (three-pass tf32) with a workspace; CUDA-core kernels without one
-    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2) == "dense_tc_ws_tf32x3_G8_K2"
+    # fp32: the workspace family (tf32 hi*hi plus bf16 cross terms) with a workspace; CUDA-core kernels without one
+    assert cci.kernel_name(torch.float32, 256, 256, 1024, 8, 2) == "dense_tc_ws_f32split_G8_K2"
 
 
 def test_kernel_names(lib):
@@ -152,7 +152,7 @@ def test_workspace_rules(lib):
     assert cci.workspace_size(cci.ALGO_EXPAND, torch.bfloat16, 256, 64) == 0
     assert cci.workspace_size(cci.ALGO_AUTO, torch.float32, 256, 64) == 256 * 64 * 8
     assert cci.workspace_size(ws, torch.float32, 256, 64) == 256 * 64 * 8
-    assert cci.kernel_name(torch.float32, 64, 64, 256, 8, 2, ws) == "dense_tc_ws_tf32x3_G8_K2"
+    assert cci.kernel_name(torch.float32, 64, 64, 256, 8, 2, ws) == "dense_tc_ws_f32split_G8_K2"
     assert cci.kernel_name(torch.float32, 64, 64, 256, 8, 2, cci.ALGO_DENSE_TC) == ""
     assert cci.workspace_size(cci.ALGO_AUTO, torch.bfloat16, 256, 64) == 256 * 64 * 2
     # the family needs a workspace: rejected before any launch (no device needed)

@@ -572,29 +572,29 @@ def test_auto_with_workspace_uses_dense_tc_ws(dev):
 
 
 # ---------------------------------------------------------------------------
-# fp32 on the tensor cores: three-pass tf32 product through the workspace family
+# fp32 on the tensor cores: the split product (tf32 hi*hi plus bf16 cross terms) through the workspace family
 # ---------------------------------------------------------------------------
 F32_DENSE = [(128, 64, 128, 8, 2), (1, 16, 128, 8, 2), (200, 36, 200, 4, 1), (300, 132, 384, 16, 4),
              (515, 64, 96, 32, 8), (129, 256, 1024, 8, 2), (77, 12, 64, 16, 8)]
 
 
 @pytest.mark.parametrize("case", F32_DENSE, ids=lambda c: "N{}_C{}x{}_G{}K{}".format(*c))
-def test_tf32x3_small(dev, case):
+def test_f32split_small(dev, case):
     N, Cin, Cout, G, K = case
     X, W = wl.random_small(N * 5 + Cin, "f32", N, Cin, Cout)
-    assert cci.kernel_name(F32, Cin, Cin, Cout, G, K, cci.ALGO_DENSE_TC_WS).startswith("dense_tc_ws_tf32x3")
+    assert cci.kernel_name(F32, Cin, Cin, Cout, G, K, cci.ALGO_DENSE_TC_WS).startswith("dense_tc_ws_f32split")
     Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC_WS)
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.linear(f64(X), Wd, mask)
     assert_within_tol(f64(Y), Yo, S, str(case))
 
 
-@pytest.mark.parametrize("algo", [cci.ALGO_DENSE_TC_WS, cci.ALGO_GENERIC], ids=["tf32x3", "generic"])
+@pytest.mark.parametrize("algo", [cci.ALGO_DENSE_TC_WS, cci.ALGO_GENERIC], ids=["f32split", "generic"])
 def test_fp32_wide_exponent_range(dev, algo):
     """Every activation row and every group of G output channels of W carries its
     own power-of-two scale (2^-30 .. 2^30), so the per-output scale S spans ~35 orders of
     magnitude: the product must hold |err| <= 1e-5 * S for each output (no absolute
-    error floor; for the three-pass tf32 split, hi and lo keep fp32's exponent
+    error floor; for the split product, hi, lo and their bf16 forms keep fp32's exponent
     range)."""
     N, Cin, Cout, G, K = 700, 256, 256, 8, 2
     g = torch.Generator().manual_seed(2024)
@@ -611,7 +611,7 @@ def test_fp32_wide_exponent_range(dev, algo):
     assert_within_tol(f64(Y), Yo, S, "fp32 wide exponent range")
 
 
-def test_tf32x3_bottleneck_full(dev):
+def test_f32split_bottleneck_full(dev):
     case = wl.BOTTLENECK_1X1
     X, W = wl.linear_inputs(case)
     Y = run_linear(dev, X, W, case.G, case.K, cci.ALGO_DENSE_TC_WS)
@@ -619,13 +619,13 @@ def test_tf32x3_bottleneck_full(dev):
     rows = sample_rows(case.N, 2048, seed=3)
     _, _, Wd, mask = oracle_reference(W, case.G, case.K)
     Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
-    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name + " tf32x3")
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, case.name + " f32split")
 
 
 @pytest.mark.parametrize("case", [c for c in CONV_SMALL if c[-1] == "f32" and c[3] % 4 == 0 and c[9] in (4, 8, 16, 32)
                                   and (c[10] & (c[10] - 1)) == 0 and c[10] <= c[9] // 2],
                          ids=lambda c: "B{}_{}x{}_{}to{}_k{}x{}_s{}_p{}_G{}K{}_{}".format(*c))
-def test_tf32x3_conv_small(dev, case):
+def test_f32split_conv_small(dev, case):
     B, H, Wi, Cin, Cout, KH, KW, stride, pad, G, K, dtype = case
     g = torch.Generator().manual_seed(B * 13 + Cin)
     X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0)
@@ -769,22 +769,22 @@ def test_pair_tiles_conv(dev, B, H, Cin, Cout, stride):
         assert_within_tol(Yg, Yo, S, f"pair conv B={B} H={H} s={stride} image {b}")
 
 
-# fp32 layers (three tf32 passes) with long reductions: odd M tile counts,
+# fp32 layers (the split product) with long reductions: odd M tile counts,
 # ragged reductions and N tails, both N tiles, 2-D and 4-D copies, checked on
 # sampled outputs (products) or every output (convolutions).
 @pytest.mark.parametrize("N,Cin,Cout,G,K", [(16429, 256, 1024, 8, 2), (5000, 300, 192, 16, 4), (300, 512, 64, 4, 1)])
-def test_tf32x3_long_reduction_product(dev, N, Cin, Cout, G, K):
+def test_f32split_long_reduction_product(dev, N, Cin, Cout, G, K):
     X, W = wl.random_small(N + Cin + 1, "f32", N, Cin, Cout)
     Y = run_linear(dev, X, W, G, K, cci.ALGO_DENSE_TC_WS)
     assert torch.isfinite(Y).all()
     rows = np.unique(np.concatenate([sample_rows(N, 768, seed=N), np.arange(N - 200, N)]))
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.linear(f64(X[rows]), Wd, mask)
-    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, f"tf32x3 product {N}x{Cin}->{Cout}")
+    assert_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yo, S, f"f32split product {N}x{Cin}->{Cout}")
 
 
 @pytest.mark.parametrize("B,H,Cin,Cout,stride", [(9, 14, 64, 128, 1), (8, 28, 32, 64, 2), (3, 7, 256, 256, 1)])
-def test_tf32x3_long_reduction_conv(dev, B, H, Cin, Cout, stride):
+def test_f32split_long_reduction_conv(dev, B, H, Cin, Cout, stride):
     G, K = 8, 2
     g = torch.Generator().manual_seed(B * 37 + H + Cin)
     X = torch.randn((B, H, H, Cin), generator=g).clamp_min(0)
@@ -793,7 +793,7 @@ def test_tf32x3_long_reduction_conv(dev, B, H, Cin, Cout, stride):
     assert torch.isfinite(Y).all()
     _, _, Wd, mask = oracle_reference(W, G, K)
     Yo, S = oracle.conv2d(f64(X), Wd, mask, 3, 3, (stride, stride), (1, 1))
-    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, f"tf32x3 conv B={B} H={H} s={stride}")
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, f"f32split conv B={B} H={H} s={stride}")
 
 
 # ---------------------------------------------------------------------------
@@ -942,22 +942,13 @@ def test_pack_stats_estimates_eq1(dev, G, Ps):
 # the same tensor-core GEMM on dense (unpruned) weights: the reference line of
 # what the sparsity buys
 # ---------------------------------------------------------------------------
-def dense_planes(W: torch.Tensor) -> torch.Tensor:
-    """The dense family's weight layout: bf16 as is; fp32 as hi / lo tf32 planes
-    (hi = the low 13 mantissa bits cleared, lo = w - hi, both exact)."""
-    if W.dtype == BF16:
-        return W.contiguous()
-    hi = (W.view(torch.int32) & -8192).view(torch.float32)
-    return torch.stack([hi, W - hi]).contiguous()
-
-
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("N,Cin,Cout", [(300, 64, 256), (129, 72, 40), (1000, 256, 1024), (2048, 512, 512)])
 def test_dense_linear_tc(dev, dtype, N, Cin, Cout):
     X, W = wl.random_small(N + Cin + 1, dtype, N, Cin, Cout)
     Y = torch.full((N, Cout), float("nan"), device=dev)
     st = cci.new_status(dev)
-    cci.dense_linear_tc(X.to(dev), dense_planes(W).to(dev), Cout, out=Y, status=st)
+    cci.dense_linear_tc(X.to(dev), cci.dense_planes(W.to(dev)), Cout, out=Y, status=st)
     assert cci.read_status(st) == 0
     Yo, S = oracle.linear(f64(X), f64(W), np.ones((Cout, Cin), dtype=bool))
     assert_within_tol(f64(Y), Yo, S, f"dense {dtype} {N}x{Cin}->{Cout}")
@@ -972,7 +963,7 @@ def test_dense_conv2d_tc(dev, case):
     X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(_dt(dtype))
     W = torch.randn((Cout, KH * KW * Cin), generator=g).to(_dt(dtype))
     st = cci.new_status(dev)
-    Y = cci.dense_conv2d_tc(X.to(dev), dense_planes(W).to(dev), Cout, KH, KW, (s, s), (p, p), status=st)
+    Y = cci.dense_conv2d_tc(X.to(dev), cci.dense_planes(W.to(dev)), Cout, KH, KW, (s, s), (p, p), status=st)
     assert cci.read_status(st) == 0
     Yo, S = oracle.conv2d(f64(X), f64(W), np.ones(W.shape, dtype=bool), KH, KW, (s, s), (p, p))
     assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, str(case))
