@@ -161,6 +161,20 @@ def test_workspace_rules(lib):
     assert lib.cci_linear_ws(FAKE, 1, 16, 16, FAKE, FAKE, 16, 8, 2, FAKE, None, ws, FAKE + 8, 4096, None) == 11
     assert cci.kernel_name(torch.bfloat16, 64, 64, 256, 8, 2, ws) == "dense_tc_ws_bf16_G8_K2"
     assert cci.kernel_name(torch.bfloat16, 8, 36, 256, 8, 2, ws) == ""  # R % 8 != 0
+    # fp32: plane 0 [Cout][R] of 4 bytes, plane 1 [Cout][ceil(R / 32) * 64] of 2 bytes
+    assert cci.workspace_size(ws, torch.float32, 256, 72) == 256 * (72 * 4 + 3 * 128)
+
+
+def test_dense_planes_rejects(lib):
+    # argument checks run before any device call
+    need = 64 * (40 * 4 + 2 * 128)
+    assert lib.cci_dense_planes(FAKE, 0, 64, 40, FAKE, need - 1, None) == 11  # CCI_ERR_WORKSPACE
+    assert lib.cci_dense_planes(FAKE, 0, 64, 40, None, need, None) == 1       # CCI_ERR_NULL
+    assert lib.cci_dense_planes(FAKE + 8, 0, 64, 40, FAKE, need, None) == 5   # CCI_ERR_ALIGN (pointer)
+    assert lib.cci_dense_planes(FAKE, 0, 64, 42, FAKE, 10**9, None) == 5      # CCI_ERR_ALIGN (R % 4)
+    assert lib.cci_dense_planes(FAKE, 1, 64, 36, FAKE, 10**9, None) == 5      # bf16: R % 8
+    assert lib.cci_dense_planes(FAKE, 0, 0, 40, FAKE, need, None) == 2        # CCI_ERR_SHAPE
+    assert lib.cci_dense_planes(FAKE, 7, 64, 40, FAKE, need, None) == 4       # CCI_ERR_DTYPE
 
 
 def test_fma_probe_rejects(lib):
