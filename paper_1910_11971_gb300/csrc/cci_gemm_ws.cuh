@@ -83,6 +83,9 @@ struct ConvBox {
     int64_t B;       // batch size
     int hrows;       // halo copies: rows of one halo buffer (a multiple of 8)
     int nh;          // halo copies: buffers in the ring (0 otherwise)
+    int resident;    // halo copies: the layer's whole weight matrix stays in the stages
+                     // (one N tile, every stage of a tile a stage of the ring): the
+                     // weights are copied for the CTA's first tile only
 };
 
 // activation tensor maps: [0] for products (2-D over X[N][Cin]); for a
@@ -120,7 +123,9 @@ struct Cfg {
     static_assert(kStage % 1024 == 0, "stages must keep the 1024-byte swizzle alignment");
     // halo copies: fewer weight stages, the rest of shared memory for a ring of
     // halo buffers whose size and count the host sets per layer (ConvBox)
-    static constexpr int kHaloStages = kBPlane <= 8192 ? 6 : (kBPlane <= 16384 ? 4 : 3);
+    // (9 stages of 8 KB: a 3x3 layer of 64 input and 64 output channels keeps its
+    // weights resident)
+    static constexpr int kHaloStages = kBPlane <= 8192 ? 9 : (kBPlane <= 16384 ? 4 : 3);
     static constexpr int kYBuf = kM * 128;  // one output staging buffer: [128 rows][32 fp32]
     // epilogue groups: warps 0-3, and warps 4-7 too when they have no producer work
     // (TMA-copied bf16 activations); two staging buffers per group
@@ -250,6 +255,45 @@ __device__ __forceinline__ void stage_f16(uint32_t d, uint64_t adesc, uint64_t b
         "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %5, pt;\n"
         "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%6];\n}\n" ::"r"(d),
         "l"(adesc), "l"(bdesc), "r"(acc0), "r"(issue), "n"(kIdesc), "r"(bar)
+        : "memory");
+}
+
+// ---- one kernel row of a 3x3 halo tile with resident weights ----
+// The three taps (kh, 0..2) of a row: A from the halo buffer at the row's first
+// tap (descriptor adesc; + 8 units, one 128-byte row, per tap), B from the
+// stages of the three taps (bdesc, + kSU units per stage); four 16-deep MMAs per
+// tap, twelve in one block from the issuing thread, no commit (resident weight
+// stages are never released).  acc0: whether the first MMA accumulates.
+template <uint32_t kIdesc, uint32_t kSU>
+__device__ __forceinline__ void row3_f16(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t acc0)
+{
+    asm volatile(
+        "{\n.reg .pred pa, pt;\n.reg .b64 ad, bd, a1, b1;\n"
+        "setp.ne.b32 pa, %3, 0;\nsetp.eq.b32 pt, 0, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %4, pa;\n"
+        "add.s64 ad, %1, 2;\nadd.s64 bd, %2, 2;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, %1, 4;\nadd.s64 bd, %2, 4;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, %1, 6;\nadd.s64 bd, %2, 6;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 a1, %1, 8;\nadd.s64 b1, %2, %5;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a1, b1, %4, pt;\n"
+        "add.s64 ad, a1, 2;\nadd.s64 bd, b1, 2;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, a1, 4;\nadd.s64 bd, b1, 4;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, a1, 6;\nadd.s64 bd, b1, 6;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 a1, %1, 16;\nadd.s64 b1, b1, %5;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], a1, b1, %4, pt;\n"
+        "add.s64 ad, a1, 2;\nadd.s64 bd, b1, 2;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, a1, 4;\nadd.s64 bd, b1, 4;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n"
+        "add.s64 ad, a1, 6;\nadd.s64 bd, b1, 6;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %4, pt;\n}\n" ::"r"(d),
+        "l"(adesc), "l"(bdesc), "r"(acc0), "n"(kIdesc), "n"(static_cast<uint64_t>(kSU))
         : "memory");
 }
 
@@ -774,6 +818,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
             const int64_t co0 = ct * kN + crank * C::kBRows;  // this CTA's B rows
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d || ASRC == kAHalo) bi = box_of(mt, box);
+            // resident weights (halo copies): only the first tile's stages are copied
+            if (C::kHalo && box.resident && it >= nks) break;
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
                 if (it % kBIssuers != issuer) continue;
                 const int s = it % kStages;
@@ -1151,9 +1197,6 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
         // the drain)
         int it = 0, t = 0;
         bool ok = CG == 1 || crank == 0;
-        // kAHalo: stage and halo-ring positions with their phase parities
-        int hs = 0, hb = 0;
-        uint32_t hsph = 0u, hph = 0u;
         const int hchunks = ASRC == kAHalo ? nks / taps : 0;
         const uint64_t hdesc0 = tc::sw128_desc(hbuf), bdesc0 = tc::sw128_desc(base);
         const uint32_t empty0 = tc::smem_u32(&S->empty[0]);
@@ -1225,6 +1268,69 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
             }
             ok = false;  // the generic loop below is not entered
         }
+        if constexpr (!TF32 && ASRC == kAHalo) {
+            // 3x3 halo tiles, chunk by chunk (halo buffer hb of the ring), the taps in
+            // turn: tap (kh, kw) reads the halo from row kh * (Q + 2) + kw on.  One
+            // thread runs the issue loop.  Resident weights: the three taps of a
+            // kernel row go out as one block of twelve MMAs, and no weight stage is
+            // released; otherwise each tap is a stage of the ring.  Descriptors in
+            // 16-byte units: + wq_units per halo row of taps, + 8 per column,
+            // + hunits per halo buffer, + sunits per stage.
+            if (lane == 0 && ok) {
+                int hs = 0, hb = 0;
+                uint32_t hsph = 0u, hph = 0u;
+                const uint64_t wq_units = static_cast<uint64_t>(box.QB + p.KW - 1) * 8u;
+                const uint64_t hunits = hbytes >> 4, sunits = C::kStage >> 4;
+                const bool res = box.resident != 0;
+                for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
+                    const int acc = t & 1;
+                    if (t >= 2) ok = tc::mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
+                    if (!ok) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
+                    if (res) hs = 0;
+                    for (int c = 0; c < hchunks && ok; ++c) {
+                        ok = tc::mbar_wait(&S->hfull[hb], hph, abort, p.status);
+                        if (!ok) break;
+                        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                        const uint64_t hdesc = hdesc0 + static_cast<uint64_t>(hb) * hunits;
+                        for (int kh = 0; kh < 3 && ok; ++kh) {
+                            const uint64_t arow = hdesc + static_cast<uint64_t>(kh) * wq_units;
+                            if (res) {
+                                if (t == 0) {  // the row's weights land once, for the first tile
+                                    for (int kw = 0; kw < 3 && ok; ++kw)
+                                        ok = tc::mbar_wait(&S->full[hs + kw], 0u, abort, p.status);
+                                    if (!ok) break;
+                                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                                }
+                                row3_f16<C::kIdesc, (C::kStage >> 4)>(d, arow, bdesc0 + static_cast<uint64_t>(hs) * sunits,
+                                                                     (c | kh) != 0 ? 1u : 0u);
+                                hs += 3;
+                            } else {
+                                for (int kw = 0; kw < 3 && ok; ++kw) {
+                                    ok = tc::mbar_wait(&S->full[hs], hsph, abort, p.status);
+                                    if (!ok) break;
+                                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                                    stage_f16<C::kIdesc>(d, arow + kw * 8u, bdesc0 + static_cast<uint64_t>(hs) * sunits,
+                                                         (c | kh | kw) != 0 ? 1u : 0u, 1u, empty0 + 8u * hs);
+                                    if (++hs == kStages) {
+                                        hs = 0;
+                                        hsph ^= 1u;
+                                    }
+                                }
+                            }
+                        }
+                        if (ok) tc::mma_commit(&S->hempty[hb]);
+                        if (++hb == box.nh) {
+                            hb = 0;
+                            hph ^= 1u;
+                        }
+                    }
+                    if (ok) commit(&S->tmem_full[acc]);
+                }
+            }
+            ok = false;  // the generic loop below is not entered
+        }
         for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
             const int acc = t & 1;
             // CG = 2: the phase includes arrivals of the odd CTA's epilogue
@@ -1232,39 +1338,6 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
             if (!ok) break;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
-            if constexpr (ASRC == kAHalo) {
-                // chunk by chunk (halo buffer hb of the ring), the taps in turn: tap
-                // (kh, kw) reads the halo from row kh * (Q + 2) + kw on.  Counters
-                // advance by increments (no division in the issue loop).
-                // descriptors in 16-byte units: + wq_units per halo row of taps,
-                // + 8 per column, + hunits per halo buffer, + sunits per stage
-                const uint64_t wq_units = static_cast<uint64_t>(box.QB + p.KW - 1) * 8u;
-                const uint64_t hunits = hbytes >> 4, sunits = C::kStage >> 4;
-                for (int c = 0; c < hchunks && ok; ++c) {
-                    ok = tc::mbar_wait(&S->hfull[hb], hph, abort, p.status);
-                    const uint64_t hdesc = hdesc0 + static_cast<uint64_t>(hb) * hunits;
-                    for (int kh = 0; kh < p.KH && ok; ++kh) {
-                        for (int kw = 0; kw < p.KW && ok; ++kw, ++it) {
-                            ok = tc::mbar_wait(&S->full[hs], hsph, abort, p.status);
-                            if (!ok) break;
-                            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                            stage_f16<C::kIdesc>(d, hdesc + static_cast<uint64_t>(kh) * wq_units + kw * 8u,
-                                                 bdesc0 + static_cast<uint64_t>(hs) * sunits,
-                                                 (c | kh | kw) != 0 ? 1u : 0u, issue, empty0 + 8u * hs);
-                            if (kh == p.KH - 1 && kw == p.KW - 1 && lane == 0) commit(&S->hempty[hb]);
-                            __syncwarp();
-                            if (++hs == kStages) {
-                                hs = 0;
-                                hsph ^= 1u;
-                            }
-                        }
-                    }
-                    if (++hb == box.nh) {
-                        hb = 0;
-                        hph ^= 1u;
-                    }
-                }
-            } else
             for (int ks = 0; ks < nks && ok; ++ks, ++it) {
                 const int s = it % kStages;
                 // PK pairs: the phase includes the odd CTA's producers (released at cluster scope)
@@ -1608,6 +1681,7 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &t
         if (!make_map(&tmY, p.Y, ydt, yel, 2, dims, bx)) return cudaErrorInvalidValue;
     }
     const int64_t n_ct = (p.Cout + C::kN - 1) / C::kN;
+    if constexpr (C::kHalo && !PK) box.resident = (n_ct == 1 && (p.R + C::kKS - 1) / C::kKS <= C::kStages) ? 1 : 0;
     const int64_t m_tiles = (ASRC == kA4d || ASRC == kAHalo)
                                 ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)
                                          : (p.N + C::kM - 1) / C::kM;
@@ -1648,13 +1722,15 @@ struct Plan {
 // chunks or more per tile: the per-tap copies there move 9 x the halo's bytes,
 // and the halo copies measured 7-11 % faster on the 14 x 14 ResNet-50 layers;
 // with 64 or 128 channels the tile is bound by the MMAs' shared-memory reads
-// and the per-tap form measured faster) whose output rows per tile are at
-// least three quarters of the 4-D box's (images narrower than the tile fit
-// several per 4-D box, not per halo)
+// and the per-tap form measured faster), and for 64 -> 64 layers, whose nine
+// weight tiles stay resident in the stages (no per-tap weight copies either),
+// whose output rows per tile are at least three quarters of the 4-D box's
+// (images narrower than the tile fit several per 4-D box, not per halo)
 inline bool halo_box(const FwdParams &p, const ConvBox &a4d, ConvBox *hb)
 {
     if (!(p.is_conv && p.KH == 3 && p.KW == 3 && p.sh == 1 && p.sw == 1 && p.ph == 1 && p.pw == 1 &&
-          p.Cin % 64 == 0 && p.Cin >= 256 && p.P == p.H && p.Q == p.W && p.Q + 2 <= 66))
+          p.Cin % 64 == 0 && (p.Cin >= 256 || (p.Cin == 64 && p.Cout <= 64)) && p.P == p.H && p.Q == p.W &&
+          p.Q + 2 <= 66))
         return false;
     const int wq = static_cast<int>(p.Q) + 2;
     const int pb = static_cast<int>(p.P < 128 / wq ? p.P : 128 / wq);

@@ -9,7 +9,7 @@ namespace tc {
 
 constexpr long long kWaitLimit = 1ll << 31;  // clock cycles (about 1 s) per bounded wait
 
-constexpr int kMaxStages = 8;
+constexpr int kMaxStages = 9;
 constexpr int kMaxHalo = 4;  // halo buffers of a 3x3 convolution tile ring
 
 // barriers and TMEM slot of a tensor-core kernel (after its 1024-byte aligned
