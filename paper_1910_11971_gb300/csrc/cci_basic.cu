@@ -135,35 +135,29 @@ __global__ void __launch_bounds__(128) pack_vec_kernel(const TB *__restrict__ W,
     // keys are distinct, a larger key is a larger |w| or an equal |w| at a lower
     // index (the tie rule; the sign ranks nothing), and a key gives back its entry
     // (value = sign and magnitude, index = 255 - the index field).  The K kept
-    // entries are the K largest keys, found by K passes of a maximum over the
-    // keys below the previous one, then put in increasing index.
+    // entries are the K largest keys, kept sorted while the G keys pass once
+    // (insertion: slot s takes the larger of itself and the smaller of slot s - 1
+    // and the key), then put in increasing index.  A NaN magnitude outranks every
+    // other key, so the column holds a NaN exactly when its largest key does.
     using Key = typename std::conditional<sizeof(TB) == 4, uint64_t, uint32_t>::type;
 #pragma unroll
     for (int v = 0; v < 4; ++v) {
-        Key key[GT];
+        Key sel[KT];
+#pragma unroll
+        for (int k = 0; k < KT; ++k) sel[k] = 0;  // every key is above 0 (its index field is not 0)
 #pragma unroll
         for (int j = 0; j < GT; ++j) {
             const uint32_t b = static_cast<uint32_t>(w[j][v]);
-            const uint32_t a = b & kAbs;
-            nan |= a > kInf;
             // the fields do not overlap: a multiply-add builds the key (FMA pipe)
-            key[j] = static_cast<Key>(a) * 512u + static_cast<Key>(((255 - j) << 1) + (b >> (kBits - 1)));
-        }
-        Key sel[KT];
-        Key t = key[0];
+            const Key key = static_cast<Key>(b & kAbs) * 512u + static_cast<Key>(((255 - j) << 1) + (b >> (kBits - 1)));
 #pragma unroll
-        for (int j = 1; j < GT; ++j) t = key[j] > t ? key[j] : t;
-        sel[0] = t;
-#pragma unroll
-        for (int k = 1; k < KT; ++k) {
-            Key m = 0;
-#pragma unroll
-            for (int j = 0; j < GT; ++j) {
-                const Key c = key[j] < t ? key[j] : 0;
-                m = c > m ? c : m;
+            for (int k = KT - 1; k > 0; --k) {
+                const Key lo = sel[k - 1] < key ? sel[k - 1] : key;
+                sel[k] = sel[k] > lo ? sel[k] : lo;
             }
-            sel[k] = t = m;
+            sel[0] = sel[0] > key ? sel[0] : key;
         }
+        nan |= (sel[0] >> 9) > kInf;
         // increasing index = decreasing inverted-index field
 #pragma unroll
         for (int a = 0; a < KT; ++a)
@@ -208,6 +202,10 @@ __global__ void __launch_bounds__(128) pack_vec_kernel(const TB *__restrict__ W,
                                                           static_cast<uint32_t>(oi[2]), static_cast<uint32_t>(oi[3]));
     }
     if (nan) report(status, CCI_ERR_VALUE);
+    // a programmatic dependent (the decompression of the product that follows)
+    // may be scheduled once every block got here; it waits for this grid's
+    // completion before reading the packed arrays
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 template <typename TB>

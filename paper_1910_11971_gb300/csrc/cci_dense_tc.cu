@@ -46,6 +46,25 @@ cudaError_t launch_wait_probe(uint32_t *status, int arrive, cudaStream_t stream)
 // ===========================================================================
 namespace dc {
 
+// a launch as a programmatic dependent of the previous kernel on the stream: it
+// may be scheduled while that kernel finishes (the kernel itself waits for it
+// with griddepcontrol.wait before touching memory)
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, cudaStream_t stream, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute la[1];
+    la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    la[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = la;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 constexpr int kSlab = 256;  // columns r per block (= threads per block)
 
 // T = uint16_t (bf16 bits) or uint32_t (fp32 bits); SPLIT: write the two operand
@@ -59,6 +78,9 @@ __global__ void __launch_bounds__(kSlab) decompress_kernel(const T *__restrict__
 {
     constexpr int V = 16 / static_cast<int>(sizeof(T));  // elements per 16-byte store
     __shared__ __align__(16) T tile[G][kSlab];
+    // launched as a programmatic dependent of the kernel before it (the pack):
+    // nothing is read or written before that grid has completed
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     // the workspace GEMM that follows may start its prologue now; it waits for
     // this grid's completion before reading the workspace
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -109,6 +131,7 @@ __global__ void __launch_bounds__(kSlab) decompress_kernel(const T *__restrict__
 template <int K>
 __global__ void __launch_bounds__(128) decompress_rows_kernel(FwdParams p, uint16_t *__restrict__ w0)
 {
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // as decompress_kernel
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) * 8;
     if (r >= p.R) return;
@@ -147,9 +170,8 @@ cudaError_t launch(const FwdParams &p, cudaStream_t stream)
             q.G = G;
             q.K = K;
             const dim3 grid(static_cast<unsigned>((p.R / 8 + 127) / 128), static_cast<unsigned>((p.Cout + 7) / 8));
-            decompress_rows_kernel<(K <= 8 ? K : 8)><<<grid, 128, 0, stream>>>(
-                q, static_cast<uint16_t *>(const_cast<void *>(p.wdense)));
-            return cudaGetLastError();
+            return launch_pdl(decompress_rows_kernel<(K <= 8 ? K : 8)>, grid, dim3(128), stream, q,
+                              static_cast<uint16_t *>(const_cast<void *>(p.wdense)));
         }
     }
     const int64_t slabs = (p.R + kSlab - 1) / kSlab;
@@ -157,9 +179,8 @@ cudaError_t launch(const FwdParams &p, cudaStream_t stream)
     if (blocks > 0x7fffffff) return cudaErrorInvalidValue;
     T *w0 = static_cast<T *>(const_cast<void *>(p.wdense));
     T *w1 = SPLIT ? w0 + p.Cout * p.R : nullptr;
-    decompress_kernel<T, G, K, SPLIT><<<static_cast<unsigned>(blocks), kSlab, 0, stream>>>(
-        static_cast<const T *>(p.values), p.idx, p.R, slabs, w0, w1, p.status);
-    return cudaGetLastError();
+    return launch_pdl(decompress_kernel<T, G, K, SPLIT>, dim3(static_cast<unsigned>(blocks)), dim3(kSlab), stream,
+                      static_cast<const T *>(p.values), p.idx, p.R, slabs, w0, w1, p.status);
 }
 
 }  // namespace dc
