@@ -101,13 +101,18 @@ struct AMaps {
 // EPI = 2: a second epilogue group (warps 4-7, idle when bf16 activations are
 // copied by TMA) and two staging buffers per group, for layers whose tiles have
 // few stages (the output write dominates); EPI = 1: one group, more stages
-template <bool TF32, int ASRC, int BN, int CG, int EPI, bool PK = false>
+template <bool TF32, int ASRC, int BN, int CG, int EPI, bool PK = false, bool MC = false>
 struct Cfg {
     static constexpr int kM = 128, kN = BN;
     static_assert(CG == 1 || (CG == 2 && !TF32 && ASRC != kAGather), "pair mode: bf16 with TMA activations");
     static_assert(!PK || (!TF32 && ASRC != kAGather && EPI == 1 && (BN / CG) <= 128),
                   "packed weights: bf16, TMA activations, producers busy, one item per producer");
     static constexpr int kBRows = kN / CG;  // B rows held by one CTA
+    // MC: a cluster of two CTAs takes adjacent M tiles of the same N tile; each
+    // copies half of the B rows of a stage with multicast into both, and each
+    // CTA's MMAs release the stage in both (fp32 with TMA activations)
+    static_assert(!MC || (TF32 && ASRC != kAGather && CG == 1 && EPI == 1 && !PK), "weight multicast: fp32 TMA tiles");
+    static constexpr bool kPairUnits = CG == 2 || MC;  // units of two M tiles over a cluster of two
     static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
     static constexpr bool kHalo = ASRC == kAHalo;  // A: per-chunk halo buffers, stages hold B only
@@ -204,7 +209,8 @@ __device__ __forceinline__ void mma(uint32_t d, uint64_t a, uint64_t b, uint32_t
 // formed by adds: the MMA warp's instruction stream per stage bounds this
 // product (measured on GB300 with clock stamps for the three-pass form of twelve
 // MMAs: operands waited for ~130 cycles per stage, the issue of a stage took ~850).
-template <uint32_t kIdescT, uint32_t kIdescB, uint32_t kB1>
+// kMC: the commit arrives on the barrier at this offset in both CTAs of the cluster.
+template <uint32_t kIdescT, uint32_t kIdescB, uint32_t kB1, bool kMC = false>
 __device__ __forceinline__ void stage_tf32_split(uint32_t d, uint32_t a0, uint64_t b0, uint32_t acc0, uint32_t issue,
                                                  uint32_t bar)
 {
@@ -225,11 +231,22 @@ __device__ __forceinline__ void stage_tf32_split(uint32_t d, uint32_t a0, uint64
         "add.u32 a, %1, 48;\nadd.s64 b, %2, %8;\n"
         "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %6, pt;\n"
         "add.u32 a, %1, 56;\nadd.s64 b, b, 2;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %6, pt;\n"
-        "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%9];\n}\n" ::"r"(d),
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], [a], b, %6, pt;\n}\n" ::"r"(d),
         "r"(a0), "l"(b0), "r"(acc0), "r"(issue), "n"(kIdescT), "n"(kIdescB),
-        "n"(static_cast<uint64_t>(kB1 + 4)), "n"(static_cast<uint64_t>(kB1)), "r"(bar)
+        "n"(static_cast<uint64_t>(kB1 + 4)), "n"(static_cast<uint64_t>(kB1))
         : "memory");
+    if constexpr (kMC)
+        asm volatile(
+            "{\n.reg .pred pe;\nsetp.ne.b32 pe, %1, 0;\n"
+            "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %2;\n}\n" ::"r"(bar),
+            "r"(issue), "h"(static_cast<uint16_t>(3))
+            : "memory");
+    else
+        asm volatile(
+            "{\n.reg .pred pe;\nsetp.ne.b32 pe, %1, 0;\n"
+            "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(bar),
+            "r"(issue)
+            : "memory");
 }
 
 // ---- one pipeline stage of bf16 MMAs ----
@@ -378,6 +395,17 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void *tmap,
         "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, "
         "{%2, %3}], [%4];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// 2-D tile copy into the same shared-memory offset of both CTAs of a cluster of
+// two, completing on the barrier at the same offset in each
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const void *tmap, int x, int y, uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster [%0], [%1, "
+        "{%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(bar), "h"(static_cast<uint16_t>(3))
         : "memory");
 }
 
@@ -679,13 +707,13 @@ __device__ __forceinline__ BoxIdx box_of(int64_t mt, const ConvBox &box)
 
 // PK: tmB0 / tmB1 are the maps of the packed values and indices (2-D over
 // [Cout/G][R*K]); otherwise the maps of the workspace planes
-template <bool TF32, int ASRC, int BN, int CG, int EPI, bool PK = false>
-__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
+template <bool TF32, int ASRC, int BN, int CG, int EPI, bool PK = false, bool MC = false>
+__global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads, 1)
     gemm_ws_kernel(FwdParams p, const __grid_constant__ AMaps tmA, const __grid_constant__ CUtensorMap tmB0,
                    const __grid_constant__ CUtensorMap tmB1, const __grid_constant__ CUtensorMap tmY, ConvBox box,
                    int64_t n_ct, int64_t n_tiles)
 {
-    using C = Cfg<TF32, ASRC, BN, CG, EPI, PK>;
+    using C = Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>;
     constexpr int kM = C::kM, kN = C::kN, kKS = C::kKS, kStages = C::kStages;
     constexpr int kLag = 2;  // bf16 gather: stages in flight before a producer's arrive
     extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -701,16 +729,16 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
     volatile int *abort = &S->abort;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nks = static_cast<int>((p.R + kKS - 1) / kKS);
-    const uint32_t crank = CG == 2 ? cluster_rank() : 0u;  // 0: issues the pair's MMAs
+    const uint32_t crank = C::kPairUnits ? cluster_rank() : 0u;  // CG = 2: 0 issues the pair's MMAs
     // work units: tiles (CG = 1) or pair tiles of 2 x 128 rows (CG = 2), strided over
     // the CTAs (CG = 1) or the CTA pairs (CG = 2)
-    const int64_t u0 = CG == 2 ? blockIdx.x / 2 : blockIdx.x;
-    const int64_t ustep = CG == 2 ? gridDim.x / 2 : gridDim.x;
+    const int64_t u0 = C::kPairUnits ? blockIdx.x / 2 : blockIdx.x;
+    const int64_t ustep = C::kPairUnits ? gridDim.x / 2 : gridDim.x;
     // unit u -> (M tile, N tile): one 64-bit division, the remainder by multiply-subtract
     auto split_unit = [&](int64_t u, int64_t &mt, int64_t &ct) {
         const int64_t q = u / n_ct;
         ct = u - q * n_ct;
-        mt = CG == 2 ? 2 * q + crank : q;
+        mt = C::kPairUnits ? 2 * q + crank : q;
     };
 
     if (tid == 0) {
@@ -721,7 +749,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
         const uint32_t full_count = PK ? (C::kHalo ? 0u : 1u) + 4 * CG : (C::kATma ? 1u : 129u);
         for (int s = 0; s < kStages; ++s) {
             tc::mbar_init(&S->full[s], full_count);
-            tc::mbar_init(&S->empty[s], 1);
+            tc::mbar_init(&S->empty[s], MC ? 2 : 1);  // MC: released by both CTAs' MMAs
             tc::mbar_init(&S->aux[s], 1);
         }
         for (int a = 0; a < 2; ++a) {
@@ -770,7 +798,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     // the pair's barriers are initialised before either CTA signals the other's
-    if constexpr (CG == 2) cluster_sync();
+    if constexpr (C::kPairUnits) cluster_sync();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = S->tmem_base;
     // launched as a programmatic dependent of the decompression: everything above
@@ -815,7 +843,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
         for (int64_t u = u0; u < n_tiles && ok; u += ustep) {
             int64_t mt, ct;
             split_unit(u, mt, ct);
-            const int64_t co0 = ct * kN + crank * C::kBRows;  // this CTA's B rows
+            const int64_t co0 = ct * kN + (CG == 2 ? crank * C::kBRows : 0);  // this CTA's B rows
             BoxIdx bi{0, 0, 0};
             if constexpr (ASRC == kA4d || ASRC == kAHalo) bi = box_of(mt, box);
             // resident weights (halo copies): only the first tile's stages are copied
@@ -870,9 +898,19 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                         tc::mbar_arrive_expect_tx(&S->full[s], a_bytes);
                     } else {
                         tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes + (C::kATma ? a_bytes : 0u));
-                        tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
-                        if constexpr (C::kBPlanes > 1)
-                            tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * 64, static_cast<int>(co0), &S->full[s]);  // plane 1: 64 bf16 per stage
+                        if constexpr (MC) {
+                            // this CTA's half of the B rows into both CTAs (the same offsets);
+                            // each CTA's full barrier expects the whole tile
+                            const uint32_t half = crank * (C::kBPlane / 2);
+                            const int y = static_cast<int>(co0) + static_cast<int>(crank) * (kN / 2);
+                            tma_load_2d_mc(bst + half, &tmB0, ks * kKS, y, tc::smem_u32(&S->full[s]));
+                            if constexpr (C::kBPlanes > 1)
+                                tma_load_2d_mc(bst + C::kBPlane + half, &tmB1, ks * 64, y, tc::smem_u32(&S->full[s]));
+                        } else {
+                            tc::tma_load_2d(bst, &tmB0, ks * kKS, static_cast<int>(co0), &S->full[s]);
+                            if constexpr (C::kBPlanes > 1)  // fp32 plane 1: 64 bf16 per stage
+                                tc::tma_load_2d(bst + C::kBPlane, &tmB1, ks * 64, static_cast<int>(co0), &S->full[s]);
+                        }
                     }
                     if constexpr (ASRC == kA2d) {
                         tc::tma_load_2d(st, &tmA.m[0], ks * kKS, static_cast<int>(mt * kM), abar);
@@ -1223,7 +1261,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
                         ok = tc::mbar_wait(&S->full[s], (it / kStages) & 1, abort, p.status);
                         if (!ok) break;
                         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                        stage_tf32_split<C::kIdesc, C::kIdescB, (C::kBPlane >> 4)>(
+                        stage_tf32_split<C::kIdesc, C::kIdescB, (C::kBPlane >> 4), MC>(
                             d, tmem + static_cast<uint32_t>(C::kAColBase + s * 64),
                             bdesc0 + static_cast<uint64_t>(s) * (C::kStage >> 4) + (C::kBOff >> 4), ks > 0 ? 1u : 0u,
                             1u, empty0 + 8u * s);
@@ -1474,7 +1512,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK>::kThreads, 1)
     __syncthreads();
     // CG = 2: neither CTA leaves (or frees tensor memory) while the other may still
     // signal its barriers or the pair's MMAs may read its shared memory
-    if constexpr (CG == 2) cluster_sync();
+    if constexpr (C::kPairUnits) cluster_sync();
     if (warp == 8) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         if constexpr (CG == 2)
@@ -1636,11 +1674,11 @@ inline int choose_bn(int64_t m_tiles, int64_t Cout, int max_bn, int cg = 1)
     return best;
 }
 
-template <bool TF32, int ASRC, int BN, int CG, int EPI = 1, bool PK = false>
+template <bool TF32, int ASRC, int BN, int CG, int EPI = 1, bool PK = false, bool MC = false>
 cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &tmA, cudaStream_t stream)
 {
-    using C = Cfg<TF32, ASRC, BN, CG, EPI, PK>;
-    auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG, EPI, PK>;
+    using C = Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>;
+    auto kern = gemm_ws_kernel<TF32, ASRC, BN, CG, EPI, PK, MC>;
     ConvBox box = box_in;
     size_t smem = C::kSmem;
     if constexpr (C::kHalo) {
@@ -1659,13 +1697,13 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &t
     const CUtensorMapDataType dt = TF32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
     const int elem = TF32 ? 4 : 2;
     const int64_t wdims[2] = {p.R, p.Cout};
-    const int wbox[2] = {C::kKS, C::kBRows};
+    const int wbox[2] = {C::kKS, MC ? C::kBRows / 2 : C::kBRows};  // MC: each CTA copies half the rows
     if (!PK && !make_map(&tmB0, p.wdense, dt, elem, 2, wdims, wbox)) return cudaErrorInvalidValue;
     if (!PK && C::kBPlanes > 1) {
         // fp32: plane 1 of the split, bf16 [Cout][ceil(R / 32) * 64], one 128-byte row per stage
         const char *pl1 = static_cast<const char *>(p.wdense) + static_cast<size_t>(p.Cout) * p.R * elem;
         const int64_t dims1[2] = {(p.R + 31) / 32 * 64, p.Cout};
-        const int box1[2] = {64, C::kBRows};
+        const int box1[2] = {64, MC ? C::kBRows / 2 : C::kBRows};
         if (!make_map(&tmB1, pl1, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, 2, dims1, box1)) return cudaErrorInvalidValue;
     }
     // output rows of 128 bytes: 32 fp32 or 64 bf16 channels
@@ -1685,10 +1723,11 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &t
     const int64_t m_tiles = (ASRC == kA4d || ASRC == kAHalo)
                                 ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)
                                          : (p.N + C::kM - 1) / C::kM;
-    // CG = 2: units are pair tiles (two M tiles), one per CTA pair
-    const int64_t n_tiles = n_ct * (CG == 2 ? (m_tiles + 1) / 2 : m_tiles);
-    const int64_t slots = sm_count() / CG;
-    const int64_t grid = CG * (n_tiles < slots ? n_tiles : slots);
+    // CG = 2 or MC: units are pair tiles (two M tiles), one per cluster of two CTAs
+    constexpr int kCl = C::kPairUnits ? 2 : 1;
+    const int64_t n_tiles = n_ct * (kCl == 2 ? (m_tiles + 1) / 2 : m_tiles);
+    const int64_t slots = sm_count() / kCl;
+    const int64_t grid = kCl * (n_tiles < slots ? n_tiles : slots);
     // programmatic dependent launch: may start once every block of the preceding
     // kernel on the stream (the decompression) has signalled; it waits for that
     // kernel's completion before reading memory
@@ -1701,11 +1740,11 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &t
     la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     la[0].val.programmaticStreamSerializationAllowed = 1;
     la[1].id = cudaLaunchAttributeClusterDimension;
-    la[1].val.clusterDim.x = CG;
+    la[1].val.clusterDim.x = kCl;
     la[1].val.clusterDim.y = 1;
     la[1].val.clusterDim.z = 1;
     cfg.attrs = la;
-    cfg.numAttrs = CG == 2 ? 2 : 1;
+    cfg.numAttrs = kCl == 2 ? 2 : 1;
     const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, p, tmA, tmB0, tmB1, tmY, box, n_ct, n_tiles);
     return e != cudaSuccess ? e : cudaGetLastError();
 }

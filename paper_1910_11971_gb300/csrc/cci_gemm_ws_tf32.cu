@@ -12,12 +12,17 @@ cudaError_t launch_gemm_ws_tf32(const FwdParams &p, cudaStream_t stream)
     plan_layer(p, true, 32, &pl);
     const int asrc = pl.asrc;
     const int bn = choose_bn(m_tiles_of(p, asrc, pl.box), p.Cout, 128);
+    // TMA-copied activations: clusters of two CTAs on adjacent M tiles share each
+    // weight tile by multicast (half the weight copies per CTA)
+#define CCI_WS_MC(A, N) \
+    if (asrc == A && bn == N) return launch_cfg<true, A, N, 1, 1, false, true>(p, pl.box, pl.am, stream);
+    CCI_WS_MC(kA2d, 64)
+    CCI_WS_MC(kA2d, 128)
+    CCI_WS_MC(kA4d, 64)
+    CCI_WS_MC(kA4d, 128)
+#undef CCI_WS_MC
 #define CCI_WS_CASE(A, N) \
     if (asrc == A && bn == N) return launch_cfg<true, A, N, 1>(p, pl.box, pl.am, stream);
-    CCI_WS_CASE(kA2d, 64)
-    CCI_WS_CASE(kA2d, 128)
-    CCI_WS_CASE(kA4d, 64)
-    CCI_WS_CASE(kA4d, 128)
     CCI_WS_CASE(kAGather, 64)
     CCI_WS_CASE(kAGather, 128)
 #undef CCI_WS_CASE
