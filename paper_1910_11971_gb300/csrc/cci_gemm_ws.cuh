@@ -110,8 +110,11 @@ struct Cfg {
     static constexpr int kBRows = kN / CG;  // B rows held by one CTA
     // MC: a cluster of two CTAs takes adjacent M tiles of the same N tile; each
     // copies half of the B rows of a stage with multicast into both, and each
-    // CTA's MMAs release the stage in both (fp32 with TMA activations)
-    static_assert(!MC || (TF32 && ASRC != kAGather && CG == 1 && EPI == 1 && !PK), "weight multicast: fp32 TMA tiles");
+    // CTA's MMAs release the stage in both (TMA activations, 2-D or 4-D)
+    static_assert(!MC || (ASRC != kAGather && ASRC != kAHalo && CG == 1 && EPI == 1 && !PK),
+                  "weight multicast: single-CTA TMA tiles with one epilogue group");
+    // (used for fp32 layers: measured on the bf16 3x3 convolutions it did not pay,
+    // conv3x3_28 0.0273 -> 0.0283 ms, the ResNet-50 stack unchanged)
     static constexpr bool kPairUnits = CG == 2 || MC;  // units of two M tiles over a cluster of two
     static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
@@ -256,7 +259,7 @@ __device__ __forceinline__ void stage_tf32_split(uint32_t d, uint32_t a0, uint64
 // one block with the descriptors precomputed: the MMA warp's own instruction
 // latency per stage bounds layers whose MMAs are short (measured on GB300: a
 // 64-wide N tile stage is 192 tensor cycles, and the issue path was 400-700).
-template <uint32_t kIdesc>
+template <uint32_t kIdesc, bool kMC = false>
 __device__ __forceinline__ void stage_f16(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t acc0, uint32_t issue,
                                           uint32_t bar)
 {
@@ -269,10 +272,22 @@ __device__ __forceinline__ void stage_f16(uint32_t d, uint64_t adesc, uint64_t b
         "add.s64 ad, %1, 4;\nadd.s64 bd, %2, 4;\n"
         "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %5, pt;\n"
         "add.s64 ad, %1, 6;\nadd.s64 bd, %2, 6;\n"
-        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %5, pt;\n"
-        "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%6];\n}\n" ::"r"(d),
-        "l"(adesc), "l"(bdesc), "r"(acc0), "r"(issue), "n"(kIdesc), "r"(bar)
+        "@pe tcgen05.mma.cta_group::1.kind::f16 [%0], ad, bd, %5, pt;\n}\n" ::"r"(d),
+        "l"(adesc), "l"(bdesc), "r"(acc0), "r"(issue), "n"(kIdesc)
         : "memory");
+    // kMC: the commit arrives on the barrier at this offset in both CTAs of the cluster
+    if constexpr (kMC)
+        asm volatile(
+            "{\n.reg .pred pe;\nsetp.ne.b32 pe, %1, 0;\n"
+            "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %2;\n}\n" ::"r"(bar),
+            "r"(issue), "h"(static_cast<uint16_t>(3))
+            : "memory");
+    else
+        asm volatile(
+            "{\n.reg .pred pe;\nsetp.ne.b32 pe, %1, 0;\n"
+            "@pe tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(bar),
+            "r"(issue)
+            : "memory");
 }
 
 // ---- one kernel row of a 3x3 halo tile with resident weights ----
@@ -1295,7 +1310,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                         if constexpr (CG == 2)
                             stage_f16_pair<C::kIdesc>(d, ad, ad + bunits, ks > 0 ? 1u : 0u, empty0 + 8u * s);
                         else
-                            stage_f16<C::kIdesc>(d, ad, ad + bunits, ks > 0 ? 1u : 0u, 1u, empty0 + 8u * s);
+                            stage_f16<C::kIdesc, MC>(d, ad, ad + bunits, ks > 0 ? 1u : 0u, 1u, empty0 + 8u * s);
                         if (++s == kStages) {
                             s = 0;
                             ph ^= 1u;
