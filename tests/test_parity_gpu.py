@@ -713,6 +713,22 @@ def test_halo_conv3x3(dev, B, H, Wi, Cin, Cout):
     assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, f"halo conv B={B} {H}x{Wi} {Cin}->{Cout}")
 
 
+# 64 -> 64 (and narrower) 3x3 layers: halo copies with the nine weight tiles
+# resident in the stages, copied for each CTA's first tile only; more tiles than
+# SMs (later tiles reuse the weights), a ragged 48-channel N tile, a ragged last
+# row block.  Every output checked.
+@pytest.mark.parametrize("B,H,Wi,Cout", [(100, 14, 14, 64), (170, 9, 9, 64), (3, 23, 31, 48)])
+def test_halo_conv3x3_resident_weights(dev, B, H, Wi, Cout):
+    Cin, G, K = 64, 8, 2
+    g = torch.Generator().manual_seed(B * 7 + H + Cout)
+    X = torch.randn((B, H, Wi, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (3, 3, (1, 1), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    Yo, S = oracle.conv2d(f64(X), Wd, mask, 3, 3, (1, 1), (1, 1))
+    assert_within_tol(f64(Y).reshape(-1, Cout), Yo, S, f"resident halo conv B={B} {H}x{Wi} 64->{Cout}")
+
+
 def test_halo_conv3x3_wide_tiles(dev):
     """Enough tiles that the 256-wide N tile wins (three stages of 32 KB beside
     the two halo buffers); sampled outputs of the first and last images."""
