@@ -136,9 +136,12 @@ struct Cfg {
     static constexpr int kHaloStages = kBPlane <= 8192 ? 9 : (kBPlane <= 16384 ? 4 : 3);
     static constexpr int kYBuf = kM * 128;  // one output staging buffer: [128 rows][32 fp32]
     // epilogue groups: warps 0-3, and warps 4-7 too when they have no producer work
-    // (TMA-copied bf16 activations); two staging buffers per group
+    // (TMA-copied bf16 activations); two staging buffers per group, four in the
+    // two-group form with N tiles up to 128 (short tiles, bound by the output
+    // write: more stores in flight, three or four stages are enough)
     static constexpr int kEG = (kATma && EPI == 2) ? 2 : 1;
-    static constexpr int kYBufs = 2 * kEG;
+    static constexpr int kYPerGroup = (kEG == 2 && BN <= 128) ? 4 : 2;
+    static constexpr int kYBufs = kYPerGroup * kEG;
     static_assert(EPI == 1 || EPI == 2, "epilogue groups");
     static constexpr int kBudget = static_cast<int>(kMaxSmemPerBlock) - 1024 - kYBufs * kYBuf - 1024;
     static constexpr int kStagesFit = (kBudget / kStage) < tc::kMaxStages ? (kBudget / kStage) : tc::kMaxStages;
@@ -1488,10 +1491,11 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                     else
                         tc::mbar_arrive(&S->tmem_empty[acc]);
                 }
-                // the group's two buffers alternate; a buffer is rewritten once the
-                // store issued from it two chunks earlier has read it
-                const uint32_t buf = ybuf + static_cast<uint32_t>(2 * eg + (chunk_no & 1)) * C::kYBuf;
-                if (etid == 0) tc::bulk_wait_read<1>();
+                // the group's buffers take the chunks in turn; a buffer is rewritten once
+                // the store issued from it kYPerGroup chunks earlier has read it
+                constexpr int kYG = C::kYPerGroup;
+                const uint32_t buf = ybuf + static_cast<uint32_t>(kYG * eg + (chunk_no % kYG)) * C::kYBuf;
+                if (etid == 0) tc::bulk_wait_read<kYG - 1>();
                 tc::named_sync(ebar, 128);
                 // halo tiles: row m = pi * (Q + 2) + qi goes to staged row pi * Q + qi
                 // (the box of the store), the two unused columns of each row nowhere
