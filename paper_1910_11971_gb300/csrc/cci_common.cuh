@@ -32,6 +32,8 @@ struct FwdParams {
     const float *bias;   // nullptr: none
     int relu;
     int out_bf16;        // Y holds bf16 (round to nearest even) instead of fp32
+    int kin;             // workspace kernels: reduction indices copied per stage (bf16
+                         // products with R < 64: R rounded up to 16; else the whole stage)
 };
 
 __device__ __forceinline__ void report(uint32_t *status, cci_status code)

@@ -11,6 +11,9 @@ cudaError_t launch_gemm_ws_bf16(const FwdParams &p, cudaStream_t stream)
     Plan pl;
     plan_layer(p, false, 64, &pl);
     const int asrc = pl.asrc;
+    // products of fewer than 64 reduction indices copy only those (stage_k_in)
+    const int kin = stage_k_in(p, false, asrc, false);
+    if (kin < 64 && !build_a_maps(p, pl.box, asrc, false, kin, &pl.am)) return cudaErrorInvalidValue;
     const int64_t m_tiles = m_tiles_of(p, asrc, pl.box);
     const int64_t nks = (p.R + 63) / 64;
     // CTA pairs (256-row tiles, B split over the pair) halve each SM's B traffic,

@@ -393,6 +393,9 @@ DENSE_SMALL = [
     (128, 64, 256, 8, 2), (1, 64, 256, 8, 2), (200, 64, 256, 8, 2), (300, 128, 512, 8, 2),
     (130, 72, 40, 4, 1), (257, 136, 96, 4, 2), (64, 64, 64, 16, 4), (515, 192, 384, 16, 8),
     (129, 80, 64, 32, 16), (100, 256, 320, 32, 4), (1000, 64, 256, 8, 4), (77, 8, 32, 16, 1),
+    # reductions shorter than one 64-deep stage: the copies and MMAs cover R rounded up to 16
+    (300, 16, 96, 8, 2), (1000, 24, 144, 8, 2), (257, 32, 16, 8, 2), (129, 40, 64, 8, 1), (64, 48, 128, 16, 4),
+    (40000, 16, 96, 8, 2),
 ]
 
 
