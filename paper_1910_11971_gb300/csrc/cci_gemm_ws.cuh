@@ -28,7 +28,9 @@
 //               (kh, kw) reads the halo from row kh * (Q + 2) + kw on: the A
 //               operand of every tap is the same buffer at a row offset (the
 //               128-byte swizzle follows the address, so any row offset works);
-//               per stage only the tap's weight tile is copied;
+//               per stage only the tap's weight tile is copied (CTA pairs: each
+//               CTA copies its own halo and half of the weight rows, both CTAs'
+//               copies completing on the even CTA's barriers);
 //     kAGather  other convolutions: the producer warps gather rows (cp.async for
 //               bf16; registers, two stages ahead, then the hi/lo split, for fp32).
 //   fp32 activations copied by TMA land raw in shared memory; the producer warps
@@ -45,9 +47,11 @@
 //               them into rows (Alg. 2's index: each pair goes to row G*i + Idx
 //               of its group), 8 rows x 8 indices per thread, and once the stage
 //               is free stores the rows into its swizzled B tile.
-// Output: fp32 Y written by TMA stores from a swizzled staging buffer (two
-// alternating 16 KB buffers of [128 rows][32 columns]), 2-D over Y[N][Cout] or,
-// for kA4d, 4-D over Y[B][P][Q][Cout] with the tile's pixel box.
+// Output: Y (fp32, or bf16 with the fused epilogue's bias and ReLU) written by
+// TMA stores from swizzled staging buffers of [128 rows][128 bytes] (two per
+// epilogue group, four in the two-group form with N tiles up to 128), 2-D over
+// Y[N][Cout] or, for kA4d and kAHalo, 4-D over Y[B][P][Q][Cout] with the tile's
+// pixel box.
 // Roles: warps 0-3 epilogue (TMEM lanes), warps 4-7 producers of the activation
 // planes that are not copied by TMA (PK: of the weight tiles, with warps
 // 9 + kIssuers .. + 3 as the second producer group), warp 8 allocates TMEM and
@@ -119,7 +123,7 @@ struct Cfg {
     static constexpr int kKS = TF32 ? 32 : 64;  // r per stage: one 128-byte row
     static constexpr bool kATma = !TF32 && ASRC != kAGather;  // A copied by TMA into its plane
     static constexpr bool kHalo = ASRC == kAHalo;  // A: per-chunk halo buffers, stages hold B only
-    static_assert(!kHalo || (!TF32 && CG == 1), "halo copies: bf16 single-CTA tiles");
+    static_assert(!kHalo || (!TF32 && (CG == 1 || !PK)), "halo copies: bf16 tiles (pairs: workspace weights)");
     // raw fp32 A by TMA; the producers split it into its two planes and write both to
     // tensor memory, where the MMAs read A (no A planes in shared memory)
     static constexpr bool kARaw = TF32 && ASRC != kAGather;
@@ -872,9 +876,17 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                     if (hc >= box.nh) ok = tc::mbar_wait(&S->hempty[hb], ((hc / box.nh) - 1) & 1, abort, p.status);
                     if (!ok) break;
                     if (lane == 0) {
-                        tc::mbar_arrive_expect_tx(&S->hfull[hb], halo_bytes);
-                        tc::tma_load_4d(hbuf + hb * hbytes, &tmA.m[0], c * 64, -p.pw, bi.pb * box.PB - p.ph,
-                                        static_cast<int>(bi.bb), &S->hfull[hb]);
+                        if constexpr (CG == 2) {
+                            // each CTA's halo (its own M tile) completes on the even CTA's
+                            // barrier, which expects both
+                            if (crank == 0) tc::mbar_arrive_expect_tx(&S->hfull[hb], 2 * halo_bytes);
+                            tma_load_4d_pair(hbuf + hb * hbytes, &tmA.m[0], c * 64, -p.pw, bi.pb * box.PB - p.ph,
+                                             static_cast<int>(bi.bb), map_to_rank(tc::smem_u32(&S->hfull[hb]), 0));
+                        } else {
+                            tc::mbar_arrive_expect_tx(&S->hfull[hb], halo_bytes);
+                            tc::tma_load_4d(hbuf + hb * hbytes, &tmA.m[0], c * 64, -p.pw, bi.pb * box.PB - p.ph,
+                                            static_cast<int>(bi.bb), &S->hfull[hb]);
+                        }
                     }
                     __syncwarp();
                 }
@@ -896,9 +908,15 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                 if constexpr (ASRC == kAHalo) {
                     const int c = ks / taps, t = ks - c * taps;  // stages: chunk by chunk, taps in turn
                     if (lane == 0) {
-                        tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes);
-                        tc::tma_load_2d(base + s * C::kStage, &tmB0, static_cast<int>(t * p.Cin) + c * 64,
-                                        static_cast<int>(ct * kN), &S->full[s]);
+                        const int x = static_cast<int>(t * p.Cin) + c * 64;
+                        if constexpr (CG == 2) {  // this CTA's half of the rows, on the even CTA's barrier
+                            if (crank == 0) tc::mbar_arrive_expect_tx(&S->full[s], 2 * C::kBBytes);
+                            tma_load_2d_pair(base + s * C::kStage, &tmB0, x, static_cast<int>(co0),
+                                             map_to_rank(tc::smem_u32(&S->full[s]), 0));
+                        } else {
+                            tc::mbar_arrive_expect_tx(&S->full[s], C::kBBytes);
+                            tc::tma_load_2d(base + s * C::kStage, &tmB0, x, static_cast<int>(ct * kN), &S->full[s]);
+                        }
                     }
                     __syncwarp();
                     continue;
@@ -1367,7 +1385,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                 const bool res = box.resident != 0;
                 for (int64_t u = u0; u < n_tiles && ok; u += ustep, ++t) {
                     const int acc = t & 1;
-                    if (t >= 2) ok = tc::mbar_wait(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
+                    // CG = 2: the phase includes arrivals of the odd CTA's epilogue
+                    if (t >= 2) ok = tc::mbar_wait<CG == 2>(&S->tmem_empty[acc], ((t / 2) - 1) & 1, abort, p.status);
                     if (!ok) break;
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint32_t d = tmem + static_cast<uint32_t>(acc * kN);
@@ -1386,16 +1405,21 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                                     if (!ok) break;
                                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                                 }
-                                row3_f16<C::kIdesc, (C::kStage >> 4)>(d, arow, bdesc0 + static_cast<uint64_t>(hs) * sunits,
-                                                                     (c | kh) != 0 ? 1u : 0u);
+                                if constexpr (CG == 1)  // (pairs never keep their weights resident)
+                                    row3_f16<C::kIdesc, (C::kStage >> 4)>(
+                                        d, arow, bdesc0 + static_cast<uint64_t>(hs) * sunits, (c | kh) != 0 ? 1u : 0u);
                                 hs += 3;
                             } else {
                                 for (int kw = 0; kw < 3 && ok; ++kw) {
                                     ok = tc::mbar_wait(&S->full[hs], hsph, abort, p.status);
                                     if (!ok) break;
                                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-                                    stage_f16<C::kIdesc>(d, arow + kw * 8u, bdesc0 + static_cast<uint64_t>(hs) * sunits,
-                                                         (c | kh | kw) != 0 ? 1u : 0u, 1u, empty0 + 8u * hs);
+                                    const uint64_t bd = bdesc0 + static_cast<uint64_t>(hs) * sunits;
+                                    const uint32_t accf = (c | kh | kw) != 0 ? 1u : 0u;
+                                    if constexpr (CG == 2)  // the pair's MMAs; the stage released in both CTAs
+                                        stage_f16_pair<C::kIdesc>(d, arow + kw * 8u, bd, accf, empty0 + 8u * hs);
+                                    else
+                                        stage_f16<C::kIdesc>(d, arow + kw * 8u, bd, accf, 1u, empty0 + 8u * hs);
                                     if (++hs == kStages) {
                                         hs = 0;
                                         hsph ^= 1u;
@@ -1403,7 +1427,7 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                                 }
                             }
                         }
-                        if (ok) tc::mma_commit(&S->hempty[hb]);
+                        if (ok) commit(&S->hempty[hb]);  // CG = 2: the halo buffer freed in both CTAs
                         if (++hb == box.nh) {
                             hb = 0;
                             hph ^= 1u;
@@ -1780,7 +1804,8 @@ cudaError_t launch_cfg(const FwdParams &p, const ConvBox &box_in, const AMaps &t
         if (!make_map(&tmY, p.Y, ydt, yel, 2, dims, bx)) return cudaErrorInvalidValue;
     }
     const int64_t n_ct = (p.Cout + C::kN - 1) / C::kN;
-    if constexpr (C::kHalo && !PK) box.resident = (n_ct == 1 && (p.R + C::kKS - 1) / C::kKS <= C::kStages) ? 1 : 0;
+    if constexpr (C::kHalo && !PK && CG == 1)  // resident weights: single-CTA tiles
+        box.resident = (n_ct == 1 && (p.R + C::kKS - 1) / C::kKS <= C::kStages) ? 1 : 0;
     const int64_t m_tiles = (ASRC == kA4d || ASRC == kAHalo)
                                 ? static_cast<int64_t>(box.nQ) * box.nP * ((box.B + box.BB - 1) / box.BB)
                                          : (p.N + C::kM - 1) / C::kM;

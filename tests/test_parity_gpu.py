@@ -751,6 +751,23 @@ def test_halo_conv3x3_wide_tiles(dev):
         assert_within_tol(Yg, Yo, S, f"halo conv wide tiles image {b}")
 
 
+def test_halo_conv3x3_pair_tiles_odd_row_blocks(dev):
+    """Halo copies over CTA pairs (256 input channels, the 256-wide N tile wins the
+    pair count): 77 images of 9 x 9 are 77 row blocks, so the last pair's odd CTA
+    has none (its halo copy and output store fall wholly outside the batch).
+    Every output of the first, a middle and the last two images checked."""
+    B, H, Cin, Cout, G, K = 77, 9, 256, 256, 8, 2
+    g = torch.Generator().manual_seed(777)
+    X = torch.randn((B, H, H, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (3, 3, (1, 1), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    for b in (0, 38, B - 2, B - 1):
+        Yo, S = oracle.conv2d(f64(X[b:b + 1]), Wd, mask, 3, 3, (1, 1), (1, 1))
+        assert_within_tol(f64(Y[b]).reshape(-1, Cout), Yo, S, f"halo pair conv image {b}")
+
+
 # ---------------------------------------------------------------------------
 # CTA-pair tiles (tcgen05 cta_group::2): bf16 layers with at least 16 stages of
 # 64 reduction indices and 256-wide N tiles run as 256-row tiles split over two
