@@ -912,6 +912,26 @@ def test_fused_pair_tiles(dev):
     assert_fused_within_tol(f64(Y[torch.from_numpy(rows).to(dev)]), Yr, Sr, True, "fused pair")
 
 
+def test_fused_halo_pair_tiles(dev):
+    """Bias, ReLU and bf16 output on halo copies over CTA pairs (256 input
+    channels, two 256-wide N tiles), through the workspace family; every output of
+    the first and last images."""
+    B, H, Cin, Cout, G, K = 64, 14, 256, 512, 8, 2
+    g = torch.Generator().manual_seed(5150)
+    X = torch.randn((B, H, H, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin), generator=g).to(BF16)
+    b = _bias(Cout, 7)
+    v, i = cci.pack(W.to(dev), G, K)
+    ws = cci.new_workspace(cci.ALGO_DENSE_TC_WS, BF16, Cout, 9 * Cin, dev)
+    Y = cci.conv2d_fused(X.to(dev), v, i, Cout, G, K, 3, 3, (1, 1), (1, 1), bias=b.to(dev), relu=True,
+                         out_dtype=BF16, workspace=ws)
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    for img in (0, B - 1):
+        Yo, S = oracle.conv2d(f64(X[img:img + 1]), Wd, mask, 3, 3, (1, 1), (1, 1))
+        Yr, Sr = oracle.epilogue(Yo, S, f64(b), True)
+        assert_fused_within_tol(f64(Y[img]).reshape(-1, Cout), Yr, Sr, True, f"fused halo pair image {img}")
+
+
 def test_fused_identity_equals_plain_product(dev):
     """No bias, no ReLU, fp32 output: bit for bit the plain product of the family
     AUTO picks (the binding passes both calls the workspace AUTO asks for), and,
