@@ -768,6 +768,24 @@ def test_halo_conv3x3_pair_tiles_odd_row_blocks(dev):
         assert_within_tol(f64(Y[b]).reshape(-1, Cout), Yo, S, f"halo pair conv image {b}")
 
 
+def test_halo_conv3x3_pair_tiles_ragged(dev):
+    """Halo copies over CTA pairs with a ragged N tile (320 = 256 + 64 output
+    channels, the second pair's tile three quarters out of range) and five
+    64-channel chunks per tile (the ring of halo buffers wraps within and across
+    tiles); 38 images of 14 x 14 make 38 pair units, where the 256-wide tile ties
+    the 64-wide one in the pair count.  Every output of four images checked."""
+    B, H, Cin, Cout, G, K = 38, 14, 320, 320, 8, 2
+    g = torch.Generator().manual_seed(3838)
+    X = torch.randn((B, H, H, Cin), generator=g).clamp_min(0).to(BF16)
+    W = torch.randn((Cout, 9 * Cin), generator=g).to(BF16)
+    Y = run_conv(dev, X, W, (3, 3, (1, 1), (1, 1), Cout), G, K, cci.ALGO_DENSE_TC_WS)
+    assert torch.isfinite(Y).all()
+    _, _, Wd, mask = oracle_reference(W, G, K)
+    for b in (0, 17, B - 2, B - 1):
+        Yo, S = oracle.conv2d(f64(X[b:b + 1]), Wd, mask, 3, 3, (1, 1), (1, 1))
+        assert_within_tol(f64(Y[b]).reshape(-1, Cout), Yo, S, f"ragged halo pair conv image {b}")
+
+
 # ---------------------------------------------------------------------------
 # CTA-pair tiles (tcgen05 cta_group::2): bf16 layers with at least 16 stages of
 # 64 reduction indices and 256-wide N tiles run as 256-row tiles split over two
