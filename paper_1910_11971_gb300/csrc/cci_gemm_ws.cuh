@@ -1520,6 +1520,10 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
             for (int c0 = 0; c0 < cend; c0 += sc, ++chunk_no) {
                 uint32_t v[32];
                 const uint32_t tcol = tmem + lane_off + static_cast<uint32_t>(acc * kN + c0);
+                // output columns of this chunk inside the layer (the store clips the rest):
+                // the 16-byte pieces of each staged row that need writing
+                const int valid = (cend - c0) < sc ? cend - c0 : sc;
+                const int nq = p.out_bf16 ? (valid + 7) / 8 : (valid + 3) / 4;
                 if (!p.out_bf16) {
                     tc::tmem_ld32(tcol, v);
                     epilogue_math(v, p, co0 + c0);
@@ -1529,10 +1533,12 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                     epilogue_math(w, p, co0 + c0);
 #pragma unroll
                     for (int j = 0; j < 16; ++j) v[j] = bf16x2_rn(w[2 * j], w[2 * j + 1]);
-                    tc::tmem_ld32(tcol + 32, w);
-                    epilogue_math(w, p, co0 + c0 + 32);
+                    if (valid > 32) {  // the second 32 columns (a narrower last chunk has none)
+                        tc::tmem_ld32(tcol + 32, w);
+                        epilogue_math(w, p, co0 + c0 + 32);
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) v[16 + j] = bf16x2_rn(w[2 * j], w[2 * j + 1]);
+                        for (int j = 0; j < 16; ++j) v[16 + j] = bf16x2_rn(w[2 * j], w[2 * j + 1]);
+                    }
                 }
                 if (c0 + sc >= cend) {
                     // the tile's accumulator is all in registers: release it to the MMAs
@@ -1561,7 +1567,8 @@ __global__ void __launch_bounds__(Cfg<TF32, ASRC, BN, CG, EPI, PK, MC>::kThreads
                 if (stage_row) {
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
-                        st_shared_v4(buf + sw_chunk(srow, q), v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                        if (q < nq)
+                            st_shared_v4(buf + sw_chunk(srow, q), v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
                 }
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 tc::named_sync(ebar, 128);

@@ -863,6 +863,11 @@ FUSED_PRODUCTS = [
     (1000, 128, 136, 8, 2, "bf16", False, True, "bf16"),
     (517, 96, 128, 16, 4, "f32", True, True, "bf16"),
     (129, 256, 1024, 8, 2, "f32", True, False, "f32"),
+    # narrow last chunks: 16, 24 and 88 (= 64 + 24) bf16 output channels, 20 fp32 ones
+    (2000, 32, 16, 8, 2, "bf16", True, True, "bf16"),
+    (1000, 64, 24, 8, 2, "bf16", True, False, "bf16"),
+    (700, 128, 88, 8, 2, "bf16", False, True, "bf16"),
+    (900, 64, 20, 4, 2, "bf16", True, True, "f32"),
 ]
 
 
